@@ -1,0 +1,9 @@
+"""Oracle for the GMC / GMC+ step -- test infrastructure only.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU baseline
+(and its reference arm) may import this package. See ``gmc_oracle`` for what it
+computes and which passages of the paper each part follows.
+"""
+from .gmc_oracle import (GMC, RBGS, TOPK, below, floyd_blocks, magnitude_key,  # noqa: F401
+                         rbgs_draw, rbgs_stream_key, rbgs_support, splitmix64_mix,
+                         splitmix64_sequence, top_s_support, topk_count)

@@ -1,0 +1,287 @@
+"""GMC / GMC+ oracle: a plain, slow, CPU statement of the paper's update rules.
+
+TEST INFRASTRUCTURE. Only the tests, ``__graft_entry__.smoke()`` and the CPU
+baseline / reference arm of ``bench.py`` may import this module. The product
+path (the CUDA library and its Python binding) never imports it and shares no
+code with it.
+
+What it follows (Shi et al., "Global Momentum Compression for Sparse
+Communication in Distributed Learning", arXiv 1905.12948):
+  * Algorithm 1 (GMC), Sec. 3.1: w_{-1} = w_0, e_{0,k} = 0;
+        e_{t+1/2,k} = e_{t,k} + g_{t,k} - (beta/eta) (w_t - w_{t-1})
+        e_{t+1,k}   = e_{t+1/2,k} - C(e_{t+1/2,k})
+        w_{t+1}     = w_t - (eta/K) sum_k C(e_{t+1/2,k})
+  * Algorithm 2 (GMC+), Sec. 4: the same step plus the detach
+        w_{t+1,k}   = w_{t+1} - lambda*eta*e_{t+1,k},   w_{0,k} = w_0.
+    Gradients are inputs here, so the detached points are an output only.
+  * Compressors (Sec. 4): top-s (the s components of largest magnitude) and
+    RBGS (random blocks chosen with one seed shared by all workers, Sec. 5.2).
+  * Relative communication cost (Sec. 5, RCC), halved for RBGS (Sec. 5.2).
+
+Precision. The paper fixes none. Top-s turns floating-point magnitudes into an
+integer decision (which indices are sent), so that decision is taken in the
+kernel's precision, fp32; every later state depends on those decisions, so the
+whole state (w, w_{t-1}, e) is fp32. Each elementary operation is one IEEE-754
+round-to-nearest-even fp32 operation, evaluated in the order the algorithm
+writes it: e_{t+1/2} = ((e + g) - (c * (w_t - w_{t-1}))) with c = fl(beta/eta);
+the aggregate sums the workers' values in ascending worker order starting from
++0; w_{t+1} = w_t - (a * sum) with a = fl(eta/K); the detach is
+w - (b * e) with b = fl(lambda*eta). numpy float32 ufuncs round each operation
+once and never fuse a multiply into an add, which is exactly that.
+
+Readings where the paper is silent:
+  * top-s ties: the lower index wins; magnitudes compare through the IEEE bit
+    pattern with the sign cleared, so +0 and -0 tie;
+  * s = max(1, floor(ratio * d)) for a compression ratio;
+  * RBGS: d is cut into aligned blocks of B (the last one may be short),
+    m = max(1, floor(ratio * nb)) distinct blocks are drawn with Floyd's
+    sampling (Bentley & Floyd, CACM 1987) from a SplitMix64 counter stream
+    (Steele, Lea & Flood, OOPSLA 2014) keyed by (seed, t) -- or (seed, t, k)
+    in the per-worker mode -- with multiply-shift range reduction;
+  * the residual at a sent coordinate is +0 exactly (v - v for finite v).
+"""
+from __future__ import annotations
+
+import math
+from typing import List, Optional
+
+import numpy as np
+
+F32 = np.float32
+U32 = np.uint32
+
+TOPK = "topk"
+RBGS = "rbgs"
+
+# ---------------------------------------------------------------------------
+# Compressors
+# ---------------------------------------------------------------------------
+
+
+def magnitude_key(x: np.ndarray) -> np.ndarray:
+    """|x| as an unsigned integer that orders like |x|: the fp32 bit pattern
+    with the sign bit cleared (monotone for non-negative floats)."""
+    return np.ascontiguousarray(x, F32).view(U32) & U32(0x7FFFFFFF)
+
+
+def topk_count(d: int, ratio: float) -> int:
+    """s = max(1, floor(ratio * d)), the number of components top-s keeps."""
+    return max(1, math.floor(ratio * d))
+
+
+def top_s_support(x: np.ndarray, s: int) -> np.ndarray:
+    """Support of the top-s compressor (Sec. 4): the s components of largest
+    |x|, ties going to the lower index. Returned in ascending index order.
+
+    Written from the definition: let kth be the s-th largest magnitude key;
+    every component above kth is kept, then the lowest-index components equal
+    to kth until s are kept.
+    """
+    d = x.size
+    if not 1 <= s <= d:
+        raise ValueError("s must be in [1, d]")
+    key = magnitude_key(x)
+    kth = np.partition(key, d - s)[d - s]
+    above = np.flatnonzero(key > kth)
+    ties = np.flatnonzero(key == kth)[: s - above.size]
+    return np.sort(np.concatenate([above, ties]))
+
+
+GOLDEN_GAMMA = 0x9E3779B97F4A7C15
+_M64 = (1 << 64) - 1
+
+
+def splitmix64_mix(z: int) -> int:
+    """SplitMix64 output function (Steele, Lea & Flood 2014): two
+    xor-shift-multiply rounds and a final xor-shift on a 64-bit word."""
+    z &= _M64
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _M64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _M64
+    return z ^ (z >> 31)
+
+
+def splitmix64_sequence(seed: int, n: int) -> List[int]:
+    """The first n outputs of a SplitMix64 generator whose state starts at
+    ``seed``: the state advances by the golden gamma, then is mixed."""
+    out, state = [], seed & _M64
+    for _ in range(n):
+        state = (state + GOLDEN_GAMMA) & _M64
+        out.append(splitmix64_mix(state))
+    return out
+
+
+def rbgs_stream_key(seed: int, t: int, stream: int) -> int:
+    """Key of the block-choice stream of step t. ``stream`` is 0 when all
+    workers share the choice (the paper's setting) and k+1 for worker k in the
+    per-worker mode."""
+    k1 = splitmix64_mix((seed + GOLDEN_GAMMA * (t + 1)) & _M64)
+    return splitmix64_mix((k1 + GOLDEN_GAMMA * (stream + 1)) & _M64)
+
+
+def rbgs_draw(key: int, i: int) -> int:
+    """The i-th 64-bit draw of a stream: SplitMix64 in counter form."""
+    return splitmix64_mix((key + GOLDEN_GAMMA * (i + 1)) & _M64)
+
+
+def below(x: int, n: int) -> int:
+    """Map a 64-bit draw to [0, n) by multiply-shift on its top 32 bits."""
+    return ((x >> 32) * n) >> 32
+
+
+def floyd_blocks(key: int, nb: int, m: int) -> np.ndarray:
+    """m distinct block ids out of [0, nb), Floyd's sampling without
+    replacement, returned sorted ascending."""
+    chosen = set()
+    for i, j in enumerate(range(nb - m, nb)):
+        r = below(rbgs_draw(key, i), j + 1)
+        chosen.add(j if r in chosen else r)
+    return np.array(sorted(chosen), np.int64)
+
+
+def rbgs_support(blocks: np.ndarray, B: int, d: int) -> np.ndarray:
+    """Coordinates covered by the chosen blocks, ascending."""
+    if blocks.size == 0:
+        return np.zeros(0, np.int64)
+    return np.concatenate([np.arange(b * B, min((b + 1) * B, d)) for b in blocks])
+
+
+# ---------------------------------------------------------------------------
+# GMC / GMC+ state and step
+# ---------------------------------------------------------------------------
+
+
+class StepResult:
+    """What one step produced (kept for the tests)."""
+
+    def __init__(self, e_half, supports, values, w_next, blocks, stats):
+        self.e_half = e_half          # e_{t+1/2,k}, float32 [K, d]
+        self.supports = supports      # list of K int64 index arrays (ascending)
+        self.values = values          # list of K float32 arrays: C(e_{t+1/2,k}) on its support
+        self.w_next = w_next          # w_{t+1}
+        self.blocks = blocks          # RBGS: list of chosen block arrays (per stream), else None
+        self.stats = stats            # dict of per-step counters
+
+
+class GMC:
+    """Algorithm 1 (GMC) and Algorithm 2 (GMC+) for K workers, dense arrays."""
+
+    def __init__(self, d: int, K: int, beta: float, eta: float, compressor: str = TOPK,
+                 ratio: float = 0.01, block: int = 4096, lam: float = 0.0, seed: int = 0,
+                 per_worker: bool = False):
+        if d < 1 or K < 1:
+            raise ValueError("d and K must be >= 1")
+        if not 0.0 <= beta < 1.0:
+            raise ValueError("beta must be in [0, 1)")
+        if not eta > 0.0:
+            raise ValueError("eta must be > 0")
+        if not 0.0 < ratio <= 1.0:
+            raise ValueError("ratio must be in (0, 1]")
+        if compressor not in (TOPK, RBGS):
+            raise ValueError("unknown compressor")
+        self.d, self.K = d, K
+        self.beta = F32(beta)
+        self.lam = F32(lam)
+        self.compressor = compressor
+        self.ratio = ratio
+        self.seed = seed
+        self.per_worker = per_worker
+        if compressor == TOPK:
+            self.s = topk_count(d, ratio)
+        else:
+            if block < 1:
+                raise ValueError("block must be >= 1")
+            self.B = block
+            self.nb = -(-d // block)
+            self.m = max(1, math.floor(ratio * self.nb))
+        self.set_eta(eta)
+        self.w = None
+
+    def set_eta(self, eta: float) -> None:
+        """Constants of the step, each one fp32 rounding of the paper's ratio."""
+        self.eta = F32(eta)
+        self.c = F32(self.beta / self.eta)          # beta / eta
+        self.a = F32(self.eta / F32(self.K))        # eta / K
+        self.b = F32(self.lam * self.eta)           # lambda * eta
+
+    def set_params(self, w0: np.ndarray) -> None:
+        """Initial state: w_{-1} = w_0 and e_{0,k} = 0 (Alg. 1 and Alg. 2)."""
+        w0 = np.asarray(w0, F32)
+        if w0.shape != (self.d,):
+            raise ValueError("w0 must have shape (d,)")
+        self.w = w0.copy()
+        self.w_prev = w0.copy()
+        self.e = np.zeros((self.K, self.d), F32)
+        self.t = 0
+        self.totals = dict(steps=0, pairs=0, nnz=0, union=0, changed=0)
+
+    # -- compressor support for worker k at the current step -----------------
+    def _blocks(self) -> List[np.ndarray]:
+        streams = range(1, self.K + 1) if self.per_worker else [0]
+        return [floyd_blocks(rbgs_stream_key(self.seed, self.t, s), self.nb, self.m)
+                for s in streams]
+
+    def step(self, grads: np.ndarray) -> StepResult:
+        """One iteration t of Algorithm 1 / 2 with g_{t,k} = grads[k]."""
+        if self.w is None:
+            raise RuntimeError("set_params first")
+        g = np.asarray(grads, F32)
+        if g.shape != (self.K, self.d):
+            raise ValueError("grads must have shape (K, d)")
+        K = self.K
+
+        # workers: e_{t+1/2,k} = e_{t,k} + g_{t,k} - (beta/eta)(w_t - w_{t-1})
+        momentum = self.c * (self.w - self.w_prev)
+        e_half = (self.e + g) - momentum
+
+        # workers: C(e_{t+1/2,k}) -- its support and values
+        blocks = None
+        if self.compressor == TOPK:
+            supports = [top_s_support(e_half[k], self.s) for k in range(K)]
+        else:
+            blocks = self._blocks()
+            per_stream = [rbgs_support(b, self.B, self.d) for b in blocks]
+            supports = [per_stream[k if self.per_worker else 0] for k in range(K)]
+        values = [e_half[k, supports[k]].copy() for k in range(K)]
+
+        # workers: e_{t+1,k} = e_{t+1/2,k} - C(e_{t+1/2,k})
+        e_next = e_half.copy()
+        for k in range(K):
+            e_next[k, supports[k]] = F32(0.0)
+
+        # server: w_{t+1} = w_t - (eta/K) sum_k C(e_{t+1/2,k}), workers summed in order
+        total = np.zeros(self.d, F32)
+        for k in range(K):
+            total[supports[k]] = total[supports[k]] + values[k]
+        w_next = self.w - self.a * total
+
+        in_union = np.zeros(self.d, bool)
+        for k in range(K):
+            in_union[supports[k]] = True
+        stats = dict(
+            pairs=int(sum(s.size for s in supports)),
+            nnz=int(sum(np.count_nonzero(v) for v in values)),
+            union=int(np.count_nonzero(in_union)),
+            changed=int(np.count_nonzero(w_next - self.w)),
+        )
+        for key, val in stats.items():
+            self.totals[key] += val
+        self.totals["steps"] += 1
+
+        self.w_prev, self.w, self.e = self.w, w_next, e_next
+        self.t += 1
+        return StepResult(e_half, supports, values, w_next, blocks, stats)
+
+    def worker_params(self, k: int) -> np.ndarray:
+        """GMC+ detached point of worker k: w_{t,k} = w_t - lambda*eta*e_{t,k}."""
+        return self.w - self.b * self.e[k]
+
+    def rcc(self) -> float:
+        """Relative communication cost over the steps so far (Sec. 5):
+        (1/(d K T)) sum_t (K ||w_{t+1}-w_t||_0 + sum_k ||C_k||_0), halved for
+        RBGS, whose messages carry no indices (Sec. 5.2)."""
+        T = self.totals["steps"]
+        if T == 0:
+            return 0.0
+        num = self.K * self.totals["changed"] + self.totals["nnz"]
+        r = num / (self.d * self.K * T)
+        return r / 2 if self.compressor == RBGS else r

@@ -1,0 +1,447 @@
+"""Pins of the oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle (oracle/gmc_oracle.py) against something other
+than itself: a reduction to a textbook method in float64, a closed form, an
+identity the paper derives (Sec. 3.3 update rule, Lemma 1, the GMC+ mean-iterate
+recursion of Sec. 4), brute force on tiny inputs, published generator outputs
+or a value the paper prints. Together they are chosen so that a dropped term,
+a wrong sign or coefficient, a wrong index or a transposed operand in the oracle
+fails at least one of them.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import GMC, RBGS, TOPK
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+U = 2.0 ** -24  # unit roundoff of fp32
+
+
+def _golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _grads(rng, T, K, d, scale=1.0):
+    return [(rng.standard_normal((K, d)) * scale).astype(np.float32) for _ in range(T)]
+
+
+# ---------------------------------------------------------------------------
+# P1: beta = 0 and no compression -> distributed SGD (Sec. 2.3, Sec. 3.3)
+# ---------------------------------------------------------------------------
+
+def test_p1_sgd_reduction():
+    rng = np.random.default_rng(1)
+    d, K, T, eta = 257, 3, 20, 0.1
+    o = GMC(d, K, beta=0.0, eta=eta, compressor=TOPK, ratio=1.0)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    o.set_params(w0)
+    grads = _grads(rng, T, K, d)
+    w_ref = w0.astype(np.float64)
+    tol = np.zeros(d)
+    eta32 = float(np.float32(eta))
+    for g in grads:
+        o.step(g)
+        assert not np.any(o.e), "with no compression the residual must stay exactly 0"
+        g64 = g.astype(np.float64)
+        w_ref = w_ref - eta32 / K * g64.sum(0)
+        tol += (K + 3) * U * eta32 / K * np.abs(g64).sum(0) + 2 * U * np.abs(o.w)
+        np.testing.assert_array_less(np.abs(o.w - w_ref), 2 * tol + 1e-30)
+
+
+# ---------------------------------------------------------------------------
+# P2: no compression, beta > 0 -> heavy-ball MSGD (Sec. 2.3, eq. (2))
+# ---------------------------------------------------------------------------
+
+def _heavy_ball(w0, grads, eta, beta):
+    """w_{t+1} = w_t - eta*mean_k g_{t,k} + beta*(w_t - w_{t-1}), w_{-1} = w_0, in float64."""
+    w_prev, w = w0.copy(), w0.copy()
+    out = [w.copy()]
+    for g in grads:
+        w_next = w - eta * g.mean(0) + beta * (w - w_prev)
+        w_prev, w = w, w_next
+        out.append(w.copy())
+    return out
+
+
+def test_p2_heavy_ball_closed_form():
+    """The float64 recursion itself against the textbook closed form for a
+    constant gradient: w_t = w_0 - eta*g/(1-beta) * [t - beta(1-beta^t)/(1-beta)]."""
+    eta, beta, T = 0.05, 0.9, 60
+    g = np.array([[0.3, -1.2, 2.0]])
+    w0 = np.array([1.0, -2.0, 0.5])
+    traj = _heavy_ball(w0, [g] * T, eta, beta)
+    for t in range(T + 1):
+        closed = w0 - eta * g[0] / (1 - beta) * (t - beta * (1 - beta ** t) / (1 - beta))
+        np.testing.assert_allclose(traj[t], closed, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("K", [1, 4])
+def test_p2_heavy_ball_reduction(K):
+    rng = np.random.default_rng(2 + K)
+    d, T, eta, beta = 129, 40, 0.05, 0.9
+    o = GMC(d, K, beta=beta, eta=eta, compressor=TOPK, ratio=1.0)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    o.set_params(w0)
+    grads = _grads(rng, T, K, d)
+    eta32, beta32 = float(np.float32(eta)), float(np.float32(beta))
+    ref = _heavy_ball(w0.astype(np.float64), [g.astype(np.float64) for g in grads], eta32, beta32)
+    budget = np.zeros(d)
+    w_prev = w0.astype(np.float64)
+    for t, g in enumerate(grads):
+        w_t = o.w.astype(np.float64)
+        o.step(g)
+        assert not np.any(o.e)
+        w_next = o.w.astype(np.float64)
+        dlt = np.abs(w_t - w_prev)
+        local = 6 * U * (np.abs(w_next) + np.abs(w_t) + (K + 3) * eta32 / K *
+                         (np.abs(g.astype(np.float64)).sum(0) + K * beta32 / eta32 * dlt) + beta32 * dlt)
+        budget += local
+        err = np.abs(w_next - ref[t + 1])
+        np.testing.assert_array_less(err, 2 * budget / (1 - beta32) + 1e-30)
+        w_prev = w_t
+
+
+def test_p2_constant_gradient_against_closed_form():
+    """The fp32 oracle (ratio = 1, K workers with the same constant gradient)
+    tracks the closed form of P2 to fp32 accuracy."""
+    d, K, T, eta, beta = 5, 2, 50, 0.05, 0.9
+    g = np.array([0.3, -1.2, 2.0, 0.0, 1e-3], np.float32)
+    w0 = np.array([1.0, -2.0, 0.5, 3.0, 0.0], np.float32)
+    o = GMC(d, K, beta=beta, eta=eta, compressor=TOPK, ratio=1.0)
+    o.set_params(w0)
+    eta64, beta64 = float(np.float32(eta)), float(np.float32(beta))
+    for t in range(1, T + 1):
+        o.step(np.stack([g] * K))
+        closed = w0 - eta64 * g / (1 - beta64) * (t - beta64 * (1 - beta64 ** t) / (1 - beta64))
+        np.testing.assert_allclose(o.w, closed, rtol=2e-5, atol=2e-6)
+
+
+# ---------------------------------------------------------------------------
+# P3: C(v) + e = v exactly, for every worker, coordinate and step (Alg. 1)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("compressor", [TOPK, RBGS])
+def test_p3_exact_split(compressor):
+    rng = np.random.default_rng(3)
+    d, K, T = 1000, 4, 12
+    o = GMC(d, K, beta=0.9, eta=0.1, compressor=compressor, ratio=0.05, block=64, seed=5,
+            per_worker=True)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    for g in _grads(rng, T, K, d):
+        r = o.step(g)
+        for k in range(K):
+            S = r.supports[k]
+            sel = np.zeros(d, bool)
+            sel[S] = True
+            vbits = r.e_half[k].view(np.uint32)
+            ebits = o.e[k].view(np.uint32)
+            assert np.all(ebits[sel] == 0), "sent coordinates leave +0 behind"
+            assert np.all(ebits[~sel] == vbits[~sel]), "unsent coordinates keep v bitwise"
+            assert np.all(r.values[k].view(np.uint32) == vbits[S]), "C(v) carries v bitwise"
+            np.testing.assert_array_equal(S, np.sort(S))
+
+
+# ---------------------------------------------------------------------------
+# P4: top-s by brute force on tiny inputs, ties and signed zeros included
+# ---------------------------------------------------------------------------
+
+def _brute_top_s(x, s):
+    order = sorted(range(x.size), key=lambda j: (-abs(float(x[j])), j))
+    return np.array(sorted(order[:s]), np.int64)
+
+
+def _tiny_inputs(rng, n_cases):
+    kinds = ["normal", "small_set", "all_equal", "zeros", "signed_zero", "wide"]
+    for case in range(n_cases):
+        d = int(rng.integers(1, 257))
+        kind = kinds[case % len(kinds)]
+        if kind == "normal":
+            x = rng.standard_normal(d)
+        elif kind == "small_set":
+            x = rng.choice([-2.0, -1.0, -0.0, 0.0, 1.0, 2.0], size=d)
+        elif kind == "all_equal":
+            x = np.full(d, rng.choice([-3.5, 0.25, 7.0]))
+        elif kind == "zeros":
+            x = np.zeros(d)
+        elif kind == "signed_zero":
+            x = rng.choice([-0.0, 0.0, 1e-45, -1e-45, 1.0], size=d)
+        else:
+            x = rng.standard_normal(d) * np.exp(rng.uniform(-80, 80, size=d))
+        s = int(rng.integers(1, d + 1))
+        yield x.astype(np.float32), s
+
+
+def test_p4_top_s_brute_force():
+    rng = np.random.default_rng(4)
+    for x, s in _tiny_inputs(rng, 10_000):
+        got = oracle.top_s_support(x, s)
+        np.testing.assert_array_equal(got, _brute_top_s(x, s))
+
+
+def test_p4_top_s_properties():
+    """min kept |x| >= max dropped |x|, and the delta-approximate bound of
+    Assumption 1 with delta = s/d holds deterministically for top-s."""
+    rng = np.random.default_rng(44)
+    for x, s in _tiny_inputs(rng, 2_000):
+        S = oracle.top_s_support(x, s)
+        keep = np.zeros(x.size, bool)
+        keep[S] = True
+        a = np.abs(x.astype(np.float64))
+        if keep.all():
+            continue
+        assert a[keep].min() >= a[~keep].max()
+        cx = np.where(keep, x.astype(np.float64), 0.0)
+        lhs = np.sum((cx - x) ** 2)
+        assert lhs <= (1 - s / x.size) * np.sum(x.astype(np.float64) ** 2) * (1 + 1e-12) + 1e-300
+
+
+def test_magnitude_key_orders_like_abs():
+    rng = np.random.default_rng(45)
+    x = np.concatenate([rng.standard_normal(500) * np.exp(rng.uniform(-85, 85, 500)),
+                        [0.0, -0.0, 1e-45, -1e-45, np.inf, -np.inf, 3.0e38]]).astype(np.float32)
+    key = oracle.magnitude_key(x)
+    a = np.abs(x.astype(np.float64))
+    for i, j in itertools.combinations(range(x.size), 2):
+        assert (key[i] < key[j]) == (a[i] < a[j])
+        assert (key[i] == key[j]) == (a[i] == a[j])
+
+
+def test_full_ratio_is_identity():
+    x = np.random.default_rng(46).standard_normal(77).astype(np.float32)
+    np.testing.assert_array_equal(oracle.top_s_support(x, x.size), np.arange(x.size))
+
+
+def test_topk_count():
+    """s = max(1, floor(ratio*d)) gives the configured sizes."""
+    assert oracle.topk_count(65_536, 0.01) == 655
+    assert oracle.topk_count(272_474, 0.01) == 2_724
+    assert oracle.topk_count(11_173_962, 0.001) == 11_173
+    assert oracle.topk_count(138_357_544, 0.001) == 138_357
+    assert oracle.topk_count(10, 0.01) == 1
+
+
+# ---------------------------------------------------------------------------
+# P5, P6: the update rule with C eliminated (Sec. 3.3) and Lemma 1
+# ---------------------------------------------------------------------------
+
+def _update_rule_residual(o, grads):
+    """Yield, after each step: both sides of w_{t+1} - w_t = -eta*gbar - eta*ebar_t +
+    eta*ebar_{t+1} + beta*(w_t - w_{t-1}), with an fp32 rounding budget."""
+    eta = float(o.eta)
+    beta = float(o.beta)
+    K = o.K
+    c = float(o.c)
+    w_prev = o.w.astype(np.float64)
+    for g in grads:
+        w_t = o.w.astype(np.float64)
+        e_t = o.e.astype(np.float64)
+        r = o.step(g)
+        w_n = o.w.astype(np.float64)
+        e_n = o.e.astype(np.float64)
+        g64 = g.astype(np.float64)
+        lhs = w_n - w_t
+        rhs = -eta * g64.mean(0) - eta * e_t.mean(0) + eta * e_n.mean(0) + beta * (w_t - w_prev)
+        dl = np.abs(w_t - w_prev)
+        v = np.abs(r.e_half.astype(np.float64))
+        scale = (np.abs(e_t) + np.abs(g64) + c * dl + v + np.abs(e_n)).sum(0)
+        budget = 8 * U * (np.abs(w_n) + np.abs(w_t) + (K + 3) * eta / K * scale + beta * dl)
+        yield lhs, rhs, budget, w_t, w_prev, e_t, e_n, g64
+        w_prev = w_t
+
+
+@pytest.mark.parametrize("compressor", [TOPK, RBGS])
+def test_p5_update_rule(compressor):
+    rng = np.random.default_rng(5)
+    d, K, T = 600, 4, 30
+    o = GMC(d, K, beta=0.9, eta=0.1, compressor=compressor, ratio=0.05, block=16, seed=9)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    for lhs, rhs, budget, *_ in _update_rule_residual(o, _grads(rng, T, K, d)):
+        np.testing.assert_array_less(np.abs(lhs - rhs), budget + 1e-30)
+
+
+@pytest.mark.parametrize("compressor", [TOPK, RBGS])
+def test_p6_lemma1_z_sequence(compressor):
+    """z_t = w_t + beta/(1-beta)(w_t - w_{t-1}) - eta/(1-beta) ebar_t obeys
+    z_{t+1} = z_t - eta/(1-beta) gbar_t for any compressor (Lemma 1)."""
+    rng = np.random.default_rng(6)
+    d, K, T = 400, 3, 25
+    o = GMC(d, K, beta=0.9, eta=0.1, compressor=compressor, ratio=0.02, block=8, seed=3)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    beta, eta = float(o.beta), float(o.eta)
+    for lhs, rhs, budget, w_t, w_prev, e_t, e_n, g in _update_rule_residual(o, _grads(rng, T, K, d)):
+        w_n = w_t + lhs
+        z_t = w_t + beta / (1 - beta) * (w_t - w_prev) - eta / (1 - beta) * e_t.mean(0)
+        z_n = w_n + beta / (1 - beta) * (w_n - w_t) - eta / (1 - beta) * e_n.mean(0)
+        err = np.abs(z_n - (z_t - eta / (1 - beta) * g.mean(0)))
+        np.testing.assert_array_less(err, 2 * budget / (1 - beta) + 1e-30)
+
+
+# ---------------------------------------------------------------------------
+# P6b, P7: GMC+ (Alg. 2) -- the mean-iterate recursion and lambda = 0
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("compressor", [RBGS, TOPK])
+def test_p6b_gmcplus_mean_iterate(compressor):
+    """With wbar_t = mean_k w_{t,k} (the detached points), Sec. 4's
+    zbar_t = wbar_t + beta/(1-beta)(wbar_t - wbar_{t-1})
+             - [(1-lam) eta ebar_t + beta lam eta ebar_{t-1}] / (1-beta)
+    obeys zbar_{t+1} = zbar_t - eta/(1-beta) * mean_k g_{t,k}."""
+    rng = np.random.default_rng(7)
+    d, K, T, lam = 300, 4, 25, 0.5
+    o = GMC(d, K, beta=0.9, eta=0.1, compressor=compressor, ratio=0.05, block=10, lam=lam, seed=1)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    beta, eta = float(o.beta), float(o.eta)
+    lam = float(o.lam)
+
+    def wbar():
+        return np.mean([o.worker_params(k).astype(np.float64) for k in range(K)], axis=0)
+
+    wb_prev = o.w.astype(np.float64)       # wbar_{-1} = w_0
+    eb_prev = np.zeros(d)                  # ebar_{-1} = 0
+    wb = wbar()
+    eb = o.e.astype(np.float64).mean(0)
+    z = wb + beta / (1 - beta) * (wb - wb_prev) - ((1 - lam) * eta * eb + beta * lam * eta * eb_prev) / (1 - beta)
+    for lhs, rhs, budget, w_t, w_prev, e_t, e_n, g in _update_rule_residual(o, _grads(rng, T, K, d)):
+        wb_n = wbar()
+        eb_n = o.e.astype(np.float64).mean(0)
+        z_n = wb_n + beta / (1 - beta) * (wb_n - wb) - ((1 - lam) * eta * eb_n + beta * lam * eta * eb) / (1 - beta)
+        err = np.abs(z_n - (z - eta / (1 - beta) * g.mean(0)))
+        detach_budget = 4 * U * (np.abs(wb) + np.abs(wb_n) + lam * eta * (np.abs(e_t) + np.abs(e_n)).sum(0))
+        np.testing.assert_array_less(err, 2 * (budget + detach_budget) / (1 - beta) + 1e-30)
+        wb, eb, z = wb_n, eb_n, z_n
+
+
+def test_p7_lambda_zero_is_gmc():
+    rng = np.random.default_rng(8)
+    d, K, T = 200, 3, 10
+    runs = []
+    for lam in (0.0, 0.5):
+        o = GMC(d, K, beta=0.9, eta=0.1, compressor=RBGS, ratio=0.1, block=7, lam=lam, seed=2)
+        o.set_params(np.ones(d, np.float32))
+        for g in _grads(np.random.default_rng(80), T, K, d):
+            o.step(g)
+        runs.append(o)
+    a, b = runs
+    assert np.array_equal(a.w.view(np.uint32), b.w.view(np.uint32))
+    assert np.array_equal(a.e.view(np.uint32), b.e.view(np.uint32))
+    for k in range(K):
+        assert np.array_equal(a.worker_params(k).view(np.uint32), a.w.view(np.uint32))
+    assert not np.array_equal(b.worker_params(0), b.w)
+    del rng
+
+
+# ---------------------------------------------------------------------------
+# P8: RBGS -- generator, sampler, counts, RCC
+# ---------------------------------------------------------------------------
+
+def test_splitmix64_published_outputs():
+    gold = _golden("splitmix64.json")
+    for seed, key in ((0, "seed_0"), (1234567, "seed_1234567")):
+        want = [int(h, 16) for h in gold[key]]
+        assert oracle.splitmix64_sequence(seed, len(want)) == want
+
+
+def test_below_range():
+    for n in (1, 2, 3, 6240, 2 ** 32):
+        for x in (0, 1, 2 ** 32 - 1, 2 ** 63, 2 ** 64 - 1, 0x123456789ABCDEF0):
+            assert 0 <= oracle.below(x, n) < n
+    assert oracle.below(2 ** 64 - 1, 6240) == 6239
+
+
+def test_floyd_uniform_over_subsets():
+    """Floyd's sampler fed by the generator hits every m-subset of [0, nb)
+    equally often (chi-square, 20 subsets of 3 out of 6)."""
+    nb, m, n = 6, 3, 20_000
+    counts = {}
+    for i in range(n):
+        key = oracle.rbgs_stream_key(12345, i, 0)
+        sub = tuple(oracle.floyd_blocks(key, nb, m))
+        assert len(set(sub)) == m and list(sub) == sorted(sub)
+        counts[sub] = counts.get(sub, 0) + 1
+    assert len(counts) == math.comb(nb, m)
+    expected = n / len(counts)
+    chi2 = sum((c - expected) ** 2 / expected for c in counts.values())
+    assert chi2 < 60.0  # 19 degrees of freedom; p < 1e-5 beyond this
+
+
+@pytest.mark.parametrize("per_worker", [False, True])
+def test_p8_rbgs_counts(per_worker):
+    rng = np.random.default_rng(9)
+    d, K, B, ratio = 1000, 5, 64, 0.2     # nb = 16 (last block 40 long), m = 3
+    o = GMC(d, K, beta=0.9, eta=0.1, compressor=RBGS, ratio=ratio, block=B, seed=77,
+            per_worker=per_worker)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    assert (o.nb, o.m) == (16, 3)
+    for t in range(6):
+        r = o.step(rng.standard_normal((K, d)).astype(np.float32))
+        assert len(r.blocks) == (K if per_worker else 1)
+        for blocks in r.blocks:
+            assert blocks.size == o.m and np.unique(blocks).size == o.m
+            assert blocks.min() >= 0 and blocks.max() < o.nb
+        for k in range(K):
+            blocks = r.blocks[k if per_worker else 0]
+            size = sum(min((b + 1) * B, d) - b * B for b in blocks)
+            assert r.supports[k].size == size
+            assert np.count_nonzero(r.values[k]) == size
+        if not per_worker:
+            for k in range(1, K):
+                np.testing.assert_array_equal(r.supports[k], r.supports[0])
+    if per_worker:
+        assert any(not np.array_equal(r.supports[k], r.supports[0]) for k in range(1, K))
+
+
+def test_p8_rbgs_rcc_matches_paper():
+    """One shared block of d/1024 components: RCC = 1/1024 (Sec. 5.2)."""
+    gold = _golden("rcc_rbgs.json")
+    d, K = 1024 * 37, 4
+    B = d // 1024
+    nb = -(-d // B)
+    ratio = 1.0 / nb                       # m = max(1, floor(ratio * nb)) = 1
+    o = GMC(d, K, beta=0.9, eta=0.1, compressor=RBGS, ratio=ratio, block=B, seed=4)
+    assert o.m == gold["blocks_chosen"]
+    rng = np.random.default_rng(10)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    for _ in range(5):
+        o.step((rng.standard_normal((K, d)) + 3.0).astype(np.float32))
+    assert o.rcc() == pytest.approx(gold["rcc"], rel=0, abs=1e-15)
+
+
+def test_rcc_dense_pairs():
+    """No compression with (index, value) pairs: every component is sent by
+    every worker and every parameter changes, so RCC = 2 (Sec. 5 accounting)."""
+    rng = np.random.default_rng(11)
+    d, K = 50, 3
+    o = GMC(d, K, beta=0.5, eta=0.1, compressor=TOPK, ratio=1.0)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    for _ in range(4):
+        o.step((rng.standard_normal((K, d)) + 5.0).astype(np.float32))
+    assert o.rcc() == 2.0
+
+
+# ---------------------------------------------------------------------------
+# P9: the two-worker quadratic of Sec. 3.2 (qualitative; parity unpinned)
+# ---------------------------------------------------------------------------
+
+def test_p9_toy_quadratic_converges():
+    cfg = _golden("toy_quadratic.json")
+    d, K = cfg["d"], cfg["K"]
+    i = np.arange(d)
+    wgt = (d - i).astype(np.float64)
+    o = GMC(d, K, beta=cfg["beta"], eta=cfg["eta"], compressor=TOPK, ratio=cfg["s_fraction"])
+    o.set_params(np.array(cfg["start"], np.float32))
+    dist = []
+    for _ in range(3000):
+        w = o.w.astype(np.float64)
+        g = np.stack([2 * wgt * (w - (i + 1)), 2 * wgt * (w + (i + 1))]).astype(np.float32)
+        o.step(g)
+        dist.append(float(np.linalg.norm(o.w)))
+    d0 = float(np.linalg.norm(cfg["start"]))
+    assert dist[500] < 1e-3 * d0
+    assert max(dist[-1000:]) < 1e-4 * d0
