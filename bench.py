@@ -1,0 +1,421 @@
+"""Benchmark of one GMC / GMC+ step on GB300: worker-parameters per second.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl gmc|reference]
+
+A step is one pass of the whole hot path (accumulator, compression, residual,
+aggregate and update) for the K simulated workers of the workload over one
+batch of synthetic gradients already resident in HBM. ``value`` is
+K*d*steps*ranks / (max over ranks of the device time of the timed steps).
+``e2e`` is the same metric through the host-memory entry point (host->device
+copy of the step's gradients and device->host read of the step's counters
+inside the timed region). ``roofline`` reports the dominant kernel's
+algorithmic bytes per launch over its CUDA-event duration against the measured
+HBM copy peak. ``cpu_baseline`` times the oracle on the host cores on a bounded
+sample of the same workload.
+
+Multi-GPU: the step does not shard (K workers are simulated on one GPU), so
+N > 1 runs N independent replicas, one per rank, and reports their aggregate.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import workloads  # noqa: E402
+
+METRIC = "GMC step throughput (worker-params/sec) and achieved HBM GB/s vs 8 TB/s, 1 GB300"
+UNIT = "worker-params/s"
+DEFAULT_WORKLOAD = "vgg16"
+FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129e6
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    """Samples SM clock and throttle reasons of one GPU while running: NVML
+    through ctypes (read-only queries) when available, else nvidia-smi."""
+
+    REASONS = {0x8: "hw_slowdown", 0x40: "hw_thermal_slowdown", 0x20: "sw_thermal_slowdown",
+               0x4: "sw_power_cap", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, index: int, period_s: float = 0.01):
+        self.index = index
+        self.period = period_s
+        self.samples = []  # (sm_mhz, reasons_mask)
+        self.max_mhz = None
+        self._stop = threading.Event()
+        self._nvml = None
+        self._handle = None
+        self._proc = None
+        self._csv = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() == 0:
+                h = ctypes.c_void_p()
+                if nv.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(index), ctypes.byref(h)) == 0:
+                    self._nvml, self._handle = nv, h
+                    mx = ctypes.c_uint()
+                    if nv.nvmlDeviceGetMaxClockInfo(h, ctypes.c_int(1), ctypes.byref(mx)) == 0:
+                        self.max_mhz = mx.value
+        except OSError:
+            self._nvml = None
+
+    def _sample_nvml(self):
+        nv, h = self._nvml, self._handle
+        clk, reasons = ctypes.c_uint(), ctypes.c_ulonglong()
+        if nv.nvmlDeviceGetClockInfo(h, ctypes.c_int(1), ctypes.byref(clk)) == 0:
+            nv.nvmlDeviceGetCurrentClocksThrottleReasons(h, ctypes.byref(reasons))
+            self.samples.append((clk.value, reasons.value))
+
+    def _loop(self):
+        while not self._stop.is_set():
+            self._sample_nvml()
+            time.sleep(self.period)
+
+    def start(self):
+        if self._nvml is not None:
+            self._sample_nvml()
+            self._thread = threading.Thread(target=self._loop, daemon=True)
+            self._thread.start()
+        else:
+            self._csv = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            q = ("clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,"
+                 "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_power_cap")
+            try:
+                self._proc = subprocess.Popen(
+                    ["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
+                     "--format=csv,noheader,nounits", "-lms", "50"],
+                    stdout=self._csv, stderr=subprocess.DEVNULL)
+            except OSError:
+                self._proc = None
+
+    def stop(self) -> dict:
+        if self._nvml is not None:
+            self._stop.set()
+            self._thread.join()
+            self._sample_nvml()
+        elif self._proc is not None:
+            time.sleep(0.1)
+            self._proc.terminate()
+            self._proc.wait()
+            self._csv.seek(0)
+            names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+            bits = [0x8, 0x40, 0x20, 0x4]
+            for line in self._csv.read().splitlines():
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 6 or not parts[0].isdigit():
+                    continue
+                mask = sum(b for b, v in zip(bits, parts[2:6]) if v.lower() == "active")
+                self.samples.append((int(parts[0]), mask))
+                self.max_mhz = int(parts[1]) if parts[1].isdigit() else self.max_mhz
+            del names
+            os.unlink(self._csv.name)
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": [], "samples": 0}
+        mask = 0
+        for _, m in self.samples:
+            mask |= m
+        return {"sm_mhz": statistics.median(s for s, _ in self.samples), "sm_max_mhz": self.max_mhz,
+                "reasons": [n for b, n in self.REASONS.items() if mask & b],
+                "samples": len(self.samples)}
+
+
+# ---------------------------------------------------------------------------
+# helpers
+# ---------------------------------------------------------------------------
+def measured_hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_1905_12948_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel sources (profiles/<kernel>_<workload>.md holds lines
+    `traffic_bytes_per_launch: N` and `source_hash: H`)."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    hsh = re.search(r"source_hash:\s*([0-9a-f]+)", text)
+    if not m or not hsh or hsh.group(1) != kernel_source_hash():
+        return None
+    return float(m.group(1))
+
+
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl"
+        try:
+            import torch
+            if not torch.cuda.is_available():
+                backend = "gloo"
+        except ImportError:
+            backend = "gloo"
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle on a bounded sample of the workload
+# ---------------------------------------------------------------------------
+def oracle_sample(wl, budget_s: float = 12.0, max_steps: int = 50, workers: int = 1,
+                  d_sample: int = 1 << 24, first_step: int = 0):
+    """Time the oracle (as it stands) on a bounded sample of the workload:
+    `workers` of its workers over the leading `d_sample` parameters (same
+    per-parameter gradient scales, same compression ratio), running steps
+    until `budget_s` of CPU time is spent. Input generation is not timed."""
+    import oracle
+    K_s = min(workers, wl.K)
+    d_s = min(wl.d, d_sample)
+    gen = workloads.NumpyGradients(wl, seed=0, d=d_s, K=K_s)
+    o = oracle.GMC(d_s, K_s, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
+                   block=wl.block, lam=wl.lam, seed=0, per_worker=wl.per_worker)
+    o.set_params(workloads.init_params(wl.d)[:d_s])
+    spent, steps = 0.0, 0
+    while steps < max_steps and (spent < budget_s or steps == 0):
+        g = gen(first_step + steps)
+        t0 = time.perf_counter()
+        o.step(g)
+        spent += time.perf_counter() - t0
+        steps += 1
+        del g
+    return {"value": K_s * d_s * steps / spent, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{steps} oracle step(s) of {K_s} of the {wl.K} workers over the first "
+                      f"{d_s:,} of d={wl.d:,} parameters (numpy, one thread), {spent:.1f} s",
+            "seconds": round(spent, 3), "d_sample": d_s}
+
+
+# ---------------------------------------------------------------------------
+# arms
+# ---------------------------------------------------------------------------
+def run_reference(args, wl, world, rank):
+    if rank != 0:
+        return None
+    d_s = 1 << 23
+    for i in range(args.warmup):
+        oracle_sample(wl, budget_s=0.0, max_steps=1, d_sample=d_s, first_step=i)
+    t0 = time.perf_counter()
+    samples = [oracle_sample(wl, budget_s=0.0, max_steps=1, d_sample=d_s, first_step=i)
+               for i in range(args.steps)]
+    elapsed = time.perf_counter() - t0
+    spent = sum(s["seconds"] for s in samples)
+    d_s = samples[0]["d_sample"]
+    value = d_s * args.steps / spent
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * spent / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic", "config": config_of(wl, args),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"each step: one oracle step of 1 of the {wl.K} workers over "
+                                   f"the first {d_s:,} of d={wl.d:,} parameters (numpy, one "
+                                   f"thread); wall {elapsed:.1f} s including input generation"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    return line
+
+
+def config_of(wl, args):
+    return {"workload": f"{wl.name}: d={wl.d:,}, K={wl.K}, {wl.compressor}"
+                        + (f" ratio {wl.ratio}" if wl.compressor == "topk"
+                           else f" block {wl.block}, {wl.ratio:.0%} of blocks, lambda {wl.lam}")
+                        + f", beta {wl.beta}, eta {wl.eta}",
+            "d": wl.d, "K": wl.K, "compressor": wl.compressor, "ratio": wl.ratio,
+            "block": wl.block if wl.compressor == "rbgs" else None,
+            "per_worker_blocks": wl.per_worker if wl.compressor == "rbgs" else None,
+            "lambda": wl.lam, "l2": "inputs larger than L2 (gradient batches rotate)",
+            "parallelism": f"replicas x{args.gpus}"}
+
+
+def run_gmc(args, wl, world, rank, local):
+    import torch
+    from paper_1905_12948_gb300 import GMC
+    from paper_1905_12948_gb300 import build as gbuild
+    if rank == 0:
+        gbuild.build()
+    barrier(world)
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    gpu = GMC(wl.d, wl.K, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
+              block=wl.block, lam=wl.lam if wl.compressor == "rbgs" else None, seed=0,
+              per_worker=wl.per_worker, device=dev)
+    w0 = torch.from_numpy(workloads.init_params(wl.d)).to(dev)
+    gen = workloads.TorchGradients(wl, dev, seed=rank)
+    n_batches = 2 if 4.0 * wl.K * wl.d > 2 * L2_BYTES else max(2, math.ceil(4 * L2_BYTES / (4.0 * wl.K * wl.d)))
+    batches = [gen(t) for t in range(n_batches)]
+    del gen
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+
+    gpu.set_params(w0)
+    for i in range(args.warmup):
+        gpu.step(batches[i % n_batches])
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    gpu.profile(True)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        gpu.step(batches[(args.warmup + i) % n_batches])
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(world)
+    ms = ev0.elapsed_time(ev1)
+    prof = gpu.profile_read()
+    gpu.profile(False)
+    status = gpu.check()
+    ms_max = max_over_ranks(ms, world, dev)
+    value = wl.K * wl.d * args.steps * world / (ms_max / 1e3)
+
+    dom = "accumulate" if wl.compressor == "topk" else "rbgs_step"
+    p = prof.get(dom, {"ms": float("nan"), "launches": 1, "bytes": float("nan")})
+    per_launch_bytes = p["bytes"] / p["launches"]
+    avg_s = p["ms"] / p["launches"] / 1e3
+    achieved = per_launch_bytes / avg_s / 1e9
+    peak, peak_kind = measured_hbm_peak()
+    traffic = recorded_traffic(dom, wl.name)
+    step_ms = ms / args.steps
+    kernels = {k: {"ms_per_step": round(v["ms"] / args.steps, 4),
+                   "share": round(v["ms"] / max(sum(x["ms"] for x in prof.values()), 1e-12), 4)}
+               for k, v in prof.items()}
+    del batches
+    torch.cuda.synchronize()
+
+    e2e = None
+    if not args.no_e2e:
+        host = torch.empty((wl.K, wl.d), dtype=torch.float32).pin_memory()
+        host.copy_(torch.from_numpy(workloads.NumpyGradients(wl, seed=rank, K=wl.K)(0))
+                   if wl.K * wl.d <= 50_000_000 else
+                   workloads.TorchGradients(wl, dev, seed=rank)(0).cpu())
+        stats = torch.zeros(8, dtype=torch.int64).pin_memory()
+        gpu.set_params(w0)
+        for _ in range(max(1, min(args.warmup, 3))):
+            gpu.step_host(host, stats)
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            gpu.step_host(host, stats)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+        e2e = {"value": wl.K * wl.d * args.steps * world / (e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": 4 * wl.K * wl.d, "d2h_bytes_per_step": 8 * 8,
+               "ms_per_step": e_ms / args.steps}
+        del host
+    gpu.close()
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = oracle_sample(wl, budget_s=args.cpu_budget)
+        cpu.pop("seconds", None)
+
+    launches_per_step = sum(v["launches"] for v in prof.values()) / args.steps
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": config_of(wl, args),
+        "hbm_gbs_step": 12.0 * wl.K * wl.d / (step_ms / 1e3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": traffic, "algorithmic_bytes_per_launch": per_launch_bytes,
+                     "avg_launch_ms": avg_s * 1e3},
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+        "gpu_launches": int(round(launches_per_step * args.steps)),
+        "kernels": kernels, "status": status,
+    }
+    return line if rank == 0 else None
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["gmc", "reference"], default="gmc")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
+                    help="one of " + ", ".join(w.name for w in workloads.WORKLOADS))
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle CPU time")
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "gmc":
+        ap.error("--warmup must be >= 3")
+    wl = workloads.workload(args.workload)
+    world, rank, local = dist_setup(args.gpus)
+    if args.impl == "reference":
+        line = run_reference(args, wl, world, rank)
+    else:
+        line = run_gmc(args, wl, world, rank, local)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,205 @@
+/*
+ * gmc.h -- C ABI of the GB300 library for one Global Momentum Compression
+ * (GMC / GMC+) step, with K data-parallel workers simulated on one GPU.
+ *
+ * Method: Shi et al., "Global Momentum Compression for Sparse Communication in
+ * Distributed Learning", arXiv 1905.12948.
+ *   Algorithm 1 (GMC, Sec. 3.1), for every worker k and step t:
+ *     e_{t+1/2,k} = e_{t,k} + g_{t,k} - (beta/eta) (w_t - w_{t-1})
+ *     send C(e_{t+1/2,k});  e_{t+1,k} = e_{t+1/2,k} - C(e_{t+1/2,k})
+ *     w_{t+1} = w_t - (eta/K) sum_k C(e_{t+1/2,k})
+ *   with w_{-1} = w_0 and e_{0,k} = 0.
+ *   Algorithm 2 (GMC+, Sec. 4) adds the detached point
+ *     w_{t+1,k} = w_{t+1} - lambda*eta*e_{t+1,k}.
+ *   Compressors (Sec. 4, Sec. 5.2): exact top-s ("top-k"), and RBGS (random
+ *   blocks chosen with one seed shared by all workers).
+ *
+ * Arithmetic: fp32, one IEEE round-to-nearest-even rounding per operation in
+ * the order written above: v = (e + g) - (c * (w_t - w_{t-1})), c = fl(beta/eta);
+ * the aggregate adds the workers' values in ascending worker order starting
+ * from +0; w_{t+1} = w_t - (a * sum), a = fl(eta/K); detach w - (b * e),
+ * b = fl(lambda*eta). Top-k ranks |v| through the fp32 bit pattern with the
+ * sign cleared; ties go to the lower index. k = max(1, floor(ratio*d)).
+ *
+ * Conventions (all calls):
+ *   - Every pointer argument named *_dev is device memory on the GPU that was
+ *     current when the handle was created; *_host arguments are host memory.
+ *   - The library owns its state (w, w_{t-1} - w_t, residuals, workspace),
+ *     allocated once in gmc_create and freed in gmc_destroy. Caller buffers
+ *     are borrowed: they must stay valid until the stream has passed the call.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream). Calls are
+ *     stream-ordered and asynchronous unless marked "synchronising".
+ *   - Argument errors return at once and enqueue nothing. Data-dependent
+ *     errors (a non-finite accumulator value, an internal consistency check)
+ *     are recorded in a device status word read by gmc_check.
+ *   - A handle is not thread-safe; distinct handles are independent.
+ *   - No C++ exception crosses this boundary.
+ */
+#ifndef GMC_H
+#define GMC_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct gmc_ctx* gmc_t;
+
+/* Status codes. */
+#define GMC_OK          0  /* success */
+#define GMC_EINVAL      1  /* invalid argument or handle */
+#define GMC_ENOMEM      2  /* device or host allocation failed */
+#define GMC_ECUDA       3  /* a CUDA call or kernel launch failed */
+#define GMC_ENONFINITE  4  /* a step met a NaN or Inf accumulator value */
+#define GMC_ESTATE      5  /* call out of order (e.g. gmc_step before gmc_set_params) */
+#define GMC_EINTERNAL   6  /* an internal consistency check failed on the device */
+
+/* Compressors C(.). */
+#define GMC_TOPK 0 /* exact top-k by magnitude, ties to the lower index (Sec. 4 top-s) */
+#define GMC_RBGS 1 /* random aligned blocks of `block` components (Sec. 4, Sec. 5.2) */
+
+/* Top-k selection engines; both give identical results. */
+#define GMC_SELECT_SAMPLED 0 /* default: a sampled threshold filters candidates in the one
+                                dense pass; exact radix select among them; falls back to
+                                GMC_SELECT_DENSE for a worker whose filter missed */
+#define GMC_SELECT_DENSE   1 /* exact multi-pass radix select over the dense accumulator */
+
+/* Slots of the counters returned by gmc_get_stats and gmc_step_host. */
+#define GMC_STAT_STEPS      0 /* steps taken (cumulative counters only) */
+#define GMC_STAT_PAIRS      1 /* sum_k |supp C_k|: components sent by the workers */
+#define GMC_STAT_NNZ        2 /* sum_k ||C_k||_0: sent components that are non-zero */
+#define GMC_STAT_UNION      3 /* |U_t|: coordinates sent by at least one worker */
+#define GMC_STAT_CHANGED    4 /* ||w_{t+1} - w_t||_0 */
+#define GMC_STAT_FALLBACKS  5 /* workers whose sampled filter fell back to the dense select */
+#define GMC_STAT_NONFINITE  6 /* accumulator values that were NaN or Inf */
+#define GMC_STAT_COUNT      8 /* array length to pass */
+
+/* Kernel ids for gmc_profile_read. */
+#define GMC_KERNEL_ACCUMULATE  0 /* fused accumulator + candidate filter (top-k), one dense pass */
+#define GMC_KERNEL_RBGS_STEP   1 /* fused accumulator + RBGS compress + aggregate + update */
+#define GMC_KERNEL_SAMPLE      2 /* sampled threshold per worker */
+#define GMC_KERNEL_SELECT      3 /* exact radix select among candidates (3 launches per step) */
+#define GMC_KERNEL_DENSE       4 /* exact dense select for workers that fell back */
+#define GMC_KERNEL_COMPACT     5 /* index-ordered compaction of C(v) (3 launches per step) */
+#define GMC_KERNEL_AGGREGATE   6 /* worker-ordered aggregate + update (top-k) */
+#define GMC_KERNEL_RBGS_PICK   7 /* RBGS block choice (Floyd sampling) */
+#define GMC_KERNEL_DETACH      8 /* GMC+ detached points */
+#define GMC_KERNEL_OTHER       9 /* counters and small bookkeeping */
+#define GMC_KERNEL_COUNT      10
+
+/*
+ * gmc_create -- allocate a handle and its device state on the current device.
+ * Inputs of Algorithm 1 (Sec. 3.1): d parameters, K workers, momentum beta in
+ * [0,1), learning rate eta > 0, compressor C; ratio in (0,1] is the kept share
+ * (top-k: k = max(1, floor(ratio*d)); RBGS: m = max(1, floor(ratio*nb)) of the
+ * nb = ceil(d/block) blocks); block >= 1 is the RBGS block size (ignored for
+ * top-k). Requires 1 <= d < 2^31 - 2^16 and 1 <= K <= 1024.
+ * GMC+'s lambda defaults to 0 (plain GMC) for top-k and 0.5 for RBGS (Sec. 5.2
+ * uses 0.5 for GMC+). Returns GMC_EINVAL, GMC_ENOMEM or GMC_ECUDA on failure,
+ * with *out set to NULL. The state must be initialised with gmc_set_params.
+ */
+int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta,
+               int32_t compressor, double ratio, int64_t block);
+
+/* gmc_destroy -- synchronise the device and free everything the handle owns. */
+void gmc_destroy(gmc_t h);
+
+/* gmc_set_lambda -- GMC+ detach coefficient lambda in [0,1] (Alg. 2); 0 is GMC. */
+int gmc_set_lambda(gmc_t h, float lambda);
+
+/* gmc_set_rbgs_mode -- 0: one block choice per step shared by all workers, as in
+ * Sec. 4 / Sec. 5.2 (default); 1: an independent choice per worker. */
+int gmc_set_rbgs_mode(gmc_t h, int32_t per_worker);
+
+/* gmc_set_seed -- seed of the RBGS block choice (SplitMix64 counter stream
+ * keyed by (seed, t[, k]); Floyd's sampling). Default 0. */
+int gmc_set_seed(gmc_t h, uint64_t seed);
+
+/* gmc_set_eta -- change eta between steps (e.g. the cosine schedule of Sec. 5.1);
+ * takes effect at the next gmc_step. */
+int gmc_set_eta(gmc_t h, float eta);
+
+/* gmc_set_select_mode -- GMC_SELECT_SAMPLED (default) or GMC_SELECT_DENSE. */
+int gmc_set_select_mode(gmc_t h, int32_t mode);
+
+/* gmc_set_detach_output -- GMC+ (Alg. 2 detach): when out_dev is not NULL, every
+ * following gmc_step also writes w_{t+1,k} = w_{t+1} - lambda*eta*e_{t+1,k} into
+ * out_dev[k*ld + j] (K rows, row stride ld >= d floats, caller-owned and borrowed
+ * until disabled with NULL). */
+int gmc_set_detach_output(gmc_t h, float* out_dev, int64_t ld);
+
+/* gmc_set_params -- w_0 := w0_dev[0..d) (device, fp32); also sets w_{-1} = w_0,
+ * e_{0,k} = 0, t = 0 and clears the counters (Alg. 1 initialisation). */
+int gmc_set_params(gmc_t h, const float* w0_dev, void* stream);
+
+/* gmc_step -- one iteration t of Alg. 1 (Alg. 2 when lambda > 0 and a detach
+ * output is set). grads_dev: K x d fp32, row-major (worker k's gradient
+ * g_{t,k} at grads_dev[k*d .. k*d+d)), device memory, read-only, borrowed until
+ * the stream has passed the step; any alignment. Enqueues kernels only; never
+ * synchronises. Non-finite accumulator values still complete the step
+ * deterministically and are reported by gmc_check as GMC_ENONFINITE. */
+int gmc_step(gmc_t h, const float* grads_dev, void* stream);
+
+/* gmc_step_host -- gmc_step from host memory: copies grads_host (K x d fp32,
+ * row-major; pinned host memory gives an asynchronous copy) into a library
+ * staging buffer (allocated on the first call), runs the step, and copies the
+ * step's counters (GMC_STAT_COUNT uint64 slots, GMC_STAT_STEPS slot = 1) into
+ * step_stats_host, which must then be pinned host memory valid until the
+ * stream has passed the call (or NULL to skip the read-back). */
+int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, void* stream);
+
+/* gmc_get_params -- copy w_t (d floats) into w_dev_out. */
+int gmc_get_params(gmc_t h, float* w_dev_out, void* stream);
+
+/* gmc_get_residual -- copy e_{t,k} (d floats) into e_dev_out. */
+int gmc_get_residual(gmc_t h, int32_t k, float* e_dev_out, void* stream);
+
+/* gmc_get_selected -- synchronising. The last step's C(e_{t-1/2,k}) of worker k
+ * as (index, value) pairs in ascending index order: *count_host pairs written to
+ * idx_dev / val_dev (device, capacity entries each). Returns GMC_EINVAL if
+ * capacity is too small (with *count_host set to the size needed), GMC_ESTATE
+ * before the first step. */
+int gmc_get_selected(gmc_t h, int32_t k, uint32_t* idx_dev, float* val_dev,
+                     int64_t capacity, int64_t* count_host, void* stream);
+
+/* gmc_selected_capacity -- the largest number of pairs one worker can send per
+ * step (k for top-k, m*block for RBGS), or -1 for an invalid handle. */
+int64_t gmc_selected_capacity(gmc_t h);
+
+/* gmc_get_worker_params -- GMC+ detached point of worker k at the current step,
+ * w_{t,k} = w_t - lambda*eta*e_{t,k} (Alg. 2), written to out_dev (d floats). */
+int gmc_get_worker_params(gmc_t h, int32_t k, float* out_dev, void* stream);
+
+/* gmc_get_stats -- synchronising. Cumulative counters since gmc_set_params
+ * (n <= GMC_STAT_COUNT slots copied into counters_host) and the relative
+ * communication cost of Sec. 5, RCC = (K*sum_t ||w_{t+1}-w_t||_0 +
+ * sum_t sum_k ||C_k||_0) / (d K T), halved for RBGS (no indices, Sec. 5.2). */
+int gmc_get_stats(gmc_t h, uint64_t* counters_host, int32_t n, double* rcc_host);
+
+/* gmc_check -- synchronising. GMC_OK, or the first data-dependent error recorded
+ * since gmc_set_params (GMC_ENONFINITE, GMC_EINTERNAL), or GMC_ECUDA. */
+int gmc_check(gmc_t h);
+
+/* gmc_profile_enable -- when on, each kernel launch of gmc_step is bracketed by
+ * CUDA events on the step's stream; gmc_profile_read reports the totals. */
+int gmc_profile_enable(gmc_t h, int32_t on);
+
+/* gmc_profile_read -- synchronising. For kernel id `kernel` (GMC_KERNEL_*): the
+ * summed device time in ms, the number of launches, and the algorithmic bytes
+ * those launches had to move (the minimum traffic of the operation), since
+ * profiling was enabled. Resets nothing. */
+int gmc_profile_read(gmc_t h, int32_t kernel, double* total_ms, int64_t* launches,
+                     double* algorithmic_bytes);
+
+/* gmc_kernel_name -- a static name for a GMC_KERNEL_* id ("?" if unknown). */
+const char* gmc_kernel_name(int32_t kernel);
+
+/* gmc_strerror -- a static message for a status code. */
+const char* gmc_strerror(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GMC_H */

@@ -1,0 +1,648 @@
+// C ABI of libgmc (declared in include/gmc.h): handle lifecycle, argument
+// validation, device state, and the orchestration of one GMC / GMC+ step on a
+// caller-given stream. Only host code lives here; the kernels are in
+// gmc_topk.cu and gmc_rbgs.cu.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "gmc.h"
+#include "gmc_internal.h"
+
+using namespace gmc;
+
+namespace {
+
+struct ProfRec {
+  int kernel;
+  cudaEvent_t start, stop;
+};
+
+}  // namespace
+
+struct gmc_ctx {
+  int device = 0;
+  int num_sms = 1;
+  // problem
+  int64_t d = 0;
+  int K = 0;
+  float beta = 0.f, eta = 0.f, lambda = 0.f;
+  int compressor = GMC_TOPK;
+  double ratio = 0.0;
+  int64_t block = 0;
+  uint64_t seed = 0;
+  int per_worker = 0;
+  int select_mode = GMC_SELECT_SAMPLED;
+  float* detach_out = nullptr;
+  int64_t detach_ld = 0;
+  // geometry
+  int tile = 0;
+  int64_t n_tiles = 0, ld = 0;
+  uint32_t ksel = 0, cap = 0, sample_rank = 0;
+  int sample_chunks = 0;
+  int64_t nb = 0, m = 0;
+  uint32_t B_shift = 0xffffffffu;
+  int grid_acc = 1, grid_agg = 1, grid_rbgs = 1, sel_blocks = 1;
+  // state
+  int64_t t = 0;
+  bool initialized = false;
+  float* e = nullptr;
+  float* w = nullptr;
+  float* dlt = nullptr;
+  WorkerSel* sel = nullptr;
+  uint32_t* cand_idx = nullptr;
+  float* cand_val = nullptr;
+  uint32_t *chunk_base = nullptr, *chunk_cnt = nullptr, *gt_cnt = nullptr, *eq_cnt = nullptr,
+           *eq_before = nullptr, *ghist = nullptr;
+  uint32_t* pos[2] = {nullptr, nullptr};
+  uint32_t* idx[2] = {nullptr, nullptr};
+  float* val[2] = {nullptr, nullptr};
+  uint32_t* bitmap = nullptr;
+  int32_t* rank = nullptr;
+  int32_t* blocks = nullptr;
+  uint8_t* uflag[2] = {nullptr, nullptr};
+  float* slab = nullptr;
+  Counters* step_ctr = nullptr;
+  Counters* total_ctr = nullptr;
+  unsigned* status = nullptr;
+  float* gstage = nullptr;
+  std::vector<void*> allocations;
+  // profiling
+  bool prof = false;
+  std::vector<ProfRec> pending;
+  std::vector<cudaEvent_t> free_events;
+  double prof_ms[GMC_KERNEL_COUNT] = {};
+  int64_t prof_launches[GMC_KERNEL_COUNT] = {};
+  double prof_bytes[GMC_KERNEL_COUNT] = {};
+};
+
+namespace {
+
+class DeviceGuard {
+ public:
+  explicit DeviceGuard(int dev) {
+    cudaGetDevice(&prev_);
+    if (prev_ != dev) cudaSetDevice(dev);
+    dev_ = dev;
+  }
+  ~DeviceGuard() {
+    if (prev_ != dev_) cudaSetDevice(prev_);
+  }
+
+ private:
+  int prev_ = 0, dev_ = 0;
+};
+
+template <typename T>
+cudaError_t dalloc(gmc_ctx* h, T** p, size_t count) {
+  void* q = nullptr;
+  const size_t bytes = std::max<size_t>(count, 1) * sizeof(T);
+  cudaError_t err = cudaMalloc(&q, bytes);
+  if (err != cudaSuccess) {
+    *p = nullptr;
+    return err;
+  }
+  h->allocations.push_back(q);
+  *p = static_cast<T*>(q);
+  return cudaMemset(q, 0, bytes);
+}
+
+void free_all(gmc_ctx* h) {
+  for (void* p : h->allocations) cudaFree(p);
+  h->allocations.clear();
+  for (auto& r : h->pending) {
+    cudaEventDestroy(r.start);
+    cudaEventDestroy(r.stop);
+  }
+  h->pending.clear();
+  for (cudaEvent_t e : h->free_events) cudaEventDestroy(e);
+  h->free_events.clear();
+}
+
+int status_of(cudaError_t err) {
+  if (err == cudaSuccess) return GMC_OK;
+  if (err == cudaErrorMemoryAllocation) return GMC_ENOMEM;
+  return GMC_ECUDA;
+}
+
+cudaEvent_t take_event(gmc_ctx* h) {
+  if (!h->free_events.empty()) {
+    cudaEvent_t e = h->free_events.back();
+    h->free_events.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Enqueue one kernel launch, bracketed by events when profiling is on.
+template <typename F>
+cudaError_t timed(gmc_ctx* h, int kernel, double bytes, cudaStream_t s, F&& launch) {
+  if (!h->prof) return launch();
+  ProfRec r{kernel, take_event(h), take_event(h)};
+  cudaEventRecord(r.start, s);
+  cudaError_t err = launch();
+  cudaEventRecord(r.stop, s);
+  h->pending.push_back(r);
+  h->prof_bytes[kernel] += bytes;
+  return err;
+}
+
+void drain_profile(gmc_ctx* h) {
+  for (auto& r : h->pending) {
+    cudaEventSynchronize(r.stop);
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, r.start, r.stop) == cudaSuccess) {
+      h->prof_ms[r.kernel] += ms;
+      h->prof_launches[r.kernel] += 1;
+    }
+    h->free_events.push_back(r.start);
+    h->free_events.push_back(r.stop);
+  }
+  h->pending.clear();
+}
+
+void set_constants(gmc_ctx* h, TopkArgs* A) {
+  A->c = h->beta / h->eta;
+  A->a = h->eta / (float)h->K;
+}
+
+TopkArgs topk_args(gmc_ctx* h, const float* grads) {
+  TopkArgs A;
+  std::memset(&A, 0, sizeof(A));
+  const int cur = (int)(h->t & 1), prev = cur ^ 1;
+  A.e = h->e;
+  A.ld = h->ld;
+  A.grads = grads;
+  A.d = h->d;
+  A.dlt = h->dlt;
+  A.w = h->w;
+  set_constants(h, &A);
+  A.K = h->K;
+  A.n_tiles = h->n_tiles;
+  A.tile = h->tile;
+  A.ksel = h->ksel;
+  A.cap = h->cap;
+  A.sample_rank = h->sample_rank;
+  A.sample_chunks = h->sample_chunks;
+  A.has_prev = h->t > 0;
+  A.dense_mode = h->select_mode == GMC_SELECT_DENSE;
+  A.sel = h->sel;
+  A.cand_idx = h->cand_idx;
+  A.cand_val = h->cand_val;
+  A.chunk_base = h->chunk_base;
+  A.chunk_cnt = h->chunk_cnt;
+  A.gt_cnt = h->gt_cnt;
+  A.eq_cnt = h->eq_cnt;
+  A.eq_before = h->eq_before;
+  A.ghist = h->ghist;
+  A.pos_prev = h->pos[prev];
+  A.idx_prev = h->idx[prev];
+  A.pos_cur = h->pos[cur];
+  A.idx_cur = h->idx[cur];
+  A.val_cur = h->val[cur];
+  A.step_ctr = h->step_ctr;
+  A.status = h->status;
+  return A;
+}
+
+RbgsArgs rbgs_args(gmc_ctx* h, const float* grads) {
+  RbgsArgs A;
+  std::memset(&A, 0, sizeof(A));
+  const int cur = (int)(h->t & 1), prev = cur ^ 1;
+  A.e = h->e;
+  A.ld = h->ld;
+  A.grads = grads;
+  A.d = h->d;
+  A.dlt = h->dlt;
+  A.w = h->w;
+  A.c = h->beta / h->eta;
+  A.a = h->eta / (float)h->K;
+  A.K = h->K;
+  A.n_tiles = h->n_tiles;
+  A.B = h->block;
+  A.B_shift = h->B_shift;
+  A.nb = h->nb;
+  A.m = h->m;
+  A.per_worker = h->per_worker;
+  A.seed = h->seed;
+  A.t = h->t;
+  A.bitmap = h->bitmap;
+  A.rank = h->rank;
+  A.blocks = h->blocks;
+  A.uflag_prev = h->uflag[prev];
+  A.uflag_cur = h->uflag[cur];
+  A.slab = h->slab;
+  A.has_prev = h->t > 0;
+  A.step_ctr = h->step_ctr;
+  A.status = h->status;
+  return A;
+}
+
+#define GMC_TRY(expr)                          \
+  do {                                         \
+    const cudaError_t err_ = (expr);           \
+    if (err_ != cudaSuccess) return status_of(err_); \
+  } while (0)
+
+int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s) {
+  const double Kd = (double)h->K * (double)h->d;
+  GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
+  unsigned long long pairs_add = 0;
+  if (h->compressor == GMC_TOPK) {
+    const TopkArgs A = topk_args(h, grads);
+    const double kk = (double)h->K * (double)h->ksel;
+    GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
+                  [&] { return launch_accumulate(A, h->grid_acc, s); }));
+    for (int pass = 0; pass < 3; ++pass)
+      GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s,
+                    [&] { return launch_select_pass(A, pass, h->sel_blocks, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_DENSE, 0.0, s, [&] { return launch_select_dense(A, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_COMPACT, 0.0, s, [&] { return launch_chunk_count(A, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_COMPACT, 0.0, s, [&] { return launch_chunk_scan(A, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_COMPACT, 16.0 * kk, s, [&] { return launch_chunk_write(A, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk, s,
+                  [&] { return launch_aggregate(A, h->grid_agg, s); }));
+    pairs_add = (unsigned long long)h->K * h->ksel;
+  } else {
+    const RbgsArgs A = rbgs_args(h, grads);
+    GMC_TRY(cudaMemsetAsync(A.uflag_cur, 0, (size_t)h->nb, s));
+    GMC_TRY(timed(h, GMC_KERNEL_RBGS_PICK, 0.0, s, [&] { return launch_rbgs_pick(A, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_RBGS_STEP, 12.0 * Kd, s,
+                  [&] { return launch_rbgs_step(A, h->grid_rbgs, s); }));
+  }
+  if (h->detach_out) {
+    DetachArgs D{h->w, h->e, h->ld, h->d, h->lambda * h->eta, h->detach_out, h->detach_ld, 0, h->K};
+    GMC_TRY(timed(h, GMC_KERNEL_DETACH, 8.0 * Kd + 4.0 * h->d, s, [&] { return launch_detach(D, s); }));
+  }
+  GMC_TRY(timed(h, GMC_KERNEL_OTHER, 0.0, s,
+                [&] { return launch_finalize(h->step_ctr, h->total_ctr, pairs_add, s); }));
+  h->t += 1;
+  return GMC_OK;
+}
+
+bool finite_f(float x) { return std::isfinite(x); }
+
+}  // namespace
+
+extern "C" {
+
+const char* gmc_strerror(int status) {
+  switch (status) {
+    case GMC_OK: return "success";
+    case GMC_EINVAL: return "invalid argument";
+    case GMC_ENOMEM: return "out of memory";
+    case GMC_ECUDA: return "CUDA error";
+    case GMC_ENONFINITE: return "non-finite accumulator value";
+    case GMC_ESTATE: return "call out of order";
+    case GMC_EINTERNAL: return "internal consistency check failed";
+    default: return "unknown status";
+  }
+}
+
+const char* gmc_kernel_name(int32_t kernel) {
+  static const char* names[GMC_KERNEL_COUNT] = {
+      "accumulate", "rbgs_step", "sample", "select", "dense_select",
+      "compact", "aggregate", "rbgs_pick", "detach", "other"};
+  return (kernel >= 0 && kernel < GMC_KERNEL_COUNT) ? names[kernel] : "?";
+}
+
+int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t compressor,
+               double ratio, int64_t block) {
+  if (!out) return GMC_EINVAL;
+  *out = nullptr;
+  if (d < 1 || d >= (int64_t(1) << 31) - (int64_t(1) << 16)) return GMC_EINVAL;
+  if (K < 1 || K > 1024) return GMC_EINVAL;
+  if (!finite_f(beta) || !(beta >= 0.f) || !(beta < 1.f)) return GMC_EINVAL;
+  if (!finite_f(eta) || !(eta > 0.f)) return GMC_EINVAL;
+  if (!std::isfinite(ratio) || !(ratio > 0.0) || !(ratio <= 1.0)) return GMC_EINVAL;
+  if (compressor != GMC_TOPK && compressor != GMC_RBGS) return GMC_EINVAL;
+  if (compressor == GMC_RBGS && block < 1) return GMC_EINVAL;
+
+  gmc_ctx* h = new (std::nothrow) gmc_ctx();
+  if (!h) return GMC_ENOMEM;
+  cudaGetDevice(&h->device);
+  cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+  if (h->num_sms < 1) h->num_sms = 1;
+  h->d = d;
+  h->K = K;
+  h->beta = beta;
+  h->eta = eta;
+  h->compressor = compressor;
+  h->ratio = ratio;
+  h->block = block;
+  h->lambda = compressor == GMC_RBGS ? 0.5f : 0.f;
+
+  auto fail = [&](cudaError_t err) {
+    free_all(h);
+    delete h;
+    cudaGetLastError();
+    return status_of(err);
+  };
+  cudaError_t err = configure_topk_kernels();
+  if (err == cudaSuccess) err = configure_rbgs_kernels();
+  if (err != cudaSuccess) return fail(err);
+
+  const int64_t streams_wide = 2 * (int64_t)h->num_sms;
+  if (compressor == GMC_TOPK) {
+    int U = 4;
+    if (d < 4096 * streams_wide) U = 2;
+    if (d < 2048 * streams_wide) U = 1;
+    h->tile = 1024 * U;
+    h->n_tiles = (d + h->tile - 1) / h->tile;
+    h->ld = h->n_tiles * h->tile;
+    const int64_t ks = std::max<int64_t>(1, (int64_t)std::floor(ratio * (double)d));
+    h->ksel = (uint32_t)ks;
+    if (d <= kSampleAll) {
+      h->sample_chunks = 0;
+      h->sample_rank = h->ksel;
+      h->cap = (uint32_t)d;
+    } else {
+      h->sample_chunks = kSampleChunks;
+      const double ns = 8.0 * kSampleChunks;
+      const double mean = ns * (double)ks / (double)d;
+      const double r = std::min(ns, std::ceil(mean + 5.0 * std::sqrt(mean) + 8.0));
+      h->sample_rank = (uint32_t)r;
+      const double capd = std::ceil((double)d * (r + 8.0 * std::sqrt(r) + 16.0) / ns) + 4096.0;
+      h->cap = (uint32_t)std::min<double>((double)d, capd);
+    }
+    h->grid_acc = (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * accumulate_blocks_per_sm(h->tile));
+    h->grid_agg = (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * aggregate_blocks_per_sm(h->tile));
+    const int64_t per = (h->cap + 8191) / 8192;
+    h->sel_blocks = (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
+    const int64_t Kt = (int64_t)K * h->n_tiles;
+    if ((err = dalloc(h, &h->e, (size_t)K * h->ld)) != cudaSuccess ||
+        (err = dalloc(h, &h->w, (size_t)h->ld)) != cudaSuccess ||
+        (err = dalloc(h, &h->dlt, (size_t)h->ld)) != cudaSuccess ||
+        (err = dalloc(h, &h->sel, (size_t)K)) != cudaSuccess ||
+        (err = dalloc(h, &h->cand_idx, (size_t)K * h->cap)) != cudaSuccess ||
+        (err = dalloc(h, &h->cand_val, (size_t)K * h->cap)) != cudaSuccess ||
+        (err = dalloc(h, &h->chunk_base, (size_t)Kt)) != cudaSuccess ||
+        (err = dalloc(h, &h->chunk_cnt, (size_t)Kt)) != cudaSuccess ||
+        (err = dalloc(h, &h->gt_cnt, (size_t)Kt)) != cudaSuccess ||
+        (err = dalloc(h, &h->eq_cnt, (size_t)Kt)) != cudaSuccess ||
+        (err = dalloc(h, &h->eq_before, (size_t)Kt)) != cudaSuccess ||
+        (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess)
+      return fail(err);
+    for (int p = 0; p < 2; ++p) {
+      if ((err = dalloc(h, &h->pos[p], (size_t)K * (h->n_tiles + 1))) != cudaSuccess ||
+          (err = dalloc(h, &h->idx[p], (size_t)K * h->ksel)) != cudaSuccess ||
+          (err = dalloc(h, &h->val[p], (size_t)K * h->ksel)) != cudaSuccess)
+        return fail(err);
+    }
+  } else {
+    h->tile = kRbgsTile;
+    h->n_tiles = (d + h->tile - 1) / h->tile;
+    h->ld = h->n_tiles * h->tile;
+    h->nb = (d + block - 1) / block;
+    h->m = std::max<int64_t>(1, (int64_t)std::floor(ratio * (double)h->nb));
+    if (h->nb >= (int64_t(1) << 31)) return fail(cudaErrorInvalidValue);
+    if ((block & (block - 1)) == 0) {
+      uint32_t sh = 0;
+      while ((int64_t(1) << sh) < block) ++sh;
+      h->B_shift = sh;
+    }
+    h->grid_rbgs = (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * rbgs_blocks_per_sm());
+    const int64_t nbw = (h->nb + 31) / 32;
+    if ((err = dalloc(h, &h->e, (size_t)K * h->ld)) != cudaSuccess ||
+        (err = dalloc(h, &h->w, (size_t)h->ld)) != cudaSuccess ||
+        (err = dalloc(h, &h->dlt, (size_t)h->ld)) != cudaSuccess ||
+        (err = dalloc(h, &h->bitmap, (size_t)K * nbw)) != cudaSuccess ||
+        (err = dalloc(h, &h->rank, (size_t)K * h->nb)) != cudaSuccess ||
+        (err = dalloc(h, &h->blocks, (size_t)K * h->m)) != cudaSuccess ||
+        (err = dalloc(h, &h->uflag[0], (size_t)h->nb)) != cudaSuccess ||
+        (err = dalloc(h, &h->uflag[1], (size_t)h->nb)) != cudaSuccess ||
+        (err = dalloc(h, &h->slab, (size_t)K * h->m * block)) != cudaSuccess)
+      return fail(err);
+  }
+  if ((err = dalloc(h, &h->step_ctr, 1)) != cudaSuccess ||
+      (err = dalloc(h, &h->total_ctr, 1)) != cudaSuccess ||
+      (err = dalloc(h, &h->status, 1)) != cudaSuccess)
+    return fail(err);
+  if ((err = cudaDeviceSynchronize()) != cudaSuccess) return fail(err);
+  *out = h;
+  return GMC_OK;
+}
+
+void gmc_destroy(gmc_t h) {
+  if (!h) return;
+  DeviceGuard g(h->device);
+  cudaDeviceSynchronize();
+  free_all(h);
+  delete h;
+}
+
+int gmc_set_lambda(gmc_t h, float lambda) {
+  if (!h || !finite_f(lambda) || lambda < 0.f || lambda > 1.f) return GMC_EINVAL;
+  h->lambda = lambda;
+  return GMC_OK;
+}
+
+int gmc_set_rbgs_mode(gmc_t h, int32_t per_worker) {
+  if (!h || (per_worker != 0 && per_worker != 1)) return GMC_EINVAL;
+  h->per_worker = per_worker;
+  return GMC_OK;
+}
+
+int gmc_set_seed(gmc_t h, uint64_t seed) {
+  if (!h) return GMC_EINVAL;
+  h->seed = seed;
+  return GMC_OK;
+}
+
+int gmc_set_eta(gmc_t h, float eta) {
+  if (!h || !finite_f(eta) || !(eta > 0.f)) return GMC_EINVAL;
+  h->eta = eta;
+  return GMC_OK;
+}
+
+int gmc_set_select_mode(gmc_t h, int32_t mode) {
+  if (!h || (mode != GMC_SELECT_SAMPLED && mode != GMC_SELECT_DENSE)) return GMC_EINVAL;
+  h->select_mode = mode;
+  return GMC_OK;
+}
+
+int gmc_set_detach_output(gmc_t h, float* out_dev, int64_t ld) {
+  if (!h) return GMC_EINVAL;
+  if (out_dev && ld < h->d) return GMC_EINVAL;
+  h->detach_out = out_dev;
+  h->detach_ld = out_dev ? ld : 0;
+  return GMC_OK;
+}
+
+int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
+  if (!h || !w0_dev) return GMC_EINVAL;
+  DeviceGuard g(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  GMC_TRY(cudaMemcpyAsync(h->w, w0_dev, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice, s));
+  GMC_TRY(cudaMemsetAsync(h->e, 0, (size_t)h->K * h->ld * sizeof(float), s));
+  GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
+  if (h->compressor == GMC_TOPK) {
+    for (int p = 0; p < 2; ++p)
+      GMC_TRY(cudaMemsetAsync(h->pos[p], 0, (size_t)h->K * (h->n_tiles + 1) * sizeof(uint32_t), s));
+    GMC_TRY(cudaMemsetAsync(h->sel, 0, (size_t)h->K * sizeof(WorkerSel), s));
+  } else {
+    for (int p = 0; p < 2; ++p) GMC_TRY(cudaMemsetAsync(h->uflag[p], 0, (size_t)h->nb, s));
+  }
+  GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
+  GMC_TRY(cudaMemsetAsync(h->total_ctr, 0, sizeof(Counters), s));
+  GMC_TRY(cudaMemsetAsync(h->status, 0, sizeof(unsigned), s));
+  h->t = 0;
+  h->initialized = true;
+  return GMC_OK;
+}
+
+int gmc_step(gmc_t h, const float* grads_dev, void* stream) {
+  if (!h || !grads_dev) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  return enqueue_step(h, grads_dev, static_cast<cudaStream_t>(stream));
+}
+
+int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, void* stream) {
+  if (!h || !grads_host) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t n = (size_t)h->K * (size_t)h->d;
+  if (!h->gstage) {
+    cudaError_t err = dalloc(h, &h->gstage, n);
+    if (err != cudaSuccess) return status_of(err);
+  }
+  GMC_TRY(cudaMemcpyAsync(h->gstage, grads_host, n * sizeof(float), cudaMemcpyHostToDevice, s));
+  const int st = enqueue_step(h, h->gstage, s);
+  if (st != GMC_OK) return st;
+  if (step_stats_host)
+    GMC_TRY(cudaMemcpyAsync(step_stats_host, h->step_ctr, sizeof(Counters), cudaMemcpyDeviceToHost, s));
+  return GMC_OK;
+}
+
+int gmc_get_params(gmc_t h, float* w_dev_out, void* stream) {
+  if (!h || !w_dev_out) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  GMC_TRY(cudaMemcpyAsync(w_dev_out, h->w, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice,
+                          static_cast<cudaStream_t>(stream)));
+  return GMC_OK;
+}
+
+int gmc_get_residual(gmc_t h, int32_t k, float* e_dev_out, void* stream) {
+  if (!h || !e_dev_out || k < 0 || k >= h->K) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  GMC_TRY(cudaMemcpyAsync(e_dev_out, h->e + (int64_t)k * h->ld, (size_t)h->d * sizeof(float),
+                          cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream)));
+  return GMC_OK;
+}
+
+int64_t gmc_selected_capacity(gmc_t h) {
+  if (!h) return -1;
+  return h->compressor == GMC_TOPK ? (int64_t)h->ksel : h->m * h->block;
+}
+
+int gmc_get_selected(gmc_t h, int32_t k, uint32_t* idx_dev, float* val_dev, int64_t capacity,
+                     int64_t* count_host, void* stream) {
+  if (!h || !idx_dev || !val_dev || !count_host || k < 0 || k >= h->K) return GMC_EINVAL;
+  if (!h->initialized || h->t == 0) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int last = (int)((h->t - 1) & 1);
+  if (h->compressor == GMC_TOPK) {
+    *count_host = h->ksel;
+    if (capacity < (int64_t)h->ksel) return GMC_EINVAL;
+    GMC_TRY(cudaMemcpyAsync(idx_dev, h->idx[last] + (int64_t)k * h->ksel, h->ksel * sizeof(uint32_t),
+                            cudaMemcpyDeviceToDevice, s));
+    GMC_TRY(cudaMemcpyAsync(val_dev, h->val[last] + (int64_t)k * h->ksel, h->ksel * sizeof(float),
+                            cudaMemcpyDeviceToDevice, s));
+  } else {
+    int32_t last_block = 0;
+    const int32_t* blk = h->blocks + (h->per_worker ? (int64_t)k * h->m : 0) + (h->m - 1);
+    GMC_TRY(cudaMemcpyAsync(&last_block, blk, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+    GMC_TRY(cudaStreamSynchronize(s));
+    int64_t count = h->m * h->block;
+    if (last_block == h->nb - 1) count -= h->nb * h->block - h->d;
+    *count_host = count;
+    if (capacity < count) return GMC_EINVAL;
+    RbgsArgs A = rbgs_args(h, nullptr);
+    GMC_TRY(launch_rbgs_expand(A, k, idx_dev, val_dev, s));
+  }
+  GMC_TRY(cudaStreamSynchronize(s));
+  return GMC_OK;
+}
+
+int gmc_get_worker_params(gmc_t h, int32_t k, float* out_dev, void* stream) {
+  if (!h || !out_dev || k < 0 || k >= h->K) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  DetachArgs D{h->w, h->e, h->ld, h->d, h->lambda * h->eta, out_dev, h->d, k, k + 1};
+  GMC_TRY(launch_detach(D, static_cast<cudaStream_t>(stream)));
+  return GMC_OK;
+}
+
+int gmc_get_stats(gmc_t h, uint64_t* counters_host, int32_t n, double* rcc_host) {
+  if (!h || n < 0 || n > GMC_STAT_COUNT || (n > 0 && !counters_host)) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  GMC_TRY(cudaDeviceSynchronize());
+  Counters c;
+  GMC_TRY(cudaMemcpy(&c, h->total_ctr, sizeof(Counters), cudaMemcpyDeviceToHost));
+  for (int i = 0; i < n; ++i) counters_host[i] = c.v[i];
+  if (rcc_host) {
+    const double T = (double)c.v[kSteps];
+    double r = 0.0;
+    if (T > 0) {
+      r = ((double)h->K * (double)c.v[kChanged] + (double)c.v[kNnz]) /
+          ((double)h->d * (double)h->K * T);
+      if (h->compressor == GMC_RBGS) r *= 0.5;
+    }
+    *rcc_host = r;
+  }
+  return GMC_OK;
+}
+
+int gmc_check(gmc_t h) {
+  if (!h) return GMC_EINVAL;
+  if (!h->initialized) return GMC_OK;
+  DeviceGuard g(h->device);
+  cudaError_t err = cudaDeviceSynchronize();
+  if (err != cudaSuccess) return GMC_ECUDA;
+  unsigned st = 0;
+  err = cudaMemcpy(&st, h->status, sizeof(unsigned), cudaMemcpyDeviceToHost);
+  if (err != cudaSuccess) return GMC_ECUDA;
+  if (st & kStatusInternal) return GMC_EINTERNAL;
+  if (st & kStatusNonfinite) return GMC_ENONFINITE;
+  return GMC_OK;
+}
+
+int gmc_profile_enable(gmc_t h, int32_t on) {
+  if (!h) return GMC_EINVAL;
+  DeviceGuard g(h->device);
+  if (on && !h->prof) {
+    drain_profile(h);
+    for (int i = 0; i < GMC_KERNEL_COUNT; ++i) {
+      h->prof_ms[i] = 0.0;
+      h->prof_launches[i] = 0;
+      h->prof_bytes[i] = 0.0;
+    }
+  }
+  h->prof = on != 0;
+  return GMC_OK;
+}
+
+int gmc_profile_read(gmc_t h, int32_t kernel, double* total_ms, int64_t* launches,
+                     double* algorithmic_bytes) {
+  if (!h || kernel < 0 || kernel >= GMC_KERNEL_COUNT) return GMC_EINVAL;
+  DeviceGuard g(h->device);
+  drain_profile(h);
+  if (total_ms) *total_ms = h->prof_ms[kernel];
+  if (launches) *launches = h->prof_launches[kernel];
+  if (algorithmic_bytes) *algorithmic_bytes = h->prof_bytes[kernel];
+  return GMC_OK;
+}
+
+}  // extern "C"
