@@ -54,6 +54,7 @@ typedef struct gmc_ctx* gmc_t;
 #define GMC_ENONFINITE  4  /* a step met a NaN or Inf accumulator value */
 #define GMC_ESTATE      5  /* call out of order (e.g. gmc_step before gmc_set_params) */
 #define GMC_EINTERNAL   6  /* an internal consistency check failed on the device */
+#define GMC_ETOOBIG     7  /* size above the fixed scratch of gmc_topk_noalloc */
 
 /* Compressors C(.). */
 #define GMC_TOPK 0 /* exact top-k by magnitude, ties to the lower index (Sec. 4 top-s) */
@@ -194,6 +195,27 @@ int gmc_profile_read(gmc_t h, int32_t kernel, double* total_ms, int64_t* launche
 
 /* gmc_kernel_name -- a static name for a GMC_KERNEL_* id ("?" if unknown). */
 const char* gmc_kernel_name(int32_t kernel);
+
+/*
+ * gmc_topk_noalloc -- the top-k compressor of one vector without allocating.
+ * The paper has no counterpart: this is a library convenience for callers
+ * that cannot call cudaMalloc, e.g. code whose device memory is all owned by
+ * another allocator (a framework's caching pool or a fixed serving budget),
+ * so neither the library nor the caller may allocate scratch for it.
+ * Writes the k pairs (index, value) of x_dev[0..n) that come first under
+ * (|x| fp32 bit pattern descending, index ascending) -- the same selection as
+ * GMC_TOPK -- to idx_dev / val_dev (device, k entries each) in ascending index
+ * order. x_dev is device memory, fp32, read-only. Requires 1 <= k <= n
+ * (else GMC_EINVAL) and n <= 2^26 (else GMC_ETOOBIG).
+ * It allocates nothing: its scratch is one fixed array of about 270 KB in the
+ * library's device memory, which every GPU that loads the library holds until
+ * the process exits. All calls share that array, so calls that overlap on the
+ * GPU (on different streams, or from different threads) race; serialise
+ * them. The first call on each device looks up the array's device address;
+ * make that first call before any stream capture. Stream-ordered, asynchronous.
+ */
+int gmc_topk_noalloc(const float* x_dev, int64_t n, int64_t k, uint32_t* idx_dev, float* val_dev,
+                     void* stream);
 
 /* gmc_strerror -- a static message for a status code. */
 const char* gmc_strerror(int status);

@@ -23,7 +23,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libgmc.so")
 
-SOURCES = ["gmc_api.cu", "gmc_topk.cu", "gmc_rbgs.cu"]
+SOURCES = ["gmc_api.cu", "gmc_topk.cu", "gmc_rbgs.cu", "gmc_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", *ARCH,
          "-fmad=false", "-ftz=false", "-prec-div=true", "-prec-sqrt=true",

@@ -301,6 +301,7 @@ const char* gmc_strerror(int status) {
     case GMC_ENONFINITE: return "non-finite accumulator value";
     case GMC_ESTATE: return "call out of order";
     case GMC_EINTERNAL: return "internal consistency check failed";
+    case GMC_ETOOBIG: return "size exceeds the fixed scratch of gmc_topk_noalloc (n <= 2^26)";
     default: return "unknown status";
   }
 }

@@ -14,7 +14,7 @@ from typing import Optional, Tuple
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libgmc.so")
 
-GMC_OK, GMC_EINVAL, GMC_ENOMEM, GMC_ECUDA, GMC_ENONFINITE, GMC_ESTATE, GMC_EINTERNAL = range(7)
+GMC_OK, GMC_EINVAL, GMC_ENOMEM, GMC_ECUDA, GMC_ENONFINITE, GMC_ESTATE, GMC_EINTERNAL, GMC_ETOOBIG = range(8)
 GMC_TOPK, GMC_RBGS = 0, 1
 GMC_SELECT_SAMPLED, GMC_SELECT_DENSE = 0, 1
 STAT_NAMES = ["steps", "pairs", "nnz", "union", "changed", "fallbacks", "nonfinite", "reserved"]
@@ -54,6 +54,7 @@ _SIGNATURES = {
                                         ctypes.POINTER(_f64)]),
     "gmc_kernel_name": (ctypes.c_char_p, [_i32]),
     "gmc_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+    "gmc_topk_noalloc": (ctypes.c_int, [_c_p, _i64, _i64, _c_p, _c_p, _c_p]),
 }
 
 _lib = None
