@@ -186,7 +186,10 @@ class TorchGradients:
             return out
         if wl.laplace_frac > 0:
             u = torch.rand((wl.K, wl.d), generator=gen, device=self.device) - 0.5
-            lap = -wl.laplace_scale * torch.sign(u) * torch.log1p(-2.0 * u.abs())
+            # |u| < 1/2 keeps the inverse CDF finite (rand() can return exactly 0)
+            mag = torch.clamp(u.abs(), max=0.5 - 2.0 ** -25)
+            lap = -wl.laplace_scale * torch.sign(u) * torch.log1p(-2.0 * mag)
+            del mag
             heavy = torch.rand((wl.K, wl.d), generator=gen, device=self.device) < wl.laplace_frac
             out.copy_(torch.where(heavy, lap, out))
             del u, lap, heavy
