@@ -95,7 +95,7 @@ typedef struct gmc_ctx* gmc_t;
  * [0,1), learning rate eta > 0, compressor C; ratio in (0,1] is the kept share
  * (top-k: k = max(1, floor(ratio*d)); RBGS: m = max(1, floor(ratio*nb)) of the
  * nb = ceil(d/block) blocks); block >= 1 is the RBGS block size (ignored for
- * top-k). Requires 1 <= d < 2^31 - 2^16 and 1 <= K <= 1024.
+ * top-k). Requires 1 <= d < 2^31 - 2^16 and 1 <= K <= 32.
  * GMC+'s lambda defaults to 0 (plain GMC) for top-k and 0.5 for RBGS (Sec. 5.2
  * uses 0.5 for GMC+). Returns GMC_EINVAL, GMC_ENOMEM or GMC_ECUDA on failure,
  * with *out set to NULL. The state must be initialised with gmc_set_params.

@@ -53,13 +53,18 @@ struct gmc_ctx {
   float* w = nullptr;
   float* dlt = nullptr;
   WorkerSel* sel = nullptr;
-  uint32_t* cand_idx = nullptr;
-  float* cand_val = nullptr;
-  uint32_t *chunk_base = nullptr, *chunk_cnt = nullptr, *gt_cnt = nullptr, *eq_cnt = nullptr,
-           *eq_before = nullptr, *ghist = nullptr;
-  uint32_t* pos[2] = {nullptr, nullptr};
-  uint32_t* idx[2] = {nullptr, nullptr};
-  float* val[2] = {nullptr, nullptr};
+  uint32_t* ghist = nullptr;
+  uint32_t* sample_keys = nullptr;
+  uint32_t* big_tiles = nullptr;
+  uint32_t* rcount = nullptr;
+  int regions = 1;
+  uint32_t cap_region = 0;
+  int sample_blocks = 1;
+  uint32_t* cand_idx[2] = {nullptr, nullptr};
+  float* cand_val[2] = {nullptr, nullptr};
+  uint32_t* chunk_base[2] = {nullptr, nullptr};
+  uint32_t* chunk_cnt[2] = {nullptr, nullptr};
+  uint32_t* mask = nullptr;
   uint32_t* bitmap = nullptr;
   int32_t* rank = nullptr;
   int32_t* blocks = nullptr;
@@ -171,10 +176,11 @@ void set_constants(gmc_ctx* h, TopkArgs* A) {
   A->a = h->eta / (float)h->K;
 }
 
-TopkArgs topk_args(gmc_ctx* h, const float* grads) {
+// Arguments of step t's top-k kernels; chunk buffers alternate with the parity of t.
+TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   TopkArgs A;
   std::memset(&A, 0, sizeof(A));
-  const int cur = (int)(h->t & 1), prev = cur ^ 1;
+  const int cur = (int)(t & 1), prev = cur ^ 1;
   A.e = h->e;
   A.ld = h->ld;
   A.grads = grads;
@@ -189,26 +195,30 @@ TopkArgs topk_args(gmc_ctx* h, const float* grads) {
   A.cap = h->cap;
   A.sample_rank = h->sample_rank;
   A.sample_chunks = h->sample_chunks;
-  A.has_prev = h->t > 0;
+  A.sample_blocks = h->sample_blocks;
+  A.has_prev = t > 0;
   A.dense_mode = h->select_mode == GMC_SELECT_DENSE;
   A.sel = h->sel;
-  A.cand_idx = h->cand_idx;
-  A.cand_val = h->cand_val;
-  A.chunk_base = h->chunk_base;
-  A.chunk_cnt = h->chunk_cnt;
-  A.gt_cnt = h->gt_cnt;
-  A.eq_cnt = h->eq_cnt;
-  A.eq_before = h->eq_before;
   A.ghist = h->ghist;
-  A.pos_prev = h->pos[prev];
-  A.idx_prev = h->idx[prev];
-  A.pos_cur = h->pos[cur];
-  A.idx_cur = h->idx[cur];
-  A.val_cur = h->val[cur];
+  A.sample_keys = h->sample_keys;
+  A.big_tiles = h->big_tiles;
+  A.regions = h->regions;
+  A.cap_region = h->cap_region;
+  A.rcount = h->rcount;
+  A.cand_idx = h->cand_idx[cur];
+  A.cand_val = h->cand_val[cur];
+  A.chunk_base = h->chunk_base[cur];
+  A.chunk_cnt = h->chunk_cnt[cur];
+  A.mask = h->mask;
+  A.cand_idx_prev = h->cand_idx[prev];
+  A.chunk_base_prev = h->chunk_base[prev];
+  A.chunk_cnt_prev = h->chunk_cnt[prev];
   A.step_ctr = h->step_ctr;
   A.status = h->status;
   return A;
 }
+
+TopkArgs topk_args(gmc_ctx* h, const float* grads) { return topk_args_at(h, grads, h->t); }
 
 RbgsArgs rbgs_args(gmc_ctx* h, const float* grads) {
   RbgsArgs A;
@@ -262,10 +272,8 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s) {
     for (int pass = 0; pass < 3; ++pass)
       GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s,
                     [&] { return launch_select_pass(A, pass, h->sel_blocks, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] { return launch_ties(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_DENSE, 0.0, s, [&] { return launch_select_dense(A, s); }));
-    GMC_TRY(timed(h, GMC_KERNEL_COMPACT, 0.0, s, [&] { return launch_chunk_count(A, s); }));
-    GMC_TRY(timed(h, GMC_KERNEL_COMPACT, 0.0, s, [&] { return launch_chunk_scan(A, s); }));
-    GMC_TRY(timed(h, GMC_KERNEL_COMPACT, 16.0 * kk, s, [&] { return launch_chunk_write(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk, s,
                   [&] { return launch_aggregate(A, h->grid_agg, s); }));
     pairs_add = (unsigned long long)h->K * h->ksel;
@@ -318,12 +326,13 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
   if (!out) return GMC_EINVAL;
   *out = nullptr;
   if (d < 1 || d >= (int64_t(1) << 31) - (int64_t(1) << 16)) return GMC_EINVAL;
-  if (K < 1 || K > 1024) return GMC_EINVAL;
+  if (K < 1) return GMC_EINVAL;
   if (!finite_f(beta) || !(beta >= 0.f) || !(beta < 1.f)) return GMC_EINVAL;
   if (!finite_f(eta) || !(eta > 0.f)) return GMC_EINVAL;
   if (!std::isfinite(ratio) || !(ratio > 0.0) || !(ratio <= 1.0)) return GMC_EINVAL;
   if (compressor != GMC_TOPK && compressor != GMC_RBGS) return GMC_EINVAL;
   if (compressor == GMC_RBGS && block < 1) return GMC_EINVAL;
+  if (K > 32) return GMC_EINVAL;
 
   gmc_ctx* h = new (std::nothrow) gmc_ctx();
   if (!h) return GMC_ENOMEM;
@@ -373,27 +382,42 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
       h->cap = (uint32_t)std::min<double>((double)d, capd);
     }
     h->grid_acc = (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * accumulate_blocks_per_sm(h->tile));
-    h->grid_agg = (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * aggregate_blocks_per_sm(h->tile));
+    h->grid_agg = 0;  // set below from the candidate regions
+    // candidate slots: the bulk pass gives every CTA its own region per worker
+    // (twice its share of the expected candidates, plus slack); otherwise one region
+    const uint32_t cap0 = h->cap;
+    if (h->tile == 4096) {
+      h->regions = h->grid_acc;
+      h->cap_region = (uint32_t)(((2ull * cap0 + h->regions - 1) / h->regions + 1024 + 3) & ~3ull);
+    } else {
+      h->regions = 1;
+      h->cap_region = (cap0 + 3) & ~3u;
+    }
+    h->cap = (uint32_t)std::min<uint64_t>((uint64_t)h->regions * h->cap_region, 0xfffffff0ull);
     const int64_t per = (h->cap + 8191) / 8192;
-    h->sel_blocks = (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
+    h->grid_agg = h->regions > 1 ? h->regions : (int)std::max<int64_t>(1, 4 * (int64_t)h->num_sms / K);
+    // select passes: about 2048 expected candidates per block
+    const double expect = h->sample_chunks ? (double)d * h->sample_rank / (8.0 * kSampleChunks) : (double)h->ksel;
+    const int64_t want = std::max<int64_t>(1, (int64_t)(expect / 2048.0));
+    h->sel_blocks = h->regions > 1 ? (int)std::min<int64_t>(h->regions, want)
+                                   : (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
+    h->sample_blocks = (int)std::max<int64_t>(1, ((h->sample_chunks ? 8 * kSampleChunks : d) + 2047) / 2048);
     const int64_t Kt = (int64_t)K * h->n_tiles;
     if ((err = dalloc(h, &h->e, (size_t)K * h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->w, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->dlt, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->sel, (size_t)K)) != cudaSuccess ||
-        (err = dalloc(h, &h->cand_idx, (size_t)K * h->cap)) != cudaSuccess ||
-        (err = dalloc(h, &h->cand_val, (size_t)K * h->cap)) != cudaSuccess ||
-        (err = dalloc(h, &h->chunk_base, (size_t)Kt)) != cudaSuccess ||
-        (err = dalloc(h, &h->chunk_cnt, (size_t)Kt)) != cudaSuccess ||
-        (err = dalloc(h, &h->gt_cnt, (size_t)Kt)) != cudaSuccess ||
-        (err = dalloc(h, &h->eq_cnt, (size_t)Kt)) != cudaSuccess ||
-        (err = dalloc(h, &h->eq_before, (size_t)Kt)) != cudaSuccess ||
-        (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess)
+        (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess ||
+        (err = dalloc(h, &h->sample_keys, (size_t)K * 8 * kSampleChunks)) != cudaSuccess ||
+        (err = dalloc(h, &h->big_tiles, (size_t)h->n_tiles + 1)) != cudaSuccess ||
+        (err = dalloc(h, &h->rcount, (size_t)K * h->regions)) != cudaSuccess ||
+        (err = dalloc(h, &h->mask, (size_t)h->ld)) != cudaSuccess)
       return fail(err);
     for (int p = 0; p < 2; ++p) {
-      if ((err = dalloc(h, &h->pos[p], (size_t)K * (h->n_tiles + 1))) != cudaSuccess ||
-          (err = dalloc(h, &h->idx[p], (size_t)K * h->ksel)) != cudaSuccess ||
-          (err = dalloc(h, &h->val[p], (size_t)K * h->ksel)) != cudaSuccess)
+      if ((err = dalloc(h, &h->cand_idx[p], (size_t)K * h->cap)) != cudaSuccess ||
+          (err = dalloc(h, &h->cand_val[p], (size_t)K * h->cap)) != cudaSuccess ||
+          (err = dalloc(h, &h->chunk_base[p], (size_t)Kt * kChunksPerTile)) != cudaSuccess ||
+          (err = dalloc(h, &h->chunk_cnt[p], (size_t)Kt * kChunksPerTile)) != cudaSuccess)
         return fail(err);
     }
   } else {
@@ -485,7 +509,7 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
   GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
   if (h->compressor == GMC_TOPK) {
     for (int p = 0; p < 2; ++p)
-      GMC_TRY(cudaMemsetAsync(h->pos[p], 0, (size_t)h->K * (h->n_tiles + 1) * sizeof(uint32_t), s));
+      GMC_TRY(cudaMemsetAsync(h->chunk_cnt[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint32_t), s));
     GMC_TRY(cudaMemsetAsync(h->sel, 0, (size_t)h->K * sizeof(WorkerSel), s));
   } else {
     for (int p = 0; p < 2; ++p) GMC_TRY(cudaMemsetAsync(h->uflag[p], 0, (size_t)h->nb, s));
@@ -552,14 +576,11 @@ int gmc_get_selected(gmc_t h, int32_t k, uint32_t* idx_dev, float* val_dev, int6
   if (!h->initialized || h->t == 0) return GMC_ESTATE;
   DeviceGuard g(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int last = (int)((h->t - 1) & 1);
   if (h->compressor == GMC_TOPK) {
     *count_host = h->ksel;
     if (capacity < (int64_t)h->ksel) return GMC_EINVAL;
-    GMC_TRY(cudaMemcpyAsync(idx_dev, h->idx[last] + (int64_t)k * h->ksel, h->ksel * sizeof(uint32_t),
-                            cudaMemcpyDeviceToDevice, s));
-    GMC_TRY(cudaMemcpyAsync(val_dev, h->val[last] + (int64_t)k * h->ksel, h->ksel * sizeof(float),
-                            cudaMemcpyDeviceToDevice, s));
+    const TopkArgs A = topk_args_at(h, nullptr, h->t - 1);
+    GMC_TRY(launch_gather_selected(A, k, idx_dev, val_dev, s));
   } else {
     int32_t last_block = 0;
     const int32_t* blk = h->blocks + (h->per_worker ? (int64_t)k * h->m : 0) + (h->m - 1);

@@ -25,8 +25,11 @@ struct WorkerSel {
   uint32_t rank;     // 1-based rank still to find inside the current bucket
   uint32_t T;        // the k-th largest key
   uint32_t n_tie;    // elements equal to T that are kept (lowest indices first)
-  uint32_t done[3];  // finished-block counters of the three select passes
-  uint32_t pad[7];
+  uint32_t ties;     // candidates equal to T
+  uint32_t t_idx;    // a candidate equal to T is kept iff its index <= t_idx
+  uint32_t dense;    // 1: this worker's selection is made by the dense path
+  uint32_t done[4];  // finished-block counters: three select passes, the sample
+  uint32_t pad[3];
 };
 
 // Step counters (see GMC_STAT_* in gmc.h), unsigned 64-bit slots.
@@ -39,6 +42,9 @@ enum CounterSlot { kSteps = 0, kPairs = 1, kNnz = 2, kUnion = 3, kChanged = 4,
 // Device status bits (gmc_check).
 constexpr unsigned kStatusNonfinite = 1u;
 constexpr unsigned kStatusInternal = 2u;
+constexpr unsigned kStatusTimeout = 4u;     // a bounded wait gave up (see wait_bounded)
+constexpr int kChunksPerTile = 8;           // candidate sub-chunks per tile: one per warp
+constexpr uint32_t kUnsent = 0x80000000u;   // index mark of a candidate that was not sent
 
 __device__ __forceinline__ uint32_t mag_key(float v) {
   return __float_as_uint(v) & kKeyMask;
@@ -50,8 +56,22 @@ __device__ __forceinline__ bool is_nonfinite(float v) {
 __device__ __forceinline__ float accumulate(float e, float g, float c, float dl) {
   return __fsub_rn(__fadd_rn(e, g), __fmul_rn(c, dl));
 }
+// The dense path decides this worker's C(v) when its sampled filter missed:
+// fewer candidates than k, a candidate region overflowed, or too many ties.
 __device__ __forceinline__ bool needs_dense(const WorkerSel& s, uint32_t ksel, uint32_t cap) {
-  return s.count < ksel || s.count > cap;
+  return s.count < ksel || s.count > cap || s.dense != 0;
+}
+// Membership of a candidate in C(v): above the k-th key, or equal to it with
+// an index no larger than the last tie kept (ties go to the lower index).
+__device__ __forceinline__ bool selected(uint32_t key, uint32_t j, uint32_t T, uint32_t t_idx) {
+  return key > T || (key == T && j <= t_idx);
+}
+// Shared-memory histogram increment, aggregated over the lanes of a warp that
+// hit the same bucket (all lanes of the warp must call it; inactive: bin < 0).
+__device__ __forceinline__ void warp_hist_add(uint32_t* hist, int bin) {
+  const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+  const int leader = __ffs(peers) - 1;
+  if (bin >= 0 && (int)(threadIdx.x & 31) == leader) atomicAdd(&hist[bin], (uint32_t)__popc(peers));
 }
 __device__ __forceinline__ uint32_t lanemask_lt() {
   uint32_t m;
@@ -117,6 +137,65 @@ __device__ __forceinline__ void block_find_from_top(const uint32_t* hist, int nb
     }
   }
   __syncthreads();
+}
+
+// ---------------------------------------------------------------------------
+// mbarrier and bulk-copy primitives (inline PTX, sm_90+ / sm_103a)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;"
+               ::"r"(smem_addr(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Wait for the phase with the given parity to complete, giving up after about
+// two seconds (returns false): a wait never hangs the GPU.
+__device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_ns() - t0 > 2000000000ull) return false;
+  }
+  return true;
+}
+// Order this thread's generic-proxy shared-memory accesses before later
+// async-proxy (bulk copy) accesses to the same memory.
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// Bulk copy global -> this CTA's shared memory, completing on `bar` (tx bytes).
+// dst, src 16-byte aligned; bytes a multiple of 16.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
 }
 
 }  // namespace gmc

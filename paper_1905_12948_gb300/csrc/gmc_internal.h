@@ -11,6 +11,14 @@
 namespace gmc {
 
 // Arguments of the top-k kernels (one block describing the step).
+//
+// C(e_{t+1/2,k}) is kept as index-sorted (index, value) pairs in sub-chunks:
+// sub-chunk (k, tile, w) holds worker k's candidates of the w-th of the
+// kChunksPerTile equal parts of the tile, in ascending index order, at
+// cand_idx/cand_val[k*cap + base .. + cnt). The accumulate pass writes every
+// candidate; the aggregate marks the ones not sent (index | kUnsent).
+// Buffers alternate between steps:
+// the previous step's sent pairs give the non-zero positions of w_t - w_{t-1}.
 struct TopkArgs {
   float* e;                  // residuals / accumulator, K rows of ld floats
   int64_t ld;                // row stride of e (multiple of the tile)
@@ -23,25 +31,27 @@ struct TopkArgs {
   int64_t n_tiles;
   int tile;                  // elements per tile
   uint32_t ksel;             // k
-  uint32_t cap;              // candidate capacity per worker
+  uint32_t cap;              // candidate slots per worker = regions * cap_region
+  int regions;               // candidate regions per worker: one per accumulate CTA (1 = shared)
+  uint32_t cap_region;       // slots per region
+  uint32_t* rcount;          // K x regions: candidates written in each region
   uint32_t sample_rank;      // rank of the sampled threshold
   int sample_chunks;         // 0 = sample every element
+  int sample_blocks;         // blocks per worker of the sample kernel
   int has_prev;              // a previous step exists (t > 0)
   int dense_mode;            // GMC_SELECT_DENSE
   WorkerSel* sel;            // K entries
-  uint32_t* cand_idx;        // K x cap
-  float* cand_val;           // K x cap
-  uint32_t* chunk_base;      // K x n_tiles
-  uint32_t* chunk_cnt;       // K x n_tiles
-  uint32_t* gt_cnt;          // K x n_tiles
-  uint32_t* eq_cnt;          // K x n_tiles
-  uint32_t* eq_before;       // K x n_tiles
-  uint32_t* ghist;           // K x kHistBins
-  const uint32_t* pos_prev;  // K x (n_tiles+1): previous step's per-tile offsets
-  const uint32_t* idx_prev;  // K x ksel: previous step's sorted indices
-  uint32_t* pos_cur;         // K x (n_tiles+1)
-  uint32_t* idx_cur;         // K x ksel
-  float* val_cur;            // K x ksel
+  uint32_t* ghist;           // K x kHistBins (zero between uses)
+  uint32_t* sample_keys;     // K x 8*kSampleChunks
+  uint32_t* big_tiles;       // [0]: count, then tile ids left to the block aggregate
+  uint32_t* cand_idx;        // current chunks: K x cap
+  float* cand_val;
+  uint32_t* chunk_base;      // K x n_tiles x kChunksPerTile
+  uint32_t* chunk_cnt;       // K x n_tiles x kChunksPerTile
+  uint32_t* mask;            // d: workers that sent each coordinate (bit k), zero between steps
+  const uint32_t* cand_idx_prev;    // previous step's sub-chunks
+  const uint32_t* chunk_base_prev;
+  const uint32_t* chunk_cnt_prev;
   Counters* step_ctr;
   unsigned* status;
 };
@@ -89,11 +99,11 @@ struct DetachArgs {
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_select_pass(const TopkArgs& A, int pass, int blocks_per_worker, cudaStream_t s);
+cudaError_t launch_ties(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s);
-cudaError_t launch_chunk_count(const TopkArgs& A, cudaStream_t s);
-cudaError_t launch_chunk_scan(const TopkArgs& A, cudaStream_t s);
-cudaError_t launch_chunk_write(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_aggregate(const TopkArgs& A, int grid, cudaStream_t s);
+cudaError_t launch_gather_selected(const TopkArgs& A, int k, uint32_t* idx_out, float* val_out,
+                                   cudaStream_t s);
 cudaError_t launch_rbgs_pick(const RbgsArgs& A, cudaStream_t s);
 cudaError_t launch_rbgs_step(const RbgsArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_rbgs_expand(const RbgsArgs& A, int k, uint32_t* idx_out, float* val_out,
@@ -104,10 +114,8 @@ cudaError_t launch_finalize(Counters* step, Counters* total, unsigned long long 
 
 // Occupancy-derived persistent grid sizes.
 int accumulate_blocks_per_sm(int tile);
-int aggregate_blocks_per_sm(int tile);
 int rbgs_blocks_per_sm();
 int accumulate_smem_bytes(int tile);
-int aggregate_smem_bytes(int tile);
 cudaError_t configure_topk_kernels();
 cudaError_t configure_rbgs_kernels();
 

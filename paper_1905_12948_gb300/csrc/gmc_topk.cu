@@ -1,19 +1,20 @@
-// Top-k path of one GMC step (Alg. 1 with the top-s compressor of Sec. 4):
+// Top-k path of one GMC step (Alg. 1 with the top-s compressor of Sec. 4).
 //
 //   sample      per worker, e_{t+1/2} at a stratified sample -> a threshold key
 //               theta below the k-th largest |v| with overwhelming probability
-//   accumulate  ONE dense pass: v = (e + g) - c*(w_t - w_{t-1}) written over e,
-//               and every v with key >= theta appended to the worker's candidate
-//               list in per-tile chunks that are sorted by index
-//   select x3   exact k-th largest key T among the candidates (radix digits of
-//               11, 10 and 10 bits), and how many ties at T are kept
+//   accumulate  ONE dense pass: v = (e + g) - c*(w_t - w_{t-1}) written over e;
+//               every v with key >= theta is appended to the worker's chunk of
+//               its tile, in index order
+//   select x3   the exact k-th largest key T among the candidates (radix digits
+//               of 11, 10 and 10 bits) and how many ties at T are kept
+//   ties        only when more candidates equal T than are kept: the largest
+//               index of a kept tie (ties go to the lower index)
 //   dense       for a worker whose filter missed (too few or too many
-//               candidates): the exact select and compaction over dense v
-//   compact x3  per-tile counts, per-worker scan, index-ordered write of
-//               C(v) = (index, value) pairs
-//   aggregate   per tile: sum the workers' values in ascending worker order,
-//               e = 0 at sent coordinates, w -= (eta/K) * sum on the union,
-//               store w_{t+1} - w_t for the next step's accumulator
+//               candidates): exact select over dense v, chunks rewritten
+//   aggregate   per tile: keep the sent pairs in each chunk (in place: the
+//               chunks are C(e_{t+1/2,k})), e = +0 at sent coordinates, sum
+//               the workers' values in ascending worker order from +0,
+//               w -= (eta/K) * sum on the union, store w_{t+1} - w_t
 //
 // Keys are the fp32 bit patterns with the sign cleared (monotone in |v|); the
 // selected set is the first k elements under (key descending, index ascending).
@@ -21,6 +22,8 @@
 
 namespace gmc {
 namespace {
+
+constexpr int kMaxK = 64;  // workers supported by the top-k kernels
 
 __device__ __forceinline__ float4 load_g4(const float* __restrict__ g, int64_t j, int64_t d,
                                           int mode) {
@@ -52,185 +55,497 @@ __device__ __forceinline__ V warp_sum(V x) {
   return x;
 }
 
+__device__ __forceinline__ uint32_t warp_excl_scan(uint32_t x, uint32_t* total) {
+  const int lane = threadIdx.x & 31;
+  uint32_t incl = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  *total = __shfl_sync(0xffffffffu, incl, 31);
+  return incl - x;
+}
+
 // ---------------------------------------------------------------------------
-// sample: one block per worker
+// sample: blocks spread over the workers' samples; the last block of a worker
+// fixes two radix digits of the sample's r-th largest key.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kSampleThreads) k_sample(TopkArgs A) {
-  extern __shared__ uint32_t keys[];
+__global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   __shared__ uint32_t hist[kHistBins];
   __shared__ uint32_t ws[32];
-  __shared__ uint32_t s_bin, s_rank;
-  const int k = blockIdx.x;
+  __shared__ uint32_t s_last, s_bin, s_rank;
+  const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
+  if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) A.big_tiles[0] = 0;
   if (A.dense_mode) {
-    if (threadIdx.x == 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
       S.theta = kNoCandidate;
       S.count = 0;
+      S.dense = 0;
     }
     return;
   }
   const float* ek = A.e + (int64_t)k * A.ld;
   const float* gk = A.grads + (int64_t)k * A.d;
-  int n_s;
-  if (A.sample_chunks == 0) {
-    n_s = (int)A.d;
-    for (int j = threadIdx.x; j < n_s; j += blockDim.x)
-      keys[j] = mag_key(accumulate(ek[j], gk[j], A.c, A.dlt[j]));
-  } else {
-    n_s = A.sample_chunks * 8;
-    for (int ch = threadIdx.x; ch < A.sample_chunks; ch += blockDim.x) {
-      const int64_t p = ((int64_t)ch * A.d / A.sample_chunks) & ~int64_t(7);
+  uint32_t* keys = A.sample_keys + (int64_t)k * (8 * kSampleChunks);
+  const int n_s = A.sample_chunks ? A.sample_chunks * 8 : (int)A.d;
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0;
+  __syncthreads();
+  const int per = (n_s + gridDim.x - 1) / gridDim.x;
+  const int i_lo = blockIdx.x * per;
+  const int i_hi = min(n_s, i_lo + per);
+  for (int i0 = i_lo; i0 < i_hi; i0 += 8 * blockDim.x) {
+    float ev[8], gv[8], dv[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
-        keys[ch * 8 + i] = mag_key(accumulate(ek[p + i], gk[p + i], A.c, A.dlt[p + i]));
+    for (int q = 0; q < 8; ++q) {
+      const int i = i0 + q * blockDim.x + threadIdx.x;
+      ev[q] = gv[q] = dv[q] = 0.f;
+      if (i < i_hi) {
+        int64_t j = i;
+        if (A.sample_chunks) {
+          const int64_t ch = i >> 3;
+          j = ((ch * A.d / A.sample_chunks) & ~int64_t(7)) + (i & 7);
+        }
+        ev[q] = ek[j];
+        gv[q] = gk[j];
+        dv[q] = A.dlt[j];
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int i = i0 + q * blockDim.x + threadIdx.x;
+      int bin = -1;
+      if (i < i_hi) {
+        const uint32_t key = mag_key(accumulate(ev[q], gv[q], A.c, dv[q]));
+        keys[i] = key;
+        bin = (int)(key >> 20);
+      }
+      warp_hist_add(hist, bin);
     }
   }
-  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0;
+  __syncthreads();
+  uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
+    if (hist[b]) atomicAdd(&gh[b], hist[b]);
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[3], 1u) == gridDim.x - 1) ? 1u : 0u;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) {
+    hist[b] = __ldcg(&gh[b]);
+    gh[b] = 0;
+  }
   if (threadIdx.x == 0) {
+    S.done[3] = 0;
     s_bin = 0;
     s_rank = 0;
   }
   __syncthreads();
   uint32_t r = A.sample_rank < (uint32_t)n_s ? A.sample_rank : (uint32_t)n_s;
-  for (int i = threadIdx.x; i < n_s; i += blockDim.x) atomicAdd(&hist[keys[i] >> 20], 1u);
-  __syncthreads();
   block_find_from_top(hist, kHistBins, r, ws, &s_bin, &s_rank);
   const uint32_t b1 = s_bin;
   r = s_rank;
-  __syncthreads();
   for (int b = threadIdx.x; b < 1024; b += blockDim.x) hist[b] = 0;
   __syncthreads();
-  for (int i = threadIdx.x; i < n_s; i += blockDim.x) {
-    const uint32_t key = keys[i];
-    if ((key >> 20) == b1) atomicAdd(&hist[(key >> 10) & 1023u], 1u);
+  // second digit over all the worker's sample keys (n_s is a multiple of 8 or
+  // at most kSampleAll; keys are 16-byte aligned): 16 keys per thread per round
+  for (int i0 = 0; i0 < n_s; i0 += 16 * blockDim.x) {
+    uint32_t kv[16];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + (q * blockDim.x + threadIdx.x) * 4;
+      if (i + 3 < n_s) {
+        const uint4 x = __ldcg(reinterpret_cast<const uint4*>(keys + i));
+        kv[4 * q] = x.x; kv[4 * q + 1] = x.y; kv[4 * q + 2] = x.z; kv[4 * q + 3] = x.w;
+      } else {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) kv[4 * q + t] = i + t < n_s ? __ldcg(keys + i + t) : 0xffffffffu;
+      }
+    }
+#pragma unroll
+    for (int t = 0; t < 16; ++t) {
+      const uint32_t key = kv[t];
+      warp_hist_add(hist, (key != 0xffffffffu && (key >> 20) == b1) ? (int)((key >> 10) & 1023u) : -1);
+    }
   }
   __syncthreads();
   block_find_from_top(hist, 1024, r, ws, &s_bin, &s_rank);
   if (threadIdx.x == 0) {
-    S.theta = (b1 << 20) | (s_bin << 10);
+    // capped at the Inf key: every non-finite value is a candidate (and counted there)
+    S.theta = min((b1 << 20) | (s_bin << 10), 0x7f800000u);
     S.count = 0;
+    S.dense = 0;
   }
 }
 
 // ---------------------------------------------------------------------------
-// accumulate + filter: the one dense pass. Persistent blocks walk the tiles;
-// each tile is done for all K workers so the staged w_t - w_{t-1} is reused.
+// accumulate + filter. Each warp owns one sub-tile (1/kChunksPerTile) of every
+// tile; for each worker it writes v over e and appends its candidates as one
+// index-sorted sub-chunk, reserved at once -- warps never wait for each other.
 // ---------------------------------------------------------------------------
+// w_t - w_{t-1} on one warp's sub-tile [sub0, sub0 + n) into dlw: non-zero only
+// where the previous step sent pairs, listed by its sub-chunks (k', tile, w).
+__device__ __forceinline__ void stage_delta_warp(const TopkArgs& A, int64_t tile, int w,
+                                                 uint32_t sub0, int n, float* dlw, int lane) {
+  for (int i = lane; i < n / 4; i += 32)
+    reinterpret_cast<float4*>(dlw)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  __syncwarp();
+  if (A.has_prev) {
+    for (int k0 = 0; k0 < A.K; k0 += 32) {
+      const int kk = k0 + lane;
+      uint32_t base = 0, cnt = 0;
+      if (kk < A.K) {
+        const int64_t c = ((int64_t)kk * A.n_tiles + tile) * kChunksPerTile + w;
+        base = A.chunk_base_prev[c];
+        cnt = A.chunk_cnt_prev[c];
+      }
+      uint32_t total;
+      const uint32_t pre = warp_excl_scan(cnt, &total);
+      for (uint32_t e0 = 0; e0 < total; e0 += 32) {
+        const uint32_t e = e0 + lane;
+        int src = 0;  // the last lane whose non-empty sub-chunk starts at or before e
+#pragma unroll 1
+        for (int l = 1; l < 32; ++l) {
+          const uint32_t pl = __shfl_sync(0xffffffffu, pre, l);
+          const uint32_t cl = __shfl_sync(0xffffffffu, cnt, l);
+          if (cl && pl <= e) src = l;
+        }
+        const uint32_t b = __shfl_sync(0xffffffffu, base, src);
+        const uint32_t p = __shfl_sync(0xffffffffu, pre, src);
+        if (e < total) {
+          const uint32_t at = b + (e - p);
+          if (at < A.cap) {
+            const uint32_t j = A.cand_idx_prev[(int64_t)(k0 + src) * A.cap + at];
+            if (!(j & kUnsent)) {
+              const int64_t l = (int64_t)j - sub0;
+              if (l >= 0 && l < n) dlw[l] = A.dlt[j];
+              else atomicOr(A.status, kStatusInternal);
+            }
+          }
+        }
+      }
+    }
+    __syncwarp();
+    // w_t - w_{t-1} has been read for this sub-tile; clear it here (this step's
+    // aggregate writes w_{t+1} - w_t)
+    for (int l = lane; l < n; l += 32)
+      if (dlw[l] != 0.f) A.dlt[sub0 + l] = 0.f;
+  }
+  __syncwarp();
+}
+
+// Candidate flags (bit i: value i is a candidate) of 4 consecutive values at
+// sub-tile offset l; `lim` = valid values in the sub-tile (all when it is full).
+__device__ __forceinline__ uint32_t cand_bits(const float v[4], int l, int lim, uint32_t theta) {
+  uint32_t bits = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    bits |= ((mag_key(v[i]) >= theta) && (l + i < lim) ? 1u : 0u) << i;
+  return bits;
+}
+
+// Write one group's candidates (index order: lane-major, element-minor) at
+// pos; counts the non-finite ones (theta never exceeds the Inf key).
+__device__ __forceinline__ void write_group(const float v[4], uint32_t j, uint32_t bits, uint32_t lt,
+                                            uint32_t& pos, uint32_t end, uint32_t* ci, float* cv,
+                                            uint32_t& nonfinite) {
+  const uint32_t n = __popc(bits);
+  if (!__any_sync(0xffffffffu, n != 0)) return;
+  uint32_t incl = n;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if ((int)(threadIdx.x & 31) >= o) incl += y;
+  }
+  uint32_t o = pos + incl - n;
+  pos += __shfl_sync(0xffffffffu, incl, 31);
+  (void)lt;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if ((bits >> i) & 1u) {
+      if (o < end) {
+        ci[o] = j + i;
+        cv[o] = v[i];
+      }
+      nonfinite += is_nonfinite(v[i]) ? 1u : 0u;
+      ++o;
+    }
+  }
+}
+
+// load/store version for small tiles; candidates share one region per worker
 template <int U>
 __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
   constexpr int SUB = 128 * U;       // elements per warp and worker
   constexpr int T = kWarps * SUB;    // elements per tile
   extern __shared__ __align__(16) unsigned char smem[];
-  float* dl = reinterpret_cast<float*>(smem);
-  uint32_t* st_idx = reinterpret_cast<uint32_t*>(dl + T);
-  float* st_val = reinterpret_cast<float*>(st_idx + T);
-  __shared__ uint32_t s_wcnt[kWarps], s_woff[kWarps], s_base;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* dlw = reinterpret_cast<float*>(smem) + warp * SUB;
   const uint32_t lt = lanemask_lt();
   uint32_t nonfinite = 0;
 
   for (int64_t tile = blockIdx.x; tile < A.n_tiles; tile += gridDim.x) {
-    const int64_t t0 = tile * T;
-    for (int i = threadIdx.x; i < T / 4; i += kThreads)
-      reinterpret_cast<float4*>(dl)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    __syncthreads();
-    if (A.has_prev) {
-      // w_t - w_{t-1} is non-zero only on the previous step's union of sent
-      // coordinates; scatter it into the tile from the previous sorted lists.
-      for (int kk = 0; kk < A.K; ++kk) {
-        const uint32_t* pp = A.pos_prev + (int64_t)kk * (A.n_tiles + 1);
-        const uint32_t lo = pp[tile], hi = pp[tile + 1];
-        const uint32_t* ip = A.idx_prev + (int64_t)kk * A.ksel;
-        for (uint32_t i = lo + threadIdx.x; i < hi && i < A.ksel; i += kThreads) {
-          const uint32_t j = ip[i];
-          if ((uint64_t)(j - t0) < (uint64_t)T) dl[j - t0] = A.dlt[j];
-          else atomicOr(A.status, kStatusInternal);
-        }
-      }
-    }
-    __syncthreads();
-
+    const uint32_t s0 = (uint32_t)(tile * T) + warp * SUB;
+    stage_delta_warp(A, tile, warp, s0, SUB, dlw, lane);
+    const int64_t rem = A.d - (int64_t)s0;
+    const int lim = rem < SUB ? (int)rem : SUB;
     for (int k = 0; k < A.K; ++k) {
       const uint32_t theta = A.sel[k].theta;
-      float* ek = A.e + (int64_t)k * A.ld;
+      float* ekt = A.e + (int64_t)k * A.ld + s0;
       const float* gk = A.grads + (int64_t)k * A.d;
       const int gm = g_mode(gk);
-      const int64_t wbase = t0 + warp * SUB;
       float4 ev[U], gv[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const int64_t j = wbase + u * 128 + lane * 4;
-        ev[u] = __ldcs(reinterpret_cast<const float4*>(ek + j));
-        gv[u] = load_g4(gk, j, A.d, gm);
+        const int l = u * 128 + lane * 4;
+        ev[u] = __ldcs(reinterpret_cast<const float4*>(ekt + l));
+        gv[u] = load_g4(gk, (int64_t)s0 + l, A.d, gm);
       }
-      uint32_t wcnt = 0;
-      uint32_t* sti = st_idx + warp * SUB;
-      float* stv = st_val + warp * SUB;
+      float v[U][4];
+      uint32_t bits[U];
+      uint32_t nloc = 0;
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const int64_t j = wbase + u * 128 + lane * 4;
-        const float4 d4 = *reinterpret_cast<const float4*>(dl + (j - t0));
-        float v[4];
-        v[0] = accumulate(ev[u].x, gv[u].x, A.c, d4.x);
-        v[1] = accumulate(ev[u].y, gv[u].y, A.c, d4.y);
-        v[2] = accumulate(ev[u].z, gv[u].z, A.c, d4.z);
-        v[3] = accumulate(ev[u].w, gv[u].w, A.c, d4.w);
-        __stcs(reinterpret_cast<float4*>(ek + j), make_float4(v[0], v[1], v[2], v[3]));
-        bool f[4];
-        uint32_t bal[4];
-        uint32_t before = 0, total = 0;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const bool in = j + i < A.d;
-          f[i] = in && mag_key(v[i]) >= theta;
-          nonfinite += (in && is_nonfinite(v[i])) ? 1u : 0u;
-          bal[i] = __ballot_sync(0xffffffffu, f[i]);
-          before += __popc(bal[i] & lt);
-          total += __popc(bal[i]);
-        }
-        uint32_t o = wcnt + before;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          if (f[i]) {
-            sti[o] = (uint32_t)(j + i);
-            stv[o] = v[i];
-            ++o;
-          }
-        }
-        wcnt += total;
+        const int l = u * 128 + lane * 4;
+        const float4 d4 = *reinterpret_cast<const float4*>(dlw + l);
+        v[u][0] = accumulate(ev[u].x, gv[u].x, A.c, d4.x);
+        v[u][1] = accumulate(ev[u].y, gv[u].y, A.c, d4.y);
+        v[u][2] = accumulate(ev[u].z, gv[u].z, A.c, d4.z);
+        v[u][3] = accumulate(ev[u].w, gv[u].w, A.c, d4.w);
+        __stcs(reinterpret_cast<float4*>(ekt + l), make_float4(v[u][0], v[u][1], v[u][2], v[u][3]));
+        bits[u] = cand_bits(v[u], l, lim, theta);
+        nloc += __popc(bits[u]);
       }
-      if (lane == 0) s_wcnt[warp] = wcnt;
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        uint32_t tot = 0;
+      const uint32_t cnt = __reduce_add_sync(0xffffffffu, nloc);
+      uint32_t base = 0;
+      if (lane == 0 && cnt) base = atomicAdd(&A.sel[k].count, cnt);
+      base = __shfl_sync(0xffffffffu, base, 0);
+      if (cnt) {
+        uint32_t pos = base;
+        uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+        float* cv = A.cand_val + (int64_t)k * A.cap;
 #pragma unroll
-        for (int w = 0; w < kWarps; ++w) {
-          s_woff[w] = tot;
-          tot += s_wcnt[w];
-        }
-        const uint32_t base = tot ? atomicAdd(&A.sel[k].count, tot) : 0u;
-        s_base = base;
-        A.chunk_base[(int64_t)k * A.n_tiles + tile] = base;
-        A.chunk_cnt[(int64_t)k * A.n_tiles + tile] = tot;
+        for (int u = 0; u < U; ++u)
+          write_group(v[u], s0 + u * 128 + lane * 4, bits[u], lt, pos, A.cap, ci, cv, nonfinite);
       }
-      __syncthreads();
-      const uint32_t base = s_base + s_woff[warp];
-      uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
-      float* cv = A.cand_val + (int64_t)k * A.cap;
-      for (uint32_t i = lane; i < wcnt; i += 32) {
-        const uint32_t p = base + i;
-        if (p < A.cap) {
-          ci[p] = sti[i];
-          cv[p] = stv[i];
-        }
+      if (lane == 0) {
+        const int64_t c = ((int64_t)k * A.n_tiles + tile) * kChunksPerTile + warp;
+        A.chunk_base[c] = base;
+        A.chunk_cnt[c] = cnt;
       }
-      __syncwarp();
     }
-    __syncthreads();
   }
   if (nonfinite) {
     atomicOr(A.status, kStatusNonfinite);
     atomicAdd(&A.step_ctr->v[kNonfinite], (unsigned long long)nonfinite);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// bulk-copy version (tiles of 4096). One persistent CTA per SM. A producer
+// thread streams each (tile, worker) item's e and g into a ring of shared-
+// memory stages with cp.async.bulk; eight consumer warps, each owning 512
+// elements of the tile, read their part, release the stage, store v over e
+// and reserve their sub-chunk in this CTA's region of the candidate buffer
+// with a shared-memory atomic. Producer and consumers meet only at mbarriers
+// and every wait is bounded.
+// ---------------------------------------------------------------------------
+namespace bulk {
+constexpr int kT = 4096;
+constexpr int kStages = 6;
+constexpr int kConsumers = kChunksPerTile;
+constexpr int kSub = kT / kConsumers;      // 512
+constexpr int kGLen = kT + 8;              // g stage: up to 3 leading floats of misalignment
+constexpr int kThreadsAll = (kConsumers + 1) * 32;
+struct Smem {
+  float e[kStages][kT];
+  float g[kStages][kGLen];
+  float dl[kConsumers][kSub];
+  uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
+  uint64_t empty[kStages];                 // all consumer warps read the stage (8 arrivals)
+  int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
+  uint32_t rcnt[kMaxK];                    // candidates this CTA wrote per worker (its region)
+  uint32_t theta[kMaxK];
+};
+}  // namespace bulk
+
+__global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkArgs A) {
+  using namespace bulk;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kConsumers);
+    }
+    fence_mbar_init();
+  }
+  for (int kk = threadIdx.x; kk < kMaxK; kk += blockDim.x) {
+    sm.rcnt[kk] = 0;
+    sm.theta[kk] = kk < A.K ? A.sel[kk].theta : kNoCandidate;
+  }
+  __syncthreads();
+
+  if (warp == kConsumers) {
+    // ---- producer ----
+    if (lane != 0) return;
+    const char* g_lo = reinterpret_cast<const char*>(A.grads);
+    const char* g_hi = reinterpret_cast<const char*>(A.grads + (int64_t)A.K * A.d);
+    uint32_t item = 0;
+    bool ok = true;
+    for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+      const int64_t j0 = tile * kT;
+      const int64_t nvalid = A.d - j0 < kT ? A.d - j0 : kT;
+      for (int k = 0; k < A.K; ++k, ++item) {
+        const uint32_t s = item % kStages, r = item / kStages;
+        if (r > 0 && !wait_bounded(&sm.empty[s], (r - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        const float* esrc = A.e + (int64_t)k * A.ld + j0;
+        const uintptr_t ga = reinterpret_cast<uintptr_t>(A.grads + (int64_t)k * A.d + j0);
+        const uint32_t off = (uint32_t)(ga & 15) >> 2;
+        const char* gsrc = reinterpret_cast<const char*>(ga - off * 4);
+        const uint32_t gbytes = (uint32_t)(((nvalid + off) * 4 + 15) & ~int64_t(15));
+        const bool gbulk = (ga & 3) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
+        sm.gmeta[s] = gbulk ? (int32_t)off : -1;
+        mbar_arrive_expect_tx(&sm.full[s], kT * 4 + (gbulk ? gbytes : 0));
+        bulk_load(sm.e[s], esrc, kT * 4, &sm.full[s]);
+        if (gbulk) bulk_load(sm.g[s], gsrc, gbytes, &sm.full[s]);
+      }
+    }
+    if (!ok) {
+      atomicOr(A.status, kStatusTimeout);
+      // let the copies already issued land before the CTA's shared memory goes away
+      const uint32_t first = item > (uint32_t)kStages ? item - kStages : 0u;
+      for (uint32_t i = first; i < item; ++i) wait_bounded(&sm.full[i % kStages], (i / kStages) & 1);
+    }
+    return;
+  }
+
+  // ---- consumers ----
+  const uint32_t lt = lanemask_lt();
+  float* dlw = sm.dl[warp];
+  const uint32_t region0 = blockIdx.x * A.cap_region;
+  const uint32_t region_end = region0 + A.cap_region;
+  uint32_t nonfinite = 0;
+  uint32_t item = 0;
+  bool ok = true;
+  for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+    const uint32_t s0 = (uint32_t)(tile * kT) + warp * kSub;
+    stage_delta_warp(A, tile, warp, s0, kSub, dlw, lane);
+    const int64_t rem = A.d - (int64_t)s0;
+    const int lim = rem < kSub ? (int)rem : kSub;
+    const bool full = lim == kSub;
+    for (int k = 0; k < A.K; ++k, ++item) {
+      const uint32_t s = item % kStages, r = item / kStages;
+      if (!wait_bounded(&sm.full[s], r & 1)) {
+        ok = false;
+        break;
+      }
+      const int32_t off = sm.gmeta[s];
+      const float* se = sm.e[s] + warp * kSub;
+      const float* sg = sm.g[s] + (off > 0 ? off : 0) + warp * kSub;
+      float v[kSub / 128][4];
+#pragma unroll
+      for (int u = 0; u < kSub / 128; ++u) {
+        const int l = u * 128 + lane * 4;
+        const float4 e4 = *reinterpret_cast<const float4*>(se + l);
+        float4 g4;
+        if (off == 0) {
+          g4 = *reinterpret_cast<const float4*>(sg + l);
+        } else if (off == 2) {
+          const float2 a = *reinterpret_cast<const float2*>(sg + l);
+          const float2 b = *reinterpret_cast<const float2*>(sg + l + 2);
+          g4 = make_float4(a.x, a.y, b.x, b.y);
+        } else if (off > 0) {
+          g4 = make_float4(sg[l], sg[l + 1], sg[l + 2], sg[l + 3]);
+        } else {
+          const float* gk = A.grads + (int64_t)k * A.d;
+          g4 = load_g4(gk, (int64_t)s0 + l, A.d, g_mode(gk));
+        }
+        if (!full && off >= 0) {  // past d the stage holds bytes of no meaning
+          if (l >= lim) g4.x = 0.f;
+          if (l + 1 >= lim) g4.y = 0.f;
+          if (l + 2 >= lim) g4.z = 0.f;
+          if (l + 3 >= lim) g4.w = 0.f;
+        }
+        const float4 d4 = *reinterpret_cast<const float4*>(dlw + l);
+        v[u][0] = accumulate(e4.x, g4.x, A.c, d4.x);
+        v[u][1] = accumulate(e4.y, g4.y, A.c, d4.y);
+        v[u][2] = accumulate(e4.z, g4.z, A.c, d4.z);
+        v[u][3] = accumulate(e4.w, g4.w, A.c, d4.w);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.empty[s]);  // this warp is done reading stage s
+      const uint32_t theta = sm.theta[k];
+      float* ekt = A.e + (int64_t)k * A.ld + s0;
+      uint32_t bits[kSub / 128];
+      uint32_t nloc = 0;
+#pragma unroll
+      for (int u = 0; u < kSub / 128; ++u) {
+        const int l = u * 128 + lane * 4;
+        __stcs(reinterpret_cast<float4*>(ekt + l), make_float4(v[u][0], v[u][1], v[u][2], v[u][3]));
+        bits[u] = cand_bits(v[u], l, lim, theta);
+        nloc += __popc(bits[u]);
+      }
+      const uint32_t cnt = __reduce_add_sync(0xffffffffu, nloc);
+      uint32_t base = region0;
+      if (cnt) {
+        uint32_t used = 0;
+        if (lane == 0) {
+          used = atomicAdd(&sm.rcnt[k], cnt);
+          if (used + cnt > A.cap_region) A.sel[k].dense = 1;  // region full: dense path
+        }
+        base = region0 + __shfl_sync(0xffffffffu, used, 0);
+        uint32_t pos = base;
+        uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+        float* cv = A.cand_val + (int64_t)k * A.cap;
+#pragma unroll
+        for (int u = 0; u < kSub / 128; ++u)
+          write_group(v[u], s0 + u * 128 + lane * 4, bits[u], lt, pos, region_end, ci, cv, nonfinite);
+      }
+      if (lane == 0) {
+        const int64_t c = ((int64_t)k * A.n_tiles + tile) * kChunksPerTile + warp;
+        A.chunk_base[c] = base;
+        A.chunk_cnt[c] = cnt;
+      }
+    }
+  }
+  if (!ok) atomicOr(A.status, kStatusTimeout);
+  if (nonfinite) {
+    atomicOr(A.status, kStatusNonfinite);
+    atomicAdd(&A.step_ctr->v[kNonfinite], (unsigned long long)nonfinite);
+  }
+  // every consumer warp is past its last reservation: publish the region counts
+  asm volatile("bar.sync 1, %0;" ::"r"(kConsumers * 32) : "memory");
+  if (warp == 0) {
+    for (int kk = lane; kk < A.K; kk += 32) {
+      const uint32_t n = sm.rcnt[kk];
+      A.rcount[(int64_t)kk * A.regions + blockIdx.x] = n < A.cap_region ? n : A.cap_region;
+      if (n) atomicAdd(&A.sel[kk].count, n);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Candidate ranges of a worker: one per region of the bulk pass, or [0, count)
+// split evenly when the candidates share one region. Part p of nparts.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void candidate_part(const TopkArgs& A, int k, int p, int nparts,
+                                               uint32_t* lo, uint32_t* hi) {
+  if (A.regions == 1) {
+    const uint32_t cnt = min(A.sel[k].count, A.cap);
+    const uint32_t per = ((cnt + nparts - 1) / nparts + 3) & ~3u;
+    *lo = min(cnt, (uint32_t)p * per);
+    *hi = min(cnt, *lo + per);
+  } else {
+    *lo = (uint32_t)p * A.cap_region;
+    *hi = *lo + A.rcount[(int64_t)k * A.regions + p];
   }
 }
 
@@ -248,15 +563,38 @@ __global__ void __launch_bounds__(kThreads) k_select_pass(TopkArgs A) {
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
   if (needs_dense(S, A.ksel, A.cap)) return;
-  const uint32_t cnt = S.count;
   const uint32_t prefix = S.prefix;
   for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
   __syncthreads();
   const float* cv = A.cand_val + (int64_t)k * A.cap;
-  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < cnt; i += gridDim.x * blockDim.x) {
-    const uint32_t key = mag_key(cv[i]);
-    if (PASS == 0 || (key >> (shift + 10)) == prefix)
-      atomicAdd(&h[(key >> shift) & (nbins - 1)], 1u);
+  const int nparts = A.regions == 1 ? (int)gridDim.x : A.regions;
+  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+    uint32_t lo, hi;
+    candidate_part(A, k, part, nparts, &lo, &hi);
+    // 16 candidates per thread per round, 16-byte loads (lo is a multiple of 4)
+    for (uint32_t i0 = lo; i0 < hi; i0 += 16 * blockDim.x) {
+      float kv[16];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t i = i0 + (q * blockDim.x + threadIdx.x) * 4;
+        if (i + 3 < hi) {
+          const float4 x = *reinterpret_cast<const float4*>(cv + i);
+          kv[4 * q] = x.x; kv[4 * q + 1] = x.y; kv[4 * q + 2] = x.z; kv[4 * q + 3] = x.w;
+        } else {
+#pragma unroll
+          for (int t = 0; t < 4; ++t) kv[4 * q + t] = i + t < hi ? cv[i + t] : __uint_as_float(0xffffffffu);
+        }
+      }
+#pragma unroll
+      for (int t = 0; t < 16; ++t) {
+        const uint32_t raw = __float_as_uint(kv[t]);
+        const uint32_t key = raw & kKeyMask;
+        int bin = -1;
+        if (raw != 0xffffffffu && (PASS == 0 || (key >> (shift + 10)) == prefix))
+          bin = (int)((key >> shift) & (nbins - 1));
+        warp_hist_add(h, bin);
+      }
+    }
   }
   __syncthreads();
   uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
@@ -291,13 +629,76 @@ __global__ void __launch_bounds__(kThreads) k_select_pass(TopkArgs A) {
     } else {
       S.T = (prefix << 10) | s_bin;
       S.n_tie = s_rank;
+      S.ties = h[s_bin];
+      S.t_idx = 0xffffffffu;  // every tie kept, unless k_ties narrows it
     }
   }
 }
 
 // ---------------------------------------------------------------------------
-// dense exact select + compaction for workers whose filter missed; one block
-// per worker (a rare path: correct for any input, not fast).
+// ties: when more candidates equal T than are kept, the kept ones are the
+// n_tie lowest indices; t_idx = the largest of them.
+// ---------------------------------------------------------------------------
+constexpr int kTieCap = 8192;
+
+__global__ void __launch_bounds__(1024) k_ties(TopkArgs A) {
+  const int k = blockIdx.x;
+  WorkerSel& S = A.sel[k];
+  if (needs_dense(S, A.ksel, A.cap) || S.ties == S.n_tie) return;
+  __shared__ uint32_t tie_idx[kTieCap];
+  __shared__ uint32_t h[kHistBins];
+  __shared__ uint32_t ws[32];
+  __shared__ uint32_t s_n, s_bin, s_rank;
+  if (threadIdx.x == 0) s_n = 0;
+  __syncthreads();
+  const uint32_t T = S.T;
+  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const float* cv = A.cand_val + (int64_t)k * A.cap;
+  const int nparts = A.regions;
+  for (int part = 0; part < nparts; ++part) {
+    uint32_t lo, hi;
+    candidate_part(A, k, part, nparts, &lo, &hi);
+    for (uint32_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+      if (mag_key(cv[i]) == T) {
+        const uint32_t p = atomicAdd(&s_n, 1u);
+        if (p < kTieCap) tie_idx[p] = ci[i];
+      }
+    }
+  }
+  __syncthreads();
+  const uint32_t n = s_n;
+  if (n > (uint32_t)kTieCap) {  // too many ties to rank here: the dense path takes over
+    if (threadIdx.x == 0) S.dense = 1;
+    return;
+  }
+  // the n_tie-th smallest index = the (n - n_tie + 1)-th largest (radix digits 11/10/10)
+  uint32_t r = n - S.n_tie + 1, prefix = 0;
+  for (int pass = 0; pass < 3; ++pass) {
+    const int nbins = pass == 0 ? 2048 : 1024;
+    const int shift = pass == 0 ? 20 : (pass == 1 ? 10 : 0);
+    for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
+    if (threadIdx.x == 0) {
+      s_bin = 0;
+      s_rank = 0;
+    }
+    __syncthreads();
+    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) {
+      const uint32_t x = tie_idx[i];
+      if (pass == 0 || (x >> (shift + 10)) == prefix)
+        atomicAdd(&h[(x >> shift) & (uint32_t)(nbins - 1)], 1u);
+    }
+    __syncthreads();
+    block_find_from_top(h, nbins, r, ws, &s_bin, &s_rank);
+    prefix = pass == 0 ? s_bin : ((prefix << 10) | s_bin);
+    r = s_rank;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) S.t_idx = prefix;
+}
+
+// ---------------------------------------------------------------------------
+// dense exact select + chunk rewrite for workers whose filter missed; one
+// block per worker (a rare path: correct for any input, not fast).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
   const int k = blockIdx.x;
@@ -319,10 +720,15 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
       s_rank = 0;
     }
     __syncthreads();
-    for (int64_t j = threadIdx.x; j < d; j += blockDim.x) {
-      const uint32_t key = mag_key(vk[j]);
-      if (pass == 0 || (key >> (shift + 10)) == prefix)
-        atomicAdd(&h[(key >> shift) & (uint32_t)(nbins - 1)], 1u);
+    for (int64_t j0 = 0; j0 < d; j0 += blockDim.x) {
+      const int64_t j = j0 + threadIdx.x;
+      int bin = -1;
+      if (j < d) {
+        const uint32_t key = mag_key(vk[j]);
+        if (pass == 0 || (key >> (shift + 10)) == prefix)
+          bin = (int)((key >> shift) & (uint32_t)(nbins - 1));
+      }
+      warp_hist_add(h, bin);
     }
     __syncthreads();
     block_find_from_top(h, nbins, r, ws, &s_bin, &s_rank);
@@ -333,12 +739,12 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
   const uint32_t T = prefix, n_tie = r;
 
   const int P = A.tile / (int)blockDim.x;  // consecutive elements per thread
-  uint32_t* pos = A.pos_cur + (int64_t)k * (A.n_tiles + 1);
-  uint32_t* oi = A.idx_cur + (int64_t)k * A.ksel;
-  float* ov = A.val_cur + (int64_t)k * A.ksel;
+  const int per_sub = (int)blockDim.x / kChunksPerTile;  // threads per sub-tile
+  __shared__ uint32_t sb[kChunksPerTile + 1];
+  uint32_t* oi = A.cand_idx + (int64_t)k * A.cap;
+  float* ov = A.cand_val + (int64_t)k * A.cap;
   uint32_t running = 0, eqrun = 0;
   for (int64_t tile = 0; tile < A.n_tiles; ++tile) {
-    if (threadIdx.x == 0) pos[tile] = running;
     const int64_t j0 = tile * A.tile + (int64_t)threadIdx.x * P;
     uint32_t g = 0, q = 0;
     for (int i = 0; i < P; ++i) {
@@ -355,6 +761,7 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
     const uint32_t taken0 = min(eqrun, n_tie);
     uint32_t qg = eqrun + (uint32_t)exc;
     uint32_t o = running + (uint32_t)(exc >> 32) + (min(qg, n_tie) - taken0);
+    if (threadIdx.x % per_sub == 0) sb[threadIdx.x / per_sub] = o;
     for (int i = 0; i < P; ++i) {
       const int64_t j = j0 + i;
       if (j < d) {
@@ -363,7 +770,7 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
         const bool take = key > T || (key == T && qg < n_tie);
         if (key == T) ++qg;
         if (take) {
-          if (o < A.ksel) {
+          if (o < A.ksel && o < A.cap) {
             oi[o] = (uint32_t)j;
             ov[o] = v;
           }
@@ -371,217 +778,184 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
         }
       }
     }
-    running += (uint32_t)(tot >> 32) + (min(eqrun + (uint32_t)tot, n_tie) - taken0);
+    const uint32_t in_tile = (uint32_t)(tot >> 32) + (min(eqrun + (uint32_t)tot, n_tie) - taken0);
+    if (threadIdx.x == 0) sb[kChunksPerTile] = running + in_tile;
+    __syncthreads();
+    if (threadIdx.x < kChunksPerTile) {
+      const int64_t c = ((int64_t)k * A.n_tiles + tile) * kChunksPerTile + threadIdx.x;
+      A.chunk_base[c] = sb[threadIdx.x];
+      A.chunk_cnt[c] = sb[threadIdx.x + 1] - sb[threadIdx.x];
+    }
+    running += in_tile;
     eqrun += (uint32_t)tot;
+    __syncthreads();
   }
   if (threadIdx.x == 0) {
-    pos[A.n_tiles] = running;
     if (running != A.ksel) atomicOr(A.status, kStatusInternal);
-    S.T = T;
-    S.n_tie = n_tie;
+    // the sub-chunks now hold exactly C(v): the aggregate keeps all of them
+    S.T = 0;
+    S.t_idx = 0xffffffffu;
+    S.dense = 1;
     atomicAdd(&A.step_ctr->v[kFallbacks], 1ull);
   }
 }
 
 // ---------------------------------------------------------------------------
-// compaction: per-tile counts, per-worker scan, index-ordered write
+// aggregate + update, over all candidates in parallel (no per-tile order):
+//   mark  a candidate not sent gets its index marked (index | kUnsent); a sent
+//         one sets its worker's bit in the coordinate's mask
+//   sum   the sent candidate of the lowest worker in the mask (the owner) adds
+//         the workers' values in ascending worker order from +0 -- each value
+//         is still in e[k][j], where the accumulate pass wrote it -- sets those
+//         e to +0, and applies w -= (eta/K) * sum, keeping w_{t+1} - w_t.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) k_chunk_count(TopkArgs A) {
+// Candidates of worker k, part p of nparts: the dense path's [0, k) when it
+// decided this worker, else a region of the bulk pass or a slice of [0, count).
+__device__ __forceinline__ void sent_part(const TopkArgs& A, int k, int p, int nparts,
+                                          uint32_t* lo, uint32_t* hi) {
+  if (A.sel[k].dense || A.regions == 1) {
+    const uint32_t n = A.sel[k].dense ? A.ksel : min(A.sel[k].count, A.cap);
+    const uint32_t per = (n + nparts - 1) / nparts;
+    *lo = min(n, (uint32_t)p * per);
+    *hi = min(n, *lo + per);
+  } else {
+    *lo = (uint32_t)p * A.cap_region;
+    *hi = *lo + (p < A.regions ? A.rcount[(int64_t)k * A.regions + p] : 0u);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A) {
   const int k = blockIdx.y;
-  const WorkerSel& S = A.sel[k];
-  if (needs_dense(S, A.ksel, A.cap)) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t tile = (int64_t)blockIdx.x * kWarps + warp;
-  if (tile >= A.n_tiles) return;
-  const int64_t ct = (int64_t)k * A.n_tiles + tile;
-  const uint32_t base = A.chunk_base[ct], cnt = A.chunk_cnt[ct], T = S.T;
-  const float* cv = A.cand_val + (int64_t)k * A.cap + base;
-  uint32_t g = 0, q = 0;
-  for (uint32_t i = lane; i < cnt; i += 32) {
-    const uint32_t key = mag_key(cv[i]);
-    g += key > T;
-    q += key == T;
+  const uint32_t T = A.sel[k].T, tidx = A.sel[k].t_idx;
+  const uint32_t bit = 1u << k;
+  uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const float* cv = A.cand_val + (int64_t)k * A.cap;
+  const int nparts = A.regions > 1 ? A.regions : (int)gridDim.x;
+  unsigned long long nnz = 0;
+  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+    uint32_t lo, hi;
+    sent_part(A, k, part, nparts, &lo, &hi);
+    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * blockDim.x) {
+      uint32_t jq[4];
+      float vq[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t i = i0 + q * blockDim.x + threadIdx.x;
+        jq[q] = i < hi ? ci[i] : 0xffffffffu;
+        vq[q] = i < hi ? cv[i] : 0.f;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t j = jq[q];
+        if (j >= (uint32_t)A.d) continue;
+        if (selected(mag_key(vq[q]), j, T, tidx)) {
+          atomicOr(&A.mask[j], bit);
+          nnz += (vq[q] != 0.f);
+        } else {
+          ci[i0 + q * blockDim.x + threadIdx.x] = j | kUnsent;
+        }
+      }
+    }
   }
-  g = warp_sum(g);
-  q = warp_sum(q);
-  if (lane == 0) {
-    A.gt_cnt[ct] = g;
-    A.eq_cnt[ct] = q;
-  }
+  nnz = warp_sum(nnz);
+  if ((threadIdx.x & 31) == 0 && nnz) atomicAdd(&A.step_ctr->v[kNnz], nnz);
 }
 
-__global__ void __launch_bounds__(1024) k_chunk_scan(TopkArgs A) {
-  const int k = blockIdx.x;
-  const WorkerSel& S = A.sel[k];
-  if (needs_dense(S, A.ksel, A.cap)) return;
-  __shared__ unsigned long long ws[32];
-  const uint32_t n_tie = S.n_tie;
-  uint32_t* pos = A.pos_cur + (int64_t)k * (A.n_tiles + 1);
-  const int64_t row = (int64_t)k * A.n_tiles;
-  uint32_t carry_g = 0, carry_q = 0;
-  for (int64_t t0 = 0; t0 < A.n_tiles; t0 += blockDim.x) {
-    const int64_t tile = t0 + threadIdx.x;
-    uint32_t g = 0, q = 0;
-    if (tile < A.n_tiles) {
-      g = A.gt_cnt[row + tile];
-      q = A.eq_cnt[row + tile];
-    }
-    const unsigned long long x = ((unsigned long long)g << 32) | q;
-    unsigned long long tot;
-    const unsigned long long exc = block_inclusive_scan<unsigned long long>(x, ws, &tot) - x;
-    const uint32_t gb = carry_g + (uint32_t)(exc >> 32);
-    const uint32_t qb = carry_q + (uint32_t)exc;
-    if (tile < A.n_tiles) {
-      pos[tile] = gb + min(qb, n_tie);
-      A.eq_before[row + tile] = qb;
-    }
-    carry_g += (uint32_t)(tot >> 32);
-    carry_q += (uint32_t)tot;
-  }
-  if (threadIdx.x == 0) {
-    const uint32_t total = carry_g + min(carry_q, n_tie);
-    pos[A.n_tiles] = total;
-    if (total != A.ksel) atomicOr(A.status, kStatusInternal);
-  }
-}
-
-__global__ void __launch_bounds__(kThreads) k_chunk_write(TopkArgs A) {
+__global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
   const int k = blockIdx.y;
-  const WorkerSel& S = A.sel[k];
-  if (needs_dense(S, A.ksel, A.cap)) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t tile = (int64_t)blockIdx.x * kWarps + warp;
-  if (tile >= A.n_tiles) return;
-  const uint32_t lt = lanemask_lt();
-  const int64_t ct = (int64_t)k * A.n_tiles + tile;
-  const uint32_t base = A.chunk_base[ct], cnt = A.chunk_cnt[ct];
-  const uint32_t T = S.T, n_tie = S.n_tie;
-  const uint32_t p = A.pos_cur[(int64_t)k * (A.n_tiles + 1) + tile];
-  const uint32_t eb = A.eq_before[ct];
-  uint32_t* oi = A.idx_cur + (int64_t)k * A.ksel + p;
-  float* ov = A.val_cur + (int64_t)k * A.ksel + p;
-  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap + base;
-  const float* cv = A.cand_val + (int64_t)k * A.cap + base;
-  uint32_t written = 0, eqseen = 0;
-  for (uint32_t i0 = 0; i0 < cnt; i0 += 32) {
-    const uint32_t i = i0 + lane;
-    const bool valid = i < cnt;
-    float v = 0.f;
-    uint32_t idx = 0, key = 0;
-    if (valid) {
-      v = cv[i];
-      idx = ci[i];
-      key = mag_key(v);
-    }
-    const bool gt = valid && key > T;
-    const bool eq = valid && key == T;
-    const uint32_t em = __ballot_sync(0xffffffffu, eq);
-    const bool take = gt || (eq && eb + eqseen + __popc(em & lt) < n_tie);
-    const uint32_t tm = __ballot_sync(0xffffffffu, take);
-    if (take) {
-      const uint32_t o = written + __popc(tm & lt);
-      if (p + o < A.ksel) {
-        oi[o] = idx;
-        ov[o] = v;
-      } else {
-        atomicOr(A.status, kStatusInternal);
-      }
-    }
-    written += __popc(tm);
-    eqseen += __popc(em);
-  }
-}
-
-// ---------------------------------------------------------------------------
-// aggregate + update, one tile at a time (persistent blocks)
-// ---------------------------------------------------------------------------
-template <int U>
-__global__ void __launch_bounds__(kThreads) k_aggregate(TopkArgs A) {
-  constexpr int T = kWarps * 128 * U;
-  extern __shared__ __align__(16) unsigned char smem[];
-  float* s_acc = reinterpret_cast<float*>(smem);
-  uint16_t* ulist = reinterpret_cast<uint16_t*>(s_acc + T);
-  uint8_t* flag = reinterpret_cast<uint8_t*>(ulist + T);
-  __shared__ uint32_t s_ucnt;
-  __shared__ unsigned long long ws[32];
-  for (int i = threadIdx.x; i < T; i += kThreads) {
-    s_acc[i] = 0.f;
-    flag[i] = 0;
-  }
-  if (threadIdx.x == 0) s_ucnt = 0;
-  __syncthreads();
-  unsigned long long nnz = 0, uni = 0, changed = 0;
-  for (int64_t tile = blockIdx.x; tile < A.n_tiles; tile += gridDim.x) {
-    const int64_t t0 = tile * T;
-    if (A.has_prev) {
-      // w_t - w_{t-1} is rebuilt below: clear it on the previous union first
-      for (int kk = 0; kk < A.K; ++kk) {
-        const uint32_t* pp = A.pos_prev + (int64_t)kk * (A.n_tiles + 1);
-        const uint32_t lo = pp[tile], hi = pp[tile + 1];
-        const uint32_t* ip = A.idx_prev + (int64_t)kk * A.ksel;
-        for (uint32_t i = lo + threadIdx.x; i < hi && i < A.ksel; i += kThreads) {
-          const uint32_t j = ip[i];
-          if (j < (uint32_t)A.d) A.dlt[j] = 0.f;
-        }
-      }
-    }
-    // workers in ascending order: sum_k C(e_{t+1/2,k}) starting from +0
-    for (int k = 0; k < A.K; ++k) {
-      const uint32_t* pc = A.pos_cur + (int64_t)k * (A.n_tiles + 1);
-      const uint32_t lo = pc[tile], hi = pc[tile + 1];
-      const uint32_t* ic = A.idx_cur + (int64_t)k * A.ksel;
-      const float* vc = A.val_cur + (int64_t)k * A.ksel;
-      float* ek = A.e + (int64_t)k * A.ld;
-      for (uint32_t i = lo + threadIdx.x; i < hi && i < A.ksel; i += kThreads) {
-        const uint32_t j = ic[i];
-        const float v = vc[i];
-        const uint32_t l = j - (uint32_t)t0;
-        if (l >= (uint32_t)T || j >= (uint32_t)A.d) {
-          atomicOr(A.status, kStatusInternal);
-          continue;
-        }
-        s_acc[l] = __fadd_rn(s_acc[l], v);
-        if (!flag[l]) {
-          flag[l] = 1;
-          ulist[atomicAdd(&s_ucnt, 1u)] = (uint16_t)l;
-        }
-        ek[j] = 0.f;  // e_{t+1,k} = e_{t+1/2,k} - C(e_{t+1/2,k}) = +0 where sent
-        nnz += (v != 0.f);
-      }
-      __syncthreads();
-    }
-    const uint32_t n = s_ucnt;
-    for (uint32_t u = threadIdx.x; u < n; u += kThreads) {
-      const uint32_t l = ulist[u];
-      const int64_t j = t0 + l;
+  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const uint32_t mine = 1u << k, lower = mine - 1u;
+  const int nparts = A.regions > 1 ? A.regions : (int)gridDim.x;
+  unsigned long long uni = 0, changed = 0;
+  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+    uint32_t lo, hi;
+    sent_part(A, k, part, nparts, &lo, &hi);
+    for (uint32_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+      const uint32_t j = __ldcg(ci + i);
+      if (j >= (uint32_t)A.d) continue;  // not sent (marked) or out of range
+      const uint32_t m = A.mask[j];
+      if (!(m & mine) || (m & lower)) continue;  // a lower worker owns j (or done)
+      // every sender's value is still in e[b][j]: load them all at once, then
+      // add in ascending worker order from +0
       const float wo = A.w[j];
-      const float wn = __fsub_rn(wo, __fmul_rn(A.a, s_acc[l]));
+      float vals[32];
+#pragma unroll
+      for (int b = 0; b < 32; ++b)
+        vals[b] = ((m >> b) & 1u) ? __ldcg(A.e + (int64_t)b * A.ld + j) : 0.f;
+      float sum = 0.f;
+#pragma unroll
+      for (int b = 0; b < 32; ++b) {
+        if ((m >> b) & 1u) {
+          sum = __fadd_rn(sum, vals[b]);
+          A.e[(int64_t)b * A.ld + j] = 0.f;  // e_{t+1,b} = e_{t+1/2,b} - C(.) = +0 where sent
+        }
+      }
+      const float wn = __fsub_rn(wo, __fmul_rn(A.a, sum));
       A.w[j] = wn;
       const float dd = __fsub_rn(wn, wo);
       A.dlt[j] = dd;
+      A.mask[j] = 0u;
       changed += (dd != 0.f);
-      s_acc[l] = 0.f;
-      flag[l] = 0;
+      ++uni;
     }
-    if (threadIdx.x == 0) uni += n;
-    __syncthreads();
-    if (threadIdx.x == 0) s_ucnt = 0;
-    __syncthreads();
   }
-  unsigned long long tot;
-  nnz = block_inclusive_scan<unsigned long long>(nnz, ws, &tot);
-  if (threadIdx.x == 0 && tot) atomicAdd(&A.step_ctr->v[kNnz], tot);
-  block_inclusive_scan<unsigned long long>(changed, ws, &tot);
-  if (threadIdx.x == 0 && tot) atomicAdd(&A.step_ctr->v[kChanged], tot);
-  if (threadIdx.x == 0 && uni) atomicAdd(&A.step_ctr->v[kUnion], uni);
+  uni = warp_sum(uni);
+  changed = warp_sum(changed);
+  if ((threadIdx.x & 31) == 0) {
+    if (uni) atomicAdd(&A.step_ctr->v[kUnion], uni);
+    if (changed) atomicAdd(&A.step_ctr->v[kChanged], changed);
+  }
+}
+
+// (index, value) pairs of worker k's last C(.) in ascending index order: its
+// sent candidates, tile by tile, sub-chunk by sub-chunk.
+__global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uint32_t* idx_out,
+                                                          float* val_out) {
+  __shared__ uint32_t ws[32];
+  const int64_t row = (int64_t)k * A.n_tiles;
+  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const float* cv = A.cand_val + (int64_t)k * A.cap;
+  uint32_t carry = 0;
+  for (int64_t t0 = 0; t0 < A.n_tiles; t0 += blockDim.x) {
+    const int64_t tile = t0 + threadIdx.x;
+    uint32_t cnt = 0;
+    if (tile < A.n_tiles) {
+      for (int w = 0; w < kChunksPerTile; ++w) {
+        const int64_t c = (row + tile) * kChunksPerTile + w;
+        const uint32_t base = A.chunk_base[c], n = A.chunk_cnt[c];
+        for (uint32_t i = 0; i < n && base + i < A.cap; ++i) cnt += (ci[base + i] & kUnsent) ? 0u : 1u;
+      }
+    }
+    uint32_t tot;
+    uint32_t pos = carry + block_inclusive_scan<uint32_t>(cnt, ws, &tot) - cnt;
+    if (cnt) {
+      for (int w = 0; w < kChunksPerTile; ++w) {
+        const int64_t c = (row + tile) * kChunksPerTile + w;
+        const uint32_t base = A.chunk_base[c], n = A.chunk_cnt[c];
+        for (uint32_t i = 0; i < n && base + i < A.cap; ++i) {
+          const uint32_t j = ci[base + i];
+          if (j & kUnsent) continue;
+          if (pos < A.ksel) {
+            idx_out[pos] = j;
+            val_out[pos] = cv[base + i];
+          }
+          ++pos;
+        }
+      }
+    }
+    carry += tot;
+  }
+  if (threadIdx.x == 0 && carry != A.ksel) atomicOr(A.status, kStatusInternal);
 }
 
 int tile_u(int tile) { return tile / (kWarps * 128); }
+bool use_bulk(int tile) { return tile == bulk::kT; }
 
 }  // namespace
 
-int accumulate_smem_bytes(int tile) { return tile * 12; }
-int aggregate_smem_bytes(int tile) { return tile * 7; }
+int accumulate_smem_bytes(int tile) {
+  return use_bulk(tile) ? (int)sizeof(bulk::Smem) : tile * 12;
+}
 
 cudaError_t configure_topk_kernels() {
   cudaError_t err = cudaSuccess;
@@ -589,19 +963,16 @@ cudaError_t configure_topk_kernels() {
     const cudaError_t e2 = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (err == cudaSuccess) err = e2;
   };
-  set((const void*)k_sample, kSampleAll * 4);
-  set((const void*)k_accumulate<1>, accumulate_smem_bytes(1024));
-  set((const void*)k_accumulate<2>, accumulate_smem_bytes(2048));
-  set((const void*)k_accumulate<4>, accumulate_smem_bytes(4096));
-  set((const void*)k_accumulate<8>, accumulate_smem_bytes(8192));
-  set((const void*)k_aggregate<1>, aggregate_smem_bytes(1024));
-  set((const void*)k_aggregate<2>, aggregate_smem_bytes(2048));
-  set((const void*)k_aggregate<4>, aggregate_smem_bytes(4096));
-  set((const void*)k_aggregate<8>, aggregate_smem_bytes(8192));
+  set((const void*)k_accumulate<1>, 1024 * 12);
+  set((const void*)k_accumulate<2>, 2048 * 12);
+  set((const void*)k_accumulate<4>, 4096 * 12);
+  set((const void*)k_accumulate<8>, 8192 * 12);
+  set((const void*)k_accumulate_bulk, (int)sizeof(bulk::Smem));
   return err;
 }
 
 int accumulate_blocks_per_sm(int tile) {
+  if (use_bulk(tile)) return 1;  // one persistent CTA per SM
   int n = 0;
   const int smem = accumulate_smem_bytes(tile);
   switch (tile_u(tile)) {
@@ -613,27 +984,17 @@ int accumulate_blocks_per_sm(int tile) {
   return n > 0 ? n : 1;
 }
 
-int aggregate_blocks_per_sm(int tile) {
-  int n = 0;
-  const int smem = aggregate_smem_bytes(tile);
-  switch (tile_u(tile)) {
-    case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_aggregate<1>, kThreads, smem); break;
-    case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_aggregate<2>, kThreads, smem); break;
-    case 4: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_aggregate<4>, kThreads, smem); break;
-    default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_aggregate<8>, kThreads, smem); break;
-  }
-  return n > 0 ? n : 1;
-}
-
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
-  const int n_s = A.sample_chunks == 0 ? (int)A.d : A.sample_chunks * 8;
-  const int smem = A.dense_mode ? 0 : n_s * 4;
-  k_sample<<<A.K, kSampleThreads, smem, s>>>(A);
+  k_sample<<<dim3(A.sample_blocks, A.K), kThreads, 0, s>>>(A);
   return cudaGetLastError();
 }
 
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
   const int smem = accumulate_smem_bytes(A.tile);
+  if (use_bulk(A.tile)) {
+    k_accumulate_bulk<<<grid, bulk::kThreadsAll, smem, s>>>(A);
+    return cudaGetLastError();
+  }
   switch (tile_u(A.tile)) {
     case 1: k_accumulate<1><<<grid, kThreads, smem, s>>>(A); break;
     case 2: k_accumulate<2><<<grid, kThreads, smem, s>>>(A); break;
@@ -651,36 +1012,28 @@ cudaError_t launch_select_pass(const TopkArgs& A, int pass, int blocks_per_worke
   return cudaGetLastError();
 }
 
+cudaError_t launch_ties(const TopkArgs& A, cudaStream_t s) {
+  k_ties<<<A.K, 1024, 0, s>>>(A);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s) {
   k_select_dense<<<A.K, 1024, 0, s>>>(A);
   return cudaGetLastError();
 }
 
-cudaError_t launch_chunk_count(const TopkArgs& A, cudaStream_t s) {
-  const dim3 grid((unsigned)((A.n_tiles + kWarps - 1) / kWarps), A.K);
-  k_chunk_count<<<grid, kThreads, 0, s>>>(A);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_chunk_scan(const TopkArgs& A, cudaStream_t s) {
-  k_chunk_scan<<<A.K, 1024, 0, s>>>(A);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_chunk_write(const TopkArgs& A, cudaStream_t s) {
-  const dim3 grid((unsigned)((A.n_tiles + kWarps - 1) / kWarps), A.K);
-  k_chunk_write<<<grid, kThreads, 0, s>>>(A);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_aggregate(const TopkArgs& A, int grid, cudaStream_t s) {
-  const int smem = aggregate_smem_bytes(A.tile);
-  switch (tile_u(A.tile)) {
-    case 1: k_aggregate<1><<<grid, kThreads, smem, s>>>(A); break;
-    case 2: k_aggregate<2><<<grid, kThreads, smem, s>>>(A); break;
-    case 4: k_aggregate<4><<<grid, kThreads, smem, s>>>(A); break;
-    default: k_aggregate<8><<<grid, kThreads, smem, s>>>(A); break;
-  }
+  const dim3 g(grid, A.K);
+  k_mark<<<g, kThreads, 0, s>>>(A);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  k_owner_sum<<<g, kThreads, 0, s>>>(A);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_selected(const TopkArgs& A, int k, uint32_t* idx_out, float* val_out,
+                                   cudaStream_t s) {
+  k_gather_selected<<<1, 1024, 0, s>>>(A, k, idx_out, val_out);
   return cudaGetLastError();
 }
 

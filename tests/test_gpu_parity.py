@@ -54,6 +54,37 @@ def test_topk_sampled_and_dense_agree_ragged_large():
     assert pairs[1].gpu.stats()["fallbacks"] == 4 * K
 
 
+@pytest.mark.parametrize("offset", [0, 1])
+def test_topk_bulk_copy_path(offset):
+    """d large enough for the bulk-copy dense pass (tiles of 4096); odd d gives
+    rows at every alignment, and offset 1 makes the first row start 4 bytes
+    past an aligned address so its bulk copy would begin before the buffer
+    (that row is then loaded directly)."""
+    import torch
+    d, K = 1_300_001, 3
+    rng = np.random.default_rng(15 + offset)
+    p = Pair(d, K, 0.9, 0.05, ratio=0.002, seed=2)
+    for t in range(3):
+        g = (rng.standard_normal((K, d)) * np.exp(rng.uniform(-3, 0, size=d))).astype(np.float32)
+        buf = torch.empty(K * d + offset, dtype=torch.float32, device=p.dev)
+        view = buf[offset:].view(K, d)
+        view.copy_(torch.from_numpy(g))
+        p.compare(p.step(g, grads_dev=view), residuals=(t == 2))
+    assert p.gpu.stats()["fallbacks"] == 0
+    assert p.gpu.check() == 0
+
+
+def test_topk_dense_tiles_unstaged_aggregate():
+    """Every coordinate sent by 5 workers: more entries per tile than the
+    aggregate stages in shared memory."""
+    d, K = 3000, 5
+    rng = np.random.default_rng(16)
+    p = Pair(d, K, 0.9, 0.1, ratio=1.0)
+    for t in range(3):
+        p.compare(p.step(rng.standard_normal((K, d)).astype(np.float32)))
+    p.compare_stats()
+
+
 def test_topk_all_zero_gradients_fall_back():
     """Every magnitude ties: the selection is the k lowest indices; above the
     full-sample size the candidate filter overflows and the dense path runs."""
