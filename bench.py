@@ -324,6 +324,7 @@ def run_gmc(args, wl, world, rank, local):
     prof = gpu.profile_read()
     gpu.profile(False)
     status = gpu.check()
+    totals = gpu.stats()
     ms_max = max_over_ranks(ms, world, dev)
     value = wl.K * wl.d * args.steps * world / (ms_max / 1e3)
 
@@ -385,6 +386,7 @@ def run_gmc(args, wl, world, rank, local):
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
         "gpu_launches": int(round(launches_per_step * args.steps)),
         "kernels": kernels, "status": status,
+        "select_fallbacks": totals["fallbacks"], "steps_run": totals["steps"],
     }
     return line if rank == 0 else None
 

@@ -54,6 +54,8 @@ struct gmc_ctx {
   float* dlt = nullptr;
   WorkerSel* sel = nullptr;
   uint32_t* ghist = nullptr;
+  uint32_t* bucket = nullptr;  // K x 2*kBucketCap
+  int sel_shift = 20;
   uint32_t* sample_keys = nullptr;
   uint32_t* big_tiles = nullptr;
   uint32_t* rcount = nullptr;
@@ -200,6 +202,8 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.dense_mode = h->select_mode == GMC_SELECT_DENSE;
   A.sel = h->sel;
   A.ghist = h->ghist;
+  A.bucket = h->bucket;
+  A.sel_shift = h->sel_shift;
   A.sample_keys = h->sample_keys;
   A.big_tiles = h->big_tiles;
   A.regions = h->regions;
@@ -269,10 +273,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s) {
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
                   [&] { return launch_accumulate(A, h->grid_acc, s); }));
-    for (int pass = 0; pass < 3; ++pass)
-      GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s,
-                    [&] { return launch_select_pass(A, pass, h->sel_blocks, s); }));
-    GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] { return launch_ties(A, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] { return launch_select(A, h->sel_blocks, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_DENSE, 0.0, s, [&] { return launch_select_dense(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk, s,
                   [&] { return launch_aggregate(A, h->grid_agg, s); }));
@@ -402,12 +403,21 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     h->sel_blocks = h->regions > 1 ? (int)std::min<int64_t>(h->regions, want)
                                    : (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
     h->sample_blocks = (int)std::max<int64_t>(1, ((h->sample_chunks ? 8 * kSampleChunks : d) + 2047) / 2048);
+    // relative-histogram bin width 2^sel_shift keys: near the k-th key a key
+    // step of 2^23 is an octave of |v|, and a Gaussian-like tail puts about
+    // 11 ln2 * k * 2^s / 2^23 candidates in one bin; aim at 2048 (the bin is
+    // ranked in shared memory when it holds at most kBucketCap)
+    {
+      const double w = 2048.0 * 8388608.0 / (11.0 * std::log(2.0) * (double)h->ksel);
+      h->sel_shift = (int)std::min(20.0, std::max(0.0, std::floor(std::log2(w))));
+    }
     const int64_t Kt = (int64_t)K * h->n_tiles;
     if ((err = dalloc(h, &h->e, (size_t)K * h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->w, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->dlt, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->sel, (size_t)K)) != cudaSuccess ||
         (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess ||
+        (err = dalloc(h, &h->bucket, (size_t)K * 2 * kBucketCap)) != cudaSuccess ||
         (err = dalloc(h, &h->sample_keys, (size_t)K * 8 * kSampleChunks)) != cudaSuccess ||
         (err = dalloc(h, &h->big_tiles, (size_t)h->n_tiles + 1)) != cudaSuccess ||
         (err = dalloc(h, &h->rcount, (size_t)K * h->regions)) != cudaSuccess ||

@@ -16,20 +16,23 @@ constexpr int kSampleThreads = 1024;
 constexpr int kSampleChunks = 4096;          // sampled 8-element chunks per worker
 constexpr int kSampleAll = 32768;            // d at or below which every element is sampled
 constexpr int kHistBins = 2048;              // first radix digit: key bits 30..20
+constexpr int kRelBins = 2048;               // bins of the candidates' relative histogram
+constexpr int kBucketCap = 12288;            // candidates of one bin ranked in shared memory
 
 // Per-worker top-k selection state, rewritten every step.
 struct WorkerSel {
   uint32_t theta;    // candidate threshold key from the sample (kNoCandidate = none)
   uint32_t count;    // candidates appended by the accumulate pass (may exceed cap)
-  uint32_t prefix;   // radix digits fixed so far
-  uint32_t rank;     // 1-based rank still to find inside the current bucket
+  uint32_t prefix;   // select: relative-histogram bin holding the k-th key
+  uint32_t rank;     // select: the k-th key's 1-based rank inside that bin
   uint32_t T;        // the k-th largest key
   uint32_t n_tie;    // elements equal to T that are kept (lowest indices first)
   uint32_t ties;     // candidates equal to T
   uint32_t t_idx;    // a candidate equal to T is kept iff its index <= t_idx
   uint32_t dense;    // 1: this worker's selection is made by the dense path
-  uint32_t done[4];  // finished-block counters: three select passes, the sample
-  uint32_t pad[3];
+  uint32_t done[4];  // finished-block counters: the two select passes, -, the sample
+  uint32_t count_bucket;  // candidates collected from the k-th key's bin
+  uint32_t pad[2];
 };
 
 // Step counters (see GMC_STAT_* in gmc.h), unsigned 64-bit slots.

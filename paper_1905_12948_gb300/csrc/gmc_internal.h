@@ -42,6 +42,8 @@ struct TopkArgs {
   int dense_mode;            // GMC_SELECT_DENSE
   WorkerSel* sel;            // K entries
   uint32_t* ghist;           // K x kHistBins (zero between uses)
+  uint32_t* bucket;          // K x 2*kBucketCap: keys, then indices of the k-th key's bin
+  int sel_shift;             // log2 of the relative-histogram bin width (in keys)
   uint32_t* sample_keys;     // K x 8*kSampleChunks
   uint32_t* big_tiles;       // [0]: count, then tile ids left to the block aggregate
   uint32_t* cand_idx;        // current chunks: K x cap
@@ -98,8 +100,7 @@ struct DetachArgs {
 // Launch wrappers (each returns the cudaGetLastError of its launches).
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s);
-cudaError_t launch_select_pass(const TopkArgs& A, int pass, int blocks_per_worker, cudaStream_t s);
-cudaError_t launch_ties(const TopkArgs& A, cudaStream_t s);
+cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s);
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_aggregate(const TopkArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_gather_selected(const TopkArgs& A, int k, uint32_t* idx_out, float* val_out,

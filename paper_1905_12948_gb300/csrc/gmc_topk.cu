@@ -550,150 +550,200 @@ __device__ __forceinline__ void candidate_part(const TopkArgs& A, int k, int p, 
 }
 
 // ---------------------------------------------------------------------------
-// exact select among candidates: three radix passes; the last block of each
-// worker turns the global histogram into the next digit.
+// exact select among candidates, two passes:
+//   hist    a kRelBins-bin histogram of the candidates' keys above theta, in
+//           bins of 2^sel_shift keys (sel_shift is chosen from k so that the
+//           k-th key's bin holds about 2048 candidates on smooth data); the
+//           last block finds the bin holding the k-th key
+//   finish  the candidates of that bin are collected (key, index); the last
+//           block ranks them in shared memory: the k-th key T, how many keys
+//           equal T are kept, and -- when fewer are kept than there are -- the
+//           largest index kept (ties go to the lower index)
 // ---------------------------------------------------------------------------
-template <int PASS>
-__global__ void __launch_bounds__(kThreads) k_select_pass(TopkArgs A) {
-  constexpr int nbins = PASS == 0 ? 2048 : 1024;
-  constexpr int shift = PASS == 0 ? 20 : (PASS == 1 ? 10 : 0);
-  __shared__ uint32_t h[nbins];
+// Bin of a candidate key in the relative histogram: (key - theta) >> shift,
+// the top bin also taking everything further up (candidate keys are >= theta).
+__device__ __forceinline__ int rel_bin(uint32_t key, uint32_t theta, int shift) {
+  const uint32_t b = (key > theta ? key - theta : 0u) >> shift;
+  return b < (uint32_t)kRelBins ? (int)b : kRelBins - 1;
+}
+
+__global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
+  __shared__ uint32_t h[kRelBins];
   __shared__ uint32_t ws[32];
   __shared__ uint32_t s_last, s_bin, s_rank;
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
   if (needs_dense(S, A.ksel, A.cap)) return;
-  const uint32_t prefix = S.prefix;
-  for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
+  const uint32_t theta = S.theta;
+  for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) h[b] = 0;
   __syncthreads();
   const float* cv = A.cand_val + (int64_t)k * A.cap;
   const int nparts = A.regions == 1 ? (int)gridDim.x : A.regions;
   for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
     uint32_t lo, hi;
     candidate_part(A, k, part, nparts, &lo, &hi);
-    // 16 candidates per thread per round, 16-byte loads (lo is a multiple of 4)
-    for (uint32_t i0 = lo; i0 < hi; i0 += 16 * blockDim.x) {
-      float kv[16];
+    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * blockDim.x) {
+      uint32_t kv[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const uint32_t i = i0 + (q * blockDim.x + threadIdx.x) * 4;
-        if (i + 3 < hi) {
-          const float4 x = *reinterpret_cast<const float4*>(cv + i);
-          kv[4 * q] = x.x; kv[4 * q + 1] = x.y; kv[4 * q + 2] = x.z; kv[4 * q + 3] = x.w;
-        } else {
-#pragma unroll
-          for (int t = 0; t < 4; ++t) kv[4 * q + t] = i + t < hi ? cv[i + t] : __uint_as_float(0xffffffffu);
-        }
+        const uint32_t i = i0 + q * blockDim.x + threadIdx.x;
+        kv[q] = i < hi ? mag_key(cv[i]) : 0xffffffffu;
       }
 #pragma unroll
-      for (int t = 0; t < 16; ++t) {
-        const uint32_t raw = __float_as_uint(kv[t]);
-        const uint32_t key = raw & kKeyMask;
-        int bin = -1;
-        if (raw != 0xffffffffu && (PASS == 0 || (key >> (shift + 10)) == prefix))
-          bin = (int)((key >> shift) & (nbins - 1));
-        warp_hist_add(h, bin);
-      }
+      for (int q = 0; q < 4; ++q) warp_hist_add(h, kv[q] != 0xffffffffu ? rel_bin(kv[q], theta, A.sel_shift) : -1);
     }
   }
   __syncthreads();
   uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
-  for (int b = threadIdx.x; b < nbins; b += blockDim.x)
+  for (int b = threadIdx.x; b < kRelBins; b += blockDim.x)
     if (h[b]) atomicAdd(&gh[b], h[b]);
   __threadfence();
   __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[PASS], 1u) == gridDim.x - 1) ? 1u : 0u;
+  if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[0], 1u) == gridDim.x - 1) ? 1u : 0u;
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  for (int b = threadIdx.x; b < nbins; b += blockDim.x) {
+  for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) {
     h[b] = __ldcg(&gh[b]);
     gh[b] = 0;
   }
   if (threadIdx.x == 0) {
     s_bin = 0;
     s_rank = 0;
-    S.done[PASS] = 0;
+    S.done[0] = 0;
   }
   __syncthreads();
-  const uint32_t r = PASS == 0 ? A.ksel : S.rank;
-  block_find_from_top(h, nbins, r, ws, &s_bin, &s_rank);
+  block_find_from_top(h, kRelBins, A.ksel, ws, &s_bin, &s_rank);
   if (threadIdx.x == 0) {
     if (s_rank == 0) atomicOr(A.status, kStatusInternal);
-    if (PASS == 0) {
-      S.prefix = s_bin;
-      S.rank = s_rank;
-    } else if (PASS == 1) {
-      S.prefix = (prefix << 10) | s_bin;
-      S.rank = s_rank;
-    } else {
-      S.T = (prefix << 10) | s_bin;
-      S.n_tie = s_rank;
-      S.ties = h[s_bin];
-      S.t_idx = 0xffffffffu;  // every tie kept, unless k_ties narrows it
-    }
+    S.prefix = s_bin;  // relative bin of the k-th key
+    S.rank = s_rank;   // its rank inside that bin
   }
 }
 
-// ---------------------------------------------------------------------------
-// ties: when more candidates equal T than are kept, the kept ones are the
-// n_tie lowest indices; t_idx = the largest of them.
-// ---------------------------------------------------------------------------
-constexpr int kTieCap = 8192;
-
-__global__ void __launch_bounds__(1024) k_ties(TopkArgs A) {
-  const int k = blockIdx.x;
-  WorkerSel& S = A.sel[k];
-  if (needs_dense(S, A.ksel, A.cap) || S.ties == S.n_tie) return;
-  __shared__ uint32_t tie_idx[kTieCap];
-  __shared__ uint32_t h[kHistBins];
-  __shared__ uint32_t ws[32];
-  __shared__ uint32_t s_n, s_bin, s_rank;
-  if (threadIdx.x == 0) s_n = 0;
-  __syncthreads();
-  const uint32_t T = S.T;
-  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
-  const float* cv = A.cand_val + (int64_t)k * A.cap;
-  const int nparts = A.regions;
-  for (int part = 0; part < nparts; ++part) {
-    uint32_t lo, hi;
-    candidate_part(A, k, part, nparts, &lo, &hi);
-    for (uint32_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
-      if (mag_key(cv[i]) == T) {
-        const uint32_t p = atomicAdd(&s_n, 1u);
-        if (p < kTieCap) tie_idx[p] = ci[i];
-      }
-    }
-  }
-  __syncthreads();
-  const uint32_t n = s_n;
-  if (n > (uint32_t)kTieCap) {  // too many ties to rank here: the dense path takes over
-    if (threadIdx.x == 0) S.dense = 1;
-    return;
-  }
-  // the n_tie-th smallest index = the (n - n_tie + 1)-th largest (radix digits 11/10/10)
-  uint32_t r = n - S.n_tie + 1, prefix = 0;
+// Radix select in shared memory: the r-th largest of n values (digits 11/10/10).
+__device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, uint32_t r,
+                                                uint32_t* h, uint32_t* ws, uint32_t* s_bin,
+                                                uint32_t* s_rank, uint32_t* rank_out) {
+  uint32_t prefix = 0;
   for (int pass = 0; pass < 3; ++pass) {
     const int nbins = pass == 0 ? 2048 : 1024;
     const int shift = pass == 0 ? 20 : (pass == 1 ? 10 : 0);
     for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
     if (threadIdx.x == 0) {
-      s_bin = 0;
-      s_rank = 0;
+      *s_bin = 0;
+      *s_rank = 0;
     }
     __syncthreads();
-    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) {
-      const uint32_t x = tie_idx[i];
-      if (pass == 0 || (x >> (shift + 10)) == prefix)
-        atomicAdd(&h[(x >> shift) & (uint32_t)(nbins - 1)], 1u);
+    for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
+      const uint32_t i = i0 + threadIdx.x;
+      int bin = -1;
+      if (i < n) {
+        const uint32_t v = x[i];
+        if (pass == 0 || (v >> (shift + 10)) == prefix) bin = (int)((v >> shift) & (uint32_t)(nbins - 1));
+      }
+      warp_hist_add(h, bin);
     }
     __syncthreads();
-    block_find_from_top(h, nbins, r, ws, &s_bin, &s_rank);
-    prefix = pass == 0 ? s_bin : ((prefix << 10) | s_bin);
-    r = s_rank;
+    block_find_from_top(h, nbins, r, ws, s_bin, s_rank);
+    prefix = pass == 0 ? *s_bin : ((prefix << 10) | *s_bin);
+    r = *s_rank;
     __syncthreads();
   }
-  if (threadIdx.x == 0) S.t_idx = prefix;
+  *rank_out = r;
+  return prefix;
+}
+
+__global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
+  extern __shared__ __align__(16) uint32_t fin[];  // kBucketCap keys + kBucketCap indices
+  __shared__ uint32_t h[kHistBins];
+  __shared__ uint32_t ws[32];
+  __shared__ uint32_t s_last, s_bin, s_rank, s_n;
+  const int k = blockIdx.y;
+  WorkerSel& S = A.sel[k];
+  if (needs_dense(S, A.ksel, A.cap)) return;
+  const uint32_t theta = S.theta;
+  const int want = (int)S.prefix;
+  const int lane = threadIdx.x & 31;
+  const uint32_t lt = lanemask_lt();
+  uint32_t* bk = A.bucket + (int64_t)k * 2 * kBucketCap;  // keys, then indices
+  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const float* cv = A.cand_val + (int64_t)k * A.cap;
+  const int nparts = A.regions == 1 ? (int)gridDim.x : A.regions;
+  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+    uint32_t lo, hi;
+    candidate_part(A, k, part, nparts, &lo, &hi);
+    for (uint32_t i0 = lo; i0 < hi; i0 += blockDim.x) {
+      const uint32_t i = i0 + threadIdx.x;
+      uint32_t key = 0;
+      bool in = false;
+      if (i < hi) {
+        key = mag_key(cv[i]);
+        in = rel_bin(key, theta, A.sel_shift) == want;
+      }
+      const uint32_t m = __ballot_sync(0xffffffffu, in);
+      if (m) {
+        uint32_t base = 0;
+        if (lane == 0) base = atomicAdd(&S.count_bucket, (uint32_t)__popc(m));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        const uint32_t o = base + __popc(m & lt);
+        if (in && o < (uint32_t)kBucketCap) {
+          bk[o] = key;
+          bk[kBucketCap + o] = ci[i];
+        }
+      }
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[1], 1u) == gridDim.x - 1) ? 1u : 0u;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (threadIdx.x == 0) {
+    s_n = __ldcg(&S.count_bucket);
+    S.count_bucket = 0;
+    S.done[1] = 0;
+  }
+  __syncthreads();
+  const uint32_t n = s_n;
+  if (n > (uint32_t)kBucketCap) {  // the k-th key's bin is too crowded: the dense path decides
+    if (threadIdx.x == 0) S.dense = 1;
+    return;
+  }
+  uint32_t* keys = fin;
+  uint32_t* idxs = fin + kBucketCap;
+  for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) {
+    keys[i] = __ldcg(&bk[i]);
+    idxs[i] = __ldcg(&bk[kBucketCap + i]);
+  }
+  __syncthreads();
+  uint32_t n_tie;
+  const uint32_t T = smem_select(keys, n, S.rank, h, ws, &s_bin, &s_rank, &n_tie);
+  // ties: gather the indices of the keys equal to T over the keys, in place;
+  // a round writes below the end of what the block has read so far
+  if (threadIdx.x == 0) s_n = 0;
+  __syncthreads();
+  for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
+    const uint32_t i = i0 + threadIdx.x;
+    const bool tie = i < n && keys[i] == T;
+    const uint32_t j = tie ? idxs[i] : 0u;
+    __syncthreads();
+    if (tie) keys[atomicAdd(&s_n, 1u)] = j;
+  }
+  __syncthreads();
+  const uint32_t ties = s_n;
+  uint32_t t_idx = 0xffffffffu;
+  if (ties > n_tie) {  // keep the n_tie lowest indices: t_idx = (ties - n_tie + 1)-th largest
+    uint32_t unused;
+    t_idx = smem_select(keys, ties, ties - n_tie + 1, h, ws, &s_bin, &s_rank, &unused);
+  }
+  if (threadIdx.x == 0) {
+    S.T = T;
+    S.n_tie = n_tie;
+    S.ties = ties;
+    S.t_idx = t_idx;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -968,6 +1018,7 @@ cudaError_t configure_topk_kernels() {
   set((const void*)k_accumulate<4>, 4096 * 12);
   set((const void*)k_accumulate<8>, 8192 * 12);
   set((const void*)k_accumulate_bulk, (int)sizeof(bulk::Smem));
+  set((const void*)k_select_finish, 2 * kBucketCap * 4);
   return err;
 }
 
@@ -1004,16 +1055,12 @@ cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_select_pass(const TopkArgs& A, int pass, int blocks_per_worker, cudaStream_t s) {
+cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s) {
   const dim3 grid(blocks_per_worker, A.K);
-  if (pass == 0) k_select_pass<0><<<grid, kThreads, 0, s>>>(A);
-  else if (pass == 1) k_select_pass<1><<<grid, kThreads, 0, s>>>(A);
-  else k_select_pass<2><<<grid, kThreads, 0, s>>>(A);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_ties(const TopkArgs& A, cudaStream_t s) {
-  k_ties<<<A.K, 1024, 0, s>>>(A);
+  k_select_hist<<<grid, kThreads, 0, s>>>(A);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  k_select_finish<<<grid, kThreads, 2 * kBucketCap * 4, s>>>(A);
   return cudaGetLastError();
 }
 
