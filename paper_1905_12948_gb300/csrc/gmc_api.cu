@@ -67,6 +67,14 @@ struct gmc_ctx {
   uint32_t* chunk_base[2] = {nullptr, nullptr};
   uint32_t* chunk_cnt[2] = {nullptr, nullptr};
   uint32_t* mask = nullptr;
+  uint32_t* smask[2] = {nullptr, nullptr};  // senders at the sampled positions, by step parity
+  // deferred aggregation (bulk top-k pass): the last step's sent pairs are
+  // summed into w by the next step's bulk pass, or by flush() when state is read
+  bool agg_pending = false;
+  float a_pending = 0.f;       // fl(eta/K) of that step
+  cudaStream_t aux = nullptr;  // library stream for flushes outside a caller stream
+  cudaEvent_t ev_step = nullptr, ev_flush = nullptr;
+  bool wait_flush = false;     // the next launch waits for ev_flush
   uint32_t* bitmap = nullptr;
   int32_t* rank = nullptr;
   int32_t* blocks = nullptr;
@@ -120,6 +128,11 @@ cudaError_t dalloc(gmc_ctx* h, T** p, size_t count) {
 void free_all(gmc_ctx* h) {
   for (void* p : h->allocations) cudaFree(p);
   h->allocations.clear();
+  if (h->ev_step) cudaEventDestroy(h->ev_step);
+  if (h->ev_flush) cudaEventDestroy(h->ev_flush);
+  if (h->aux) cudaStreamDestroy(h->aux);
+  h->ev_step = h->ev_flush = nullptr;
+  h->aux = nullptr;
   for (auto& r : h->pending) {
     cudaEventDestroy(r.start);
     cudaEventDestroy(r.stop);
@@ -215,6 +228,12 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.chunk_cnt = h->chunk_cnt[cur];
   A.mask = h->mask;
   A.cand_idx_prev = h->cand_idx[prev];
+  A.cand_val_prev = h->cand_val[prev];
+  A.smask_rd = h->smask[prev];
+  A.smask_wr = h->smask[cur];
+  A.total_ctr = h->total_ctr;
+  A.pending = 0;
+  A.a_prev = A.a;
   A.chunk_base_prev = h->chunk_base[prev];
   A.chunk_cnt_prev = h->chunk_cnt[prev];
   A.step_ctr = h->step_ctr;
@@ -263,20 +282,50 @@ RbgsArgs rbgs_args(gmc_ctx* h, const float* grads) {
     if (err_ != cudaSuccess) return status_of(err_); \
   } while (0)
 
-int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s) {
+// Work on s that reads or writes the state waits for a flush that may have
+// been enqueued on another stream since the last step; a step (clear = true)
+// resets the flag, later work is ordered after that step by the caller.
+cudaError_t order_after_flush(gmc_ctx* h, cudaStream_t s, bool clear) {
+  if (!h->wait_flush) return cudaSuccess;
+  if (clear) h->wait_flush = false;
+  return cudaStreamWaitEvent(s, h->ev_flush, 0);
+}
+
+// One step of Alg. 1 / Alg. 2 on stream s. With the bulk top-k pass the
+// step's aggregation (sum of the sent pairs into w, residuals to +0 where
+// sent) is left pending unless `eager`: the next step's bulk pass applies it
+// while it streams the tile, or flush() does when the state is read.
+int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager) {
   const double Kd = (double)h->K * (double)h->d;
+  GMC_TRY(order_after_flush(h, s, true));
   GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
   unsigned long long pairs_add = 0;
   if (h->compressor == GMC_TOPK) {
-    const TopkArgs A = topk_args(h, grads);
+    TopkArgs A = topk_args(h, grads);
+    A.pending = h->agg_pending ? 1 : 0;
+    A.a_prev = h->a_pending;
     const double kk = (double)h->K * (double)h->ksel;
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
                   [&] { return launch_accumulate(A, h->grid_acc, s); }));
+    h->agg_pending = false;
     GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] { return launch_select(A, h->sel_blocks, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_DENSE, 0.0, s, [&] { return launch_select_dense(A, s); }));
-    GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk, s,
-                  [&] { return launch_aggregate(A, h->grid_agg, s); }));
+    const bool defer = h->tile == kBulkTile && !eager && !h->detach_out;
+    if (defer) {
+      GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 8.0 * kk, s,
+                    [&] { return launch_mark(A, kMarkSent | kMarkSample, h->grid_agg, s); }));
+      h->agg_pending = true;
+      h->a_pending = A.a;
+    } else {
+      TopkArgs B = A;
+      B.a_prev = A.a;
+      B.total_ctr = nullptr;  // k_finalize adds the step's counts to the totals
+      GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk, s, [&] {
+        cudaError_t err = launch_mark(B, kMarkSent | kMarkMask, h->grid_agg, s);
+        return err != cudaSuccess ? err : launch_owner_sum(B, h->grid_agg, s);
+      }));
+    }
     pairs_add = (unsigned long long)h->K * h->ksel;
   } else {
     const RbgsArgs A = rbgs_args(h, grads);
@@ -291,9 +340,35 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s) {
   }
   GMC_TRY(timed(h, GMC_KERNEL_OTHER, 0.0, s,
                 [&] { return launch_finalize(h->step_ctr, h->total_ctr, pairs_add, s); }));
+  if (h->ev_step) GMC_TRY(cudaEventRecord(h->ev_step, s));
   h->t += 1;
   return GMC_OK;
 }
+
+// Apply a pending aggregation on stream s (ordered after the last step):
+// the senders of every coordinate into mask, then k_owner_sum; the sampled
+// senders are cleared, since the next sample must not apply them again.
+int flush(gmc_ctx* h, cudaStream_t s) {
+  if (!h->agg_pending) return GMC_OK;
+  GMC_TRY(cudaStreamWaitEvent(s, h->ev_step, 0));
+  TopkArgs A = topk_args_at(h, nullptr, h->t - 1);
+  A.a_prev = h->a_pending;
+  A.step_ctr = h->step_ctr;    // the counts belong to the last step
+  A.total_ctr = h->total_ctr;  // which k_finalize has already added up
+  GMC_TRY(launch_mark(A, kMarkMask, h->grid_agg, s));
+  GMC_TRY(launch_owner_sum(A, h->grid_agg, s));
+  GMC_TRY(cudaMemsetAsync(A.smask_wr, 0, (size_t)kSampleSlots * sizeof(uint32_t), s));
+  GMC_TRY(cudaEventRecord(h->ev_flush, s));
+  h->wait_flush = true;
+  h->agg_pending = false;
+  return GMC_OK;
+}
+
+#define GMC_TRY_ST(expr)                 \
+  do {                                   \
+    const int st_ = (expr);              \
+    if (st_ != GMC_OK) return st_;       \
+  } while (0)
 
 bool finite_f(float x) { return std::isfinite(x); }
 
@@ -387,7 +462,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     // candidate slots: the bulk pass gives every CTA its own region per worker
     // (twice its share of the expected candidates, plus slack); otherwise one region
     const uint32_t cap0 = h->cap;
-    if (h->tile == 4096) {
+    if (h->tile == kBulkTile) {
       h->regions = h->grid_acc;
       h->cap_region = (uint32_t)(((2ull * cap0 + h->regions - 1) / h->regions + 1024 + 3) & ~3ull);
     } else {
@@ -421,7 +496,13 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->sample_keys, (size_t)K * 8 * kSampleChunks)) != cudaSuccess ||
         (err = dalloc(h, &h->big_tiles, (size_t)h->n_tiles + 1)) != cudaSuccess ||
         (err = dalloc(h, &h->rcount, (size_t)K * h->regions)) != cudaSuccess ||
-        (err = dalloc(h, &h->mask, (size_t)h->ld)) != cudaSuccess)
+        (err = dalloc(h, &h->mask, (size_t)h->ld)) != cudaSuccess ||
+        (err = dalloc(h, &h->smask[0], (size_t)kSampleSlots)) != cudaSuccess ||
+        (err = dalloc(h, &h->smask[1], (size_t)kSampleSlots)) != cudaSuccess)
+      return fail(err);
+    if ((err = cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking)) != cudaSuccess ||
+        (err = cudaEventCreateWithFlags(&h->ev_step, cudaEventDisableTiming)) != cudaSuccess ||
+        (err = cudaEventCreateWithFlags(&h->ev_flush, cudaEventDisableTiming)) != cudaSuccess)
       return fail(err);
     for (int p = 0; p < 2; ++p) {
       if ((err = dalloc(h, &h->cand_idx[p], (size_t)K * h->cap)) != cudaSuccess ||
@@ -514,6 +595,8 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
   if (!h || !w0_dev) return GMC_EINVAL;
   DeviceGuard g(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  GMC_TRY(order_after_flush(h, s, true));
+  h->agg_pending = false;  // a pending aggregation of the old state is dropped
   GMC_TRY(cudaMemcpyAsync(h->w, w0_dev, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice, s));
   GMC_TRY(cudaMemsetAsync(h->e, 0, (size_t)h->K * h->ld * sizeof(float), s));
   GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
@@ -521,6 +604,9 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
     for (int p = 0; p < 2; ++p)
       GMC_TRY(cudaMemsetAsync(h->chunk_cnt[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint32_t), s));
     GMC_TRY(cudaMemsetAsync(h->sel, 0, (size_t)h->K * sizeof(WorkerSel), s));
+    GMC_TRY(cudaMemsetAsync(h->mask, 0, (size_t)h->ld * sizeof(uint32_t), s));
+    for (int p = 0; p < 2; ++p)
+      GMC_TRY(cudaMemsetAsync(h->smask[p], 0, (size_t)kSampleSlots * sizeof(uint32_t), s));
   } else {
     for (int p = 0; p < 2; ++p) GMC_TRY(cudaMemsetAsync(h->uflag[p], 0, (size_t)h->nb, s));
   }
@@ -536,7 +622,7 @@ int gmc_step(gmc_t h, const float* grads_dev, void* stream) {
   if (!h || !grads_dev) return GMC_EINVAL;
   if (!h->initialized) return GMC_ESTATE;
   DeviceGuard g(h->device);
-  return enqueue_step(h, grads_dev, static_cast<cudaStream_t>(stream));
+  return enqueue_step(h, grads_dev, static_cast<cudaStream_t>(stream), false);
 }
 
 int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, void* stream) {
@@ -550,7 +636,7 @@ int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, v
     if (err != cudaSuccess) return status_of(err);
   }
   GMC_TRY(cudaMemcpyAsync(h->gstage, grads_host, n * sizeof(float), cudaMemcpyHostToDevice, s));
-  const int st = enqueue_step(h, h->gstage, s);
+  const int st = enqueue_step(h, h->gstage, s, true);
   if (st != GMC_OK) return st;
   if (step_stats_host)
     GMC_TRY(cudaMemcpyAsync(step_stats_host, h->step_ctr, sizeof(Counters), cudaMemcpyDeviceToHost, s));
@@ -561,6 +647,8 @@ int gmc_get_params(gmc_t h, float* w_dev_out, void* stream) {
   if (!h || !w_dev_out) return GMC_EINVAL;
   if (!h->initialized) return GMC_ESTATE;
   DeviceGuard g(h->device);
+  GMC_TRY_ST(flush(h, static_cast<cudaStream_t>(stream)));
+  GMC_TRY(order_after_flush(h, static_cast<cudaStream_t>(stream), false));
   GMC_TRY(cudaMemcpyAsync(w_dev_out, h->w, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice,
                           static_cast<cudaStream_t>(stream)));
   return GMC_OK;
@@ -570,6 +658,8 @@ int gmc_get_residual(gmc_t h, int32_t k, float* e_dev_out, void* stream) {
   if (!h || !e_dev_out || k < 0 || k >= h->K) return GMC_EINVAL;
   if (!h->initialized) return GMC_ESTATE;
   DeviceGuard g(h->device);
+  GMC_TRY_ST(flush(h, static_cast<cudaStream_t>(stream)));
+  GMC_TRY(order_after_flush(h, static_cast<cudaStream_t>(stream), false));
   GMC_TRY(cudaMemcpyAsync(e_dev_out, h->e + (int64_t)k * h->ld, (size_t)h->d * sizeof(float),
                           cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream)));
   return GMC_OK;
@@ -611,6 +701,8 @@ int gmc_get_worker_params(gmc_t h, int32_t k, float* out_dev, void* stream) {
   if (!h || !out_dev || k < 0 || k >= h->K) return GMC_EINVAL;
   if (!h->initialized) return GMC_ESTATE;
   DeviceGuard g(h->device);
+  GMC_TRY_ST(flush(h, static_cast<cudaStream_t>(stream)));
+  GMC_TRY(order_after_flush(h, static_cast<cudaStream_t>(stream), false));
   DetachArgs D{h->w, h->e, h->ld, h->d, h->lambda * h->eta, out_dev, h->d, k, k + 1};
   GMC_TRY(launch_detach(D, static_cast<cudaStream_t>(stream)));
   return GMC_OK;
@@ -620,6 +712,7 @@ int gmc_get_stats(gmc_t h, uint64_t* counters_host, int32_t n, double* rcc_host)
   if (!h || n < 0 || n > GMC_STAT_COUNT || (n > 0 && !counters_host)) return GMC_EINVAL;
   if (!h->initialized) return GMC_ESTATE;
   DeviceGuard g(h->device);
+  GMC_TRY_ST(flush(h, h->aux));
   GMC_TRY(cudaDeviceSynchronize());
   Counters c;
   GMC_TRY(cudaMemcpy(&c, h->total_ctr, sizeof(Counters), cudaMemcpyDeviceToHost));

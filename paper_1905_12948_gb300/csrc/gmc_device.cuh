@@ -15,6 +15,7 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kSampleThreads = 1024;
 constexpr int kSampleChunks = 4096;          // sampled 8-element chunks per worker
 constexpr int kSampleAll = 32768;            // d at or below which every element is sampled
+constexpr int kSampleSlots = 8 * kSampleChunks;  // sampled positions (= kSampleAll)
 constexpr int kHistBins = 2048;              // first radix digit: key bits 30..20
 constexpr int kRelBins = 2048;               // bins of the candidates' relative histogram
 constexpr int kBucketCap = 12288;            // candidates of one bin ranked in shared memory

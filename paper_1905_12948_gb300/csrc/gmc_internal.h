@@ -52,8 +52,17 @@ struct TopkArgs {
   uint32_t* chunk_cnt;       // K x n_tiles x kChunksPerTile
   uint32_t* mask;            // d: workers that sent each coordinate (bit k), zero between steps
   const uint32_t* cand_idx_prev;    // previous step's sub-chunks
+  const float* cand_val_prev;
   const uint32_t* chunk_base_prev;
   const uint32_t* chunk_cnt_prev;
+  // Deferred aggregation: the sum of a step's sent pairs into w and the
+  // zeroing of its residuals can be left to the next step's bulk pass, which
+  // streams every coordinate anyway (see k_accumulate_bulk).
+  int pending;               // the previous step's aggregation is still to be applied
+  float a_prev;              // fl(eta/K) of that step
+  const uint32_t* smask_rd;  // kSampleSlots: senders (bit k) of the previous step at each sampled position
+  uint32_t* smask_wr;        // the same for this step (cleared by the sample kernel)
+  Counters* total_ctr;       // running totals: the deferred aggregation counts there
   Counters* step_ctr;
   unsigned* status;
 };
@@ -102,7 +111,17 @@ cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s);
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s);
-cudaError_t launch_aggregate(const TopkArgs& A, int grid, cudaStream_t s);
+constexpr int kBulkTile = 4096;  // tile of the bulk-copy accumulate pass (k_accumulate_bulk)
+
+// k_mark over worker k's sent pairs; mode is a bit set of kMark*.
+constexpr int kMarkSent = 1;    // mark the candidates not sent, count the non-zero sent values
+constexpr int kMarkMask = 2;    // record the senders of every coordinate in mask (for k_owner_sum)
+constexpr int kMarkSample = 4;  // record the senders at the sampled positions only (smask_wr)
+cudaError_t launch_mark(const TopkArgs& A, int mode, int grid, cudaStream_t s);
+// Sum of the sent pairs into w (with a_prev), residuals to +0 where sent,
+// w_{t+1} - w_t into dlt, mask cleared; counts into step_ctr and total_ctr
+// (either may be null).
+cudaError_t launch_owner_sum(const TopkArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_gather_selected(const TopkArgs& A, int k, uint32_t* idx_out, float* val_out,
                                    cudaStream_t s);
 cudaError_t launch_rbgs_pick(const RbgsArgs& A, cudaStream_t s);

@@ -67,9 +67,33 @@ __device__ __forceinline__ uint32_t warp_excl_scan(uint32_t x, uint32_t* total) 
   return incl - x;
 }
 
+// w_{t+1}[j] - w_t[j] at a coordinate whose aggregation is still pending: the
+// senders' values are still in e (they were this step's accumulators), w
+// still holds w_t. Sum in ascending worker order from +0 (Alg. 1).
+__device__ __noinline__ float pending_delta(const TopkArgs& A, uint32_t senders, int64_t j) {
+  float sum = 0.f;
+  for (uint32_t m = senders; m; m &= m - 1u)
+    sum = __fadd_rn(sum, __ldcg(A.e + (int64_t)(__ffs(m) - 1) * A.ld + j));
+  const float wo = A.w[j];
+  return __fsub_rn(__fsub_rn(wo, __fmul_rn(A.a_prev, sum)), wo);
+}
+
+// Slot of coordinate j among the sampled positions, or -1: the sample takes
+// 8 consecutive coordinates from (c * d / chunks) rounded down to a multiple
+// of 8, for c = 0 .. chunks-1 (every coordinate when chunks = 0).
+__device__ __forceinline__ int sample_slot(const TopkArgs& A, uint32_t j) {
+  if (!A.sample_chunks) return j < (uint32_t)kSampleSlots ? (int)j : -1;
+  const int64_t q = (int64_t)(j & ~7u), C = A.sample_chunks;
+  const int64_t c = (q * C + A.d - 1) / A.d;  // first chunk starting at or after q
+  if (c >= C || (((c * A.d) / C) & ~int64_t(7)) != q) return -1;
+  return (int)(c * 8 + (j & 7u));
+}
+
 // ---------------------------------------------------------------------------
 // sample: blocks spread over the workers' samples; the last block of a worker
-// fixes two radix digits of the sample's r-th largest key.
+// fixes two radix digits of the sample's r-th largest key. Where the previous
+// step's aggregation is pending, the sampled accumulator is formed as if it
+// had been applied (residual +0 where the worker sent, the pending delta).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   __shared__ uint32_t hist[kHistBins];
@@ -78,6 +102,10 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
   if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) A.big_tiles[0] = 0;
+  if (k == 0) {  // this step's sampled-position senders start empty
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < kSampleSlots; i += gridDim.x * blockDim.x)
+      A.smask_wr[i] = 0u;
+  }
   if (A.dense_mode) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       S.theta = kNoCandidate;
@@ -110,6 +138,11 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
         ev[q] = ek[j];
         gv[q] = gk[j];
         dv[q] = A.dlt[j];
+        const uint32_t m = A.smask_rd[i];
+        if (m) {  // the previous step's aggregation is still pending at j
+          if ((m >> k) & 1u) ev[q] = 0.f;
+          dv[q] = pending_delta(A, m, j);
+        }
       }
     }
 #pragma unroll
@@ -237,6 +270,103 @@ __device__ __forceinline__ void stage_delta_warp(const TopkArgs& A, int64_t tile
   __syncwarp();
 }
 
+// The previous step's aggregation (Alg. 1: w_{t+1} = w_t - (eta/K) sum_k C_k(.),
+// e_{t+1,k} = e_{t+1/2,k} - C_k(.)) applied on one warp's sub-tile
+// [sub0, sub0 + n), n <= 512, when it was left pending: from the previous
+// step's sent pairs of this sub-tile (sub-chunks (k', tile, w)) it records the
+// senders of every coordinate in mkw, sums their values in ascending worker
+// order from +0, writes w_{t+1} over w_t there and leaves w_{t+1} - w_t in dlw.
+// The residuals are not touched: the caller takes e = +0 where mkw has its bit.
+__device__ __forceinline__ void stage_pending_warp(const TopkArgs& A, int64_t tile, int w,
+                                                   uint32_t sub0, int n, float* dlw, uint32_t* mkw,
+                                                   int lane, uint32_t& uni, uint32_t& chg) {
+  for (int i = lane; i < n / 4; i += 32) {
+    reinterpret_cast<float4*>(dlw)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    reinterpret_cast<uint4*>(mkw)[i] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  __syncwarp();
+  const uint32_t lt = lanemask_lt();
+  for (int k0 = 0; k0 < A.K; k0 += 32) {
+    const int kk = k0 + lane;
+    uint32_t base = 0, cnt = 0;
+    if (kk < A.K) {
+      const int64_t c = ((int64_t)kk * A.n_tiles + tile) * kChunksPerTile + w;
+      base = A.chunk_base_prev[c];
+      cnt = A.chunk_cnt_prev[c];
+    }
+    uint32_t total;
+    const uint32_t pre = warp_excl_scan(cnt, &total);
+    // entries run through the workers in ascending order, 32 per round
+    for (uint32_t e0 = 0; e0 < total; e0 += 32) {
+      const uint32_t e = e0 + lane;
+      int src = 0;
+#pragma unroll 1
+      for (int l = 1; l < 32; ++l) {
+        const uint32_t pl = __shfl_sync(0xffffffffu, pre, l);
+        const uint32_t cl = __shfl_sync(0xffffffffu, cnt, l);
+        if (cl && pl <= e) src = l;
+      }
+      const uint32_t b = __shfl_sync(0xffffffffu, base, src);
+      const uint32_t p = __shfl_sync(0xffffffffu, pre, src);
+      bool act = false;
+      uint32_t l = 0;
+      float v = 0.f;
+      if (e < total) {
+        const uint32_t at = b + (e - p);
+        if (at < A.cap) {
+          const int64_t q = (int64_t)(k0 + src) * A.cap + at;
+          const uint32_t j = A.cand_idx_prev[q];
+          if (!(j & kUnsent)) {
+            const int64_t ll = (int64_t)j - sub0;
+            if (ll >= 0 && ll < n) {
+              act = true;
+              l = (uint32_t)ll;
+              v = A.cand_val_prev[q];
+              atomicOr(&mkw[l], 1u << (k0 + src));
+            } else {
+              atomicOr(A.status, kStatusInternal);
+            }
+          }
+        }
+      }
+      // lanes holding the same coordinate add one at a time, in lane (= worker) order
+      const uint32_t peers = __match_any_sync(0xffffffffu, act ? (int)l : -1 - lane);
+      const uint32_t r = __popc(peers & lt);
+      const uint32_t rmax = __reduce_max_sync(0xffffffffu, act ? r : 0u);
+      for (uint32_t turn = 0; turn <= rmax; ++turn) {
+        if (act && r == turn) dlw[l] = __fadd_rn(dlw[l], v);
+        __syncwarp();
+      }
+    }
+  }
+  __syncwarp();
+  // coordinates of the union: w_{t+1} = w_t - a * sum (all loads issued first)
+  float wo[16];
+  uint32_t has = 0;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const int l = lane + 32 * i;
+    wo[i] = 0.f;
+    if (l < n && mkw[l]) {
+      has |= 1u << i;
+      wo[i] = A.w[sub0 + l];
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    if ((has >> i) & 1u) {
+      const int l = lane + 32 * i;
+      const float wn = __fsub_rn(wo[i], __fmul_rn(A.a_prev, dlw[l]));
+      A.w[sub0 + l] = wn;
+      const float dd = __fsub_rn(wn, wo[i]);
+      dlw[l] = dd;
+      ++uni;
+      chg += dd != 0.f;
+    }
+  }
+  __syncwarp();
+}
+
 // Candidate flags (bit i: value i is a candidate) of 4 consecutive values at
 // sub-tile offset l; `lim` = valid values in the sub-tile (all when it is full).
 __device__ __forceinline__ uint32_t cand_bits(const float v[4], int l, int lim, uint32_t theta) {
@@ -354,7 +484,7 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 // and every wait is bounded.
 // ---------------------------------------------------------------------------
 namespace bulk {
-constexpr int kT = 4096;
+constexpr int kT = kBulkTile;
 constexpr int kStages = 6;
 constexpr int kConsumers = kChunksPerTile;
 constexpr int kSub = kT / kConsumers;      // 512
@@ -364,12 +494,14 @@ struct Smem {
   float e[kStages][kT];
   float g[kStages][kGLen];
   float dl[kConsumers][kSub];
+  uint32_t mk[kConsumers][kSub];           // senders of the pending aggregation (bit k)
   uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
   uint64_t empty[kStages];                 // all consumer warps read the stage (8 arrivals)
   int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
   uint32_t rcnt[kMaxK];                    // candidates this CTA wrote per worker (its region)
   uint32_t theta[kMaxK];
 };
+static_assert(sizeof(Smem) <= 232448, "bulk pass shared memory above the 227 KB a block may use");
 }  // namespace bulk
 
 __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkArgs A) {
@@ -430,20 +562,35 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   // ---- consumers ----
   const uint32_t lt = lanemask_lt();
   float* dlw = sm.dl[warp];
+  uint32_t* mkw = sm.mk[warp];
   const uint32_t region0 = blockIdx.x * A.cap_region;
   const uint32_t region_end = region0 + A.cap_region;
-  uint32_t nonfinite = 0;
+  uint32_t nonfinite = 0, uni = 0, chg = 0;
   uint32_t item = 0;
   bool ok = true;
   for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
     const uint32_t s0 = (uint32_t)(tile * kT) + warp * kSub;
-    stage_delta_warp(A, tile, warp, s0, kSub, dlw, lane);
+    // w_t - w_{t-1} of this sub-tile (and, when the previous step's
+    // aggregation is pending, its senders: their residual is +0)
+    if (A.pending) {
+      stage_pending_warp(A, tile, warp, s0, kSub, dlw, mkw, lane, uni, chg);
+    } else {
+      stage_delta_warp(A, tile, warp, s0, kSub, dlw, lane);
+    }
+    float4 dl4[kSub / 128];
+    uint4 mk4[kSub / 128];
+#pragma unroll
+    for (int u = 0; u < kSub / 128; ++u) {
+      const int l = u * 128 + lane * 4;
+      dl4[u] = *reinterpret_cast<const float4*>(dlw + l);
+      mk4[u] = A.pending ? *reinterpret_cast<const uint4*>(mkw + l) : make_uint4(0u, 0u, 0u, 0u);
+    }
     const int64_t rem = A.d - (int64_t)s0;
     const int lim = rem < kSub ? (int)rem : kSub;
     const bool full = lim == kSub;
     for (int k = 0; k < A.K; ++k, ++item) {
       const uint32_t s = item % kStages, r = item / kStages;
-      if (!wait_bounded(&sm.full[s], r & 1)) {
+      if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
         ok = false;
         break;
       }
@@ -474,11 +621,12 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
           if (l + 2 >= lim) g4.z = 0.f;
           if (l + 3 >= lim) g4.w = 0.f;
         }
-        const float4 d4 = *reinterpret_cast<const float4*>(dlw + l);
-        v[u][0] = accumulate(e4.x, g4.x, A.c, d4.x);
-        v[u][1] = accumulate(e4.y, g4.y, A.c, d4.y);
-        v[u][2] = accumulate(e4.z, g4.z, A.c, d4.z);
-        v[u][3] = accumulate(e4.w, g4.w, A.c, d4.w);
+        const float4 d4 = dl4[u];
+        const uint4 m4 = mk4[u];
+        v[u][0] = accumulate(((m4.x >> k) & 1u) ? 0.f : e4.x, g4.x, A.c, d4.x);
+        v[u][1] = accumulate(((m4.y >> k) & 1u) ? 0.f : e4.y, g4.y, A.c, d4.y);
+        v[u][2] = accumulate(((m4.z >> k) & 1u) ? 0.f : e4.z, g4.z, A.c, d4.z);
+        v[u][3] = accumulate(((m4.w >> k) & 1u) ? 0.f : e4.w, g4.w, A.c, d4.w);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.empty[s]);  // this warp is done reading stage s
@@ -520,6 +668,12 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   if (nonfinite) {
     atomicOr(A.status, kStatusNonfinite);
     atomicAdd(&A.step_ctr->v[kNonfinite], (unsigned long long)nonfinite);
+  }
+  if (A.pending) {  // the previous step's counts, straight into the totals
+    const uint32_t u_w = __reduce_add_sync(0xffffffffu, uni);
+    const uint32_t c_w = __reduce_add_sync(0xffffffffu, chg);
+    if (lane == 0 && u_w) atomicAdd(&A.total_ctr->v[kUnion], (unsigned long long)u_w);
+    if (lane == 0 && c_w) atomicAdd(&A.total_ctr->v[kChanged], (unsigned long long)c_w);
   }
   // every consumer warp is past its last reservation: publish the region counts
   asm volatile("bar.sync 1, %0;" ::"r"(kConsumers * 32) : "memory");
@@ -874,7 +1028,7 @@ __device__ __forceinline__ void sent_part(const TopkArgs& A, int k, int p, int n
   }
 }
 
-__global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A) {
+__global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A, int mode) {
   const int k = blockIdx.y;
   const uint32_t T = A.sel[k].T, tidx = A.sel[k].t_idx;
   const uint32_t bit = 1u << k;
@@ -897,9 +1051,13 @@ __global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A) {
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const uint32_t j = jq[q];
-        if (j >= (uint32_t)A.d) continue;
-        if (selected(mag_key(vq[q]), j, T, tidx)) {
-          atomicOr(&A.mask[j], bit);
+        if (j >= (uint32_t)A.d) continue;  // beyond the part, or marked not sent already
+        if (!(mode & kMarkSent) || selected(mag_key(vq[q]), j, T, tidx)) {
+          if (mode & kMarkMask) atomicOr(&A.mask[j], bit);
+          if (mode & kMarkSample) {
+            const int slot = sample_slot(A, j);
+            if (slot >= 0) atomicOr(&A.smask_wr[slot], bit);
+          }
           nnz += (vq[q] != 0.f);
         } else {
           ci[i0 + q * blockDim.x + threadIdx.x] = j | kUnsent;
@@ -907,8 +1065,10 @@ __global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A) {
       }
     }
   }
-  nnz = warp_sum(nnz);
-  if ((threadIdx.x & 31) == 0 && nnz) atomicAdd(&A.step_ctr->v[kNnz], nnz);
+  if (mode & kMarkSent) {
+    nnz = warp_sum(nnz);
+    if ((threadIdx.x & 31) == 0 && nnz) atomicAdd(&A.step_ctr->v[kNnz], nnz);
+  }
 }
 
 __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
@@ -940,7 +1100,7 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
           A.e[(int64_t)b * A.ld + j] = 0.f;  // e_{t+1,b} = e_{t+1/2,b} - C(.) = +0 where sent
         }
       }
-      const float wn = __fsub_rn(wo, __fmul_rn(A.a, sum));
+      const float wn = __fsub_rn(wo, __fmul_rn(A.a_prev, sum));
       A.w[j] = wn;
       const float dd = __fsub_rn(wn, wo);
       A.dlt[j] = dd;
@@ -952,8 +1112,11 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
   uni = warp_sum(uni);
   changed = warp_sum(changed);
   if ((threadIdx.x & 31) == 0) {
-    if (uni) atomicAdd(&A.step_ctr->v[kUnion], uni);
-    if (changed) atomicAdd(&A.step_ctr->v[kChanged], changed);
+    for (Counters* c : {A.step_ctr, A.total_ctr}) {
+      if (!c) continue;
+      if (uni) atomicAdd(&c->v[kUnion], uni);
+      if (changed) atomicAdd(&c->v[kChanged], changed);
+    }
   }
 }
 
@@ -1069,12 +1232,13 @@ cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_aggregate(const TopkArgs& A, int grid, cudaStream_t s) {
-  const dim3 g(grid, A.K);
-  k_mark<<<g, kThreads, 0, s>>>(A);
-  cudaError_t err = cudaGetLastError();
-  if (err != cudaSuccess) return err;
-  k_owner_sum<<<g, kThreads, 0, s>>>(A);
+cudaError_t launch_mark(const TopkArgs& A, int mode, int grid, cudaStream_t s) {
+  k_mark<<<dim3(grid, A.K), kThreads, 0, s>>>(A, mode);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_owner_sum(const TopkArgs& A, int grid, cudaStream_t s) {
+  k_owner_sum<<<dim3(grid, A.K), kThreads, 0, s>>>(A);
   return cudaGetLastError();
 }
 
