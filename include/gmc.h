@@ -80,10 +80,12 @@ typedef struct gmc_ctx* gmc_t;
 #define GMC_KERNEL_ACCUMULATE  0 /* fused accumulator + candidate filter (top-k), one dense pass */
 #define GMC_KERNEL_RBGS_STEP   1 /* fused accumulator + RBGS compress + aggregate + update */
 #define GMC_KERNEL_SAMPLE      2 /* sampled threshold per worker */
-#define GMC_KERNEL_SELECT      3 /* exact radix select among candidates (3 launches per step) */
+#define GMC_KERNEL_SELECT      3 /* exact select among candidates (2 launches per step) */
 #define GMC_KERNEL_DENSE       4 /* exact dense select for workers that fell back */
-#define GMC_KERNEL_COMPACT     5 /* index-ordered compaction of C(v) (3 launches per step) */
-#define GMC_KERNEL_AGGREGATE   6 /* worker-ordered aggregate + update (top-k) */
+#define GMC_KERNEL_COMPACT     5 /* reserved: no launch (the dense pass writes C(v) as
+                                    index-ordered sub-chunks) */
+#define GMC_KERNEL_AGGREGATE   6 /* marks the sent pairs; when the aggregation is not
+                                    deferred also the worker-ordered aggregate + update */
 #define GMC_KERNEL_RBGS_PICK   7 /* RBGS block choice (Floyd sampling) */
 #define GMC_KERNEL_DETACH      8 /* GMC+ detached points */
 #define GMC_KERNEL_OTHER       9 /* counters and small bookkeeping */
@@ -139,7 +141,18 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream);
  * g_{t,k} at grads_dev[k*d .. k*d+d)), device memory, read-only, borrowed until
  * the stream has passed the step; any alignment. Enqueues kernels only; never
  * synchronises. Non-finite accumulator values still complete the step
- * deterministically and are reported by gmc_check as GMC_ENONFINITE. */
+ * deterministically and are reported by gmc_check as GMC_ENONFINITE.
+ *
+ * Deferred aggregation (top-k with d >= 4096 * 2 * SMs, about 1.25 M on GB300):
+ * the step selects and records C(e_{t+1/2,k}) but leaves the last line of
+ * Alg. 1 -- w_{t+1} = w_t - (eta/K) sum_k C_k and the zeroing of the sent
+ * residuals -- to the next gmc_step, whose single pass over the tiles applies
+ * it before forming its own accumulator. The results are the same, bit for
+ * bit: every call that reads the state (gmc_get_params, gmc_get_residual,
+ * gmc_get_worker_params, gmc_get_stats) first applies a pending aggregation,
+ * on its own stream after the step. gmc_step_host and a set detach output
+ * apply it within the step. Because a getter writes the state, a getter on
+ * one stream and a later gmc_step on another are ordered by the library. */
 int gmc_step(gmc_t h, const float* grads_dev, void* stream);
 
 /* gmc_step_host -- gmc_step from host memory: copies grads_host (K x d fp32,
@@ -150,10 +163,12 @@ int gmc_step(gmc_t h, const float* grads_dev, void* stream);
  * stream has passed the call (or NULL to skip the read-back). */
 int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, void* stream);
 
-/* gmc_get_params -- copy w_t (d floats) into w_dev_out. */
+/* gmc_get_params -- copy w_t (d floats) into w_dev_out (applying a pending
+ * aggregation first, see gmc_step). */
 int gmc_get_params(gmc_t h, float* w_dev_out, void* stream);
 
-/* gmc_get_residual -- copy e_{t,k} (d floats) into e_dev_out. */
+/* gmc_get_residual -- copy e_{t,k} (d floats) into e_dev_out (applying a
+ * pending aggregation first). */
 int gmc_get_residual(gmc_t h, int32_t k, float* e_dev_out, void* stream);
 
 /* gmc_get_selected -- synchronising. The last step's C(e_{t-1/2,k}) of worker k
@@ -172,7 +187,8 @@ int64_t gmc_selected_capacity(gmc_t h);
  * w_{t,k} = w_t - lambda*eta*e_{t,k} (Alg. 2), written to out_dev (d floats). */
 int gmc_get_worker_params(gmc_t h, int32_t k, float* out_dev, void* stream);
 
-/* gmc_get_stats -- synchronising. Cumulative counters since gmc_set_params
+/* gmc_get_stats -- synchronising (applies a pending aggregation first, on a
+ * library stream ordered after the last step). Cumulative counters since gmc_set_params
  * (n <= GMC_STAT_COUNT slots copied into counters_host) and the relative
  * communication cost of Sec. 5, RCC = (K*sum_t ||w_{t+1}-w_t||_0 +
  * sum_t sum_k ||C_k||_0) / (d K T), halved for RBGS (no indices, Sec. 5.2). */
