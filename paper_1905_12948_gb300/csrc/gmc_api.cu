@@ -60,12 +60,11 @@ struct gmc_ctx {
   uint32_t* big_tiles = nullptr;
   uint32_t* rcount = nullptr;
   int regions = 1;
-  uint32_t cap_region = 0;
+  uint32_t cap_region = 0, cap_part = 0;
   int sample_blocks = 1;
   uint32_t* cand_idx[2] = {nullptr, nullptr};
   float* cand_val[2] = {nullptr, nullptr};
-  uint32_t* chunk_base[2] = {nullptr, nullptr};
-  uint32_t* chunk_cnt[2] = {nullptr, nullptr};
+  uint2* chunk[2] = {nullptr, nullptr};
   uint32_t* mask = nullptr;
   uint32_t* smask[2] = {nullptr, nullptr};  // senders at the sampled positions, by step parity
   // deferred aggregation (bulk top-k pass): the last step's sent pairs are
@@ -221,11 +220,11 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.big_tiles = h->big_tiles;
   A.regions = h->regions;
   A.cap_region = h->cap_region;
+  A.cap_part = h->cap_part;
   A.rcount = h->rcount;
   A.cand_idx = h->cand_idx[cur];
   A.cand_val = h->cand_val[cur];
-  A.chunk_base = h->chunk_base[cur];
-  A.chunk_cnt = h->chunk_cnt[cur];
+  A.chunk = h->chunk[cur];
   A.mask = h->mask;
   A.cand_idx_prev = h->cand_idx[prev];
   A.cand_val_prev = h->cand_val[prev];
@@ -234,8 +233,7 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.total_ctr = h->total_ctr;
   A.pending = 0;
   A.a_prev = A.a;
-  A.chunk_base_prev = h->chunk_base[prev];
-  A.chunk_cnt_prev = h->chunk_cnt[prev];
+  A.chunk_prev = h->chunk[prev];
   A.step_ctr = h->step_ctr;
   A.status = h->status;
   return A;
@@ -459,15 +457,19 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     }
     h->grid_acc = (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * accumulate_blocks_per_sm(h->tile));
     h->grid_agg = 0;  // set below from the candidate regions
-    // candidate slots: the bulk pass gives every CTA its own region per worker
-    // (twice its share of the expected candidates, plus slack); otherwise one region
+    // candidate slots: the bulk pass gives every CTA its own region per worker,
+    // one part per consumer warp (twice its share of the expected candidates,
+    // plus slack, in whole 128-byte lines); otherwise one region
     const uint32_t cap0 = h->cap;
     if (h->tile == kBulkTile) {
       h->regions = h->grid_acc;
-      h->cap_region = (uint32_t)(((2ull * cap0 + h->regions - 1) / h->regions + 1024 + 3) & ~3ull);
+      const uint64_t share = (2ull * cap0 + h->regions * kChunksPerTile - 1) / (h->regions * kChunksPerTile);
+      h->cap_part = (uint32_t)((share + 128 + 31) & ~31ull);
+      h->cap_region = h->cap_part * kChunksPerTile;
     } else {
       h->regions = 1;
       h->cap_region = (cap0 + 3) & ~3u;
+      h->cap_part = h->cap_region;
     }
     h->cap = (uint32_t)std::min<uint64_t>((uint64_t)h->regions * h->cap_region, 0xfffffff0ull);
     const int64_t per = (h->cap + 8191) / 8192;
@@ -495,7 +497,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->bucket, (size_t)K * 2 * kBucketCap)) != cudaSuccess ||
         (err = dalloc(h, &h->sample_keys, (size_t)K * 8 * kSampleChunks)) != cudaSuccess ||
         (err = dalloc(h, &h->big_tiles, (size_t)h->n_tiles + 1)) != cudaSuccess ||
-        (err = dalloc(h, &h->rcount, (size_t)K * h->regions)) != cudaSuccess ||
+        (err = dalloc(h, &h->rcount, (size_t)K * h->regions * kChunksPerTile)) != cudaSuccess ||
         (err = dalloc(h, &h->mask, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->smask[0], (size_t)kSampleSlots)) != cudaSuccess ||
         (err = dalloc(h, &h->smask[1], (size_t)kSampleSlots)) != cudaSuccess)
@@ -507,8 +509,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     for (int p = 0; p < 2; ++p) {
       if ((err = dalloc(h, &h->cand_idx[p], (size_t)K * h->cap)) != cudaSuccess ||
           (err = dalloc(h, &h->cand_val[p], (size_t)K * h->cap)) != cudaSuccess ||
-          (err = dalloc(h, &h->chunk_base[p], (size_t)Kt * kChunksPerTile)) != cudaSuccess ||
-          (err = dalloc(h, &h->chunk_cnt[p], (size_t)Kt * kChunksPerTile)) != cudaSuccess)
+          (err = dalloc(h, &h->chunk[p], (size_t)Kt * kChunksPerTile)) != cudaSuccess)
         return fail(err);
     }
   } else {
@@ -602,7 +603,7 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
   GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
   if (h->compressor == GMC_TOPK) {
     for (int p = 0; p < 2; ++p)
-      GMC_TRY(cudaMemsetAsync(h->chunk_cnt[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint32_t), s));
+      GMC_TRY(cudaMemsetAsync(h->chunk[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint2), s));
     GMC_TRY(cudaMemsetAsync(h->sel, 0, (size_t)h->K * sizeof(WorkerSel), s));
     GMC_TRY(cudaMemsetAsync(h->mask, 0, (size_t)h->ld * sizeof(uint32_t), s));
     for (int p = 0; p < 2; ++p)

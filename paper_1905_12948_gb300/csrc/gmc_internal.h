@@ -33,8 +33,9 @@ struct TopkArgs {
   uint32_t ksel;             // k
   uint32_t cap;              // candidate slots per worker = regions * cap_region
   int regions;               // candidate regions per worker: one per accumulate CTA (1 = shared)
-  uint32_t cap_region;       // slots per region
-  uint32_t* rcount;          // K x regions: candidates written in each region
+  uint32_t cap_region;       // slots per region: kChunksPerTile warp parts of cap_part
+  uint32_t cap_part;         // slots per warp part (a multiple of 32: whole 128-byte lines)
+  uint32_t* rcount;          // K x regions x kChunksPerTile: candidates written in each part
   uint32_t sample_rank;      // rank of the sampled threshold
   int sample_chunks;         // 0 = sample every element
   int sample_blocks;         // blocks per worker of the sample kernel
@@ -48,13 +49,11 @@ struct TopkArgs {
   uint32_t* big_tiles;       // [0]: count, then tile ids left to the block aggregate
   uint32_t* cand_idx;        // current chunks: K x cap
   float* cand_val;
-  uint32_t* chunk_base;      // K x n_tiles x kChunksPerTile
-  uint32_t* chunk_cnt;       // K x n_tiles x kChunksPerTile
+  uint2* chunk;              // sub-chunk (base, count): n_tiles x kChunksPerTile x K, see chunk_at
   uint32_t* mask;            // d: workers that sent each coordinate (bit k), zero between steps
   const uint32_t* cand_idx_prev;    // previous step's sub-chunks
   const float* cand_val_prev;
-  const uint32_t* chunk_base_prev;
-  const uint32_t* chunk_cnt_prev;
+  const uint2* chunk_prev;
   // Deferred aggregation: the sum of a step's sent pairs into w and the
   // zeroing of its residuals can be left to the next step's bulk pass, which
   // streams every coordinate anyway (see k_accumulate_bulk).
@@ -66,6 +65,13 @@ struct TopkArgs {
   Counters* step_ctr;
   unsigned* status;
 };
+
+// Slot of sub-chunk (k, tile, w) in the sub-chunk tables: a tile's entries are
+// contiguous, each eighth of the tile holding its K workers side by side, so
+// one warp writes the K entries of its eighth with one store.
+__host__ __device__ __forceinline__ int64_t chunk_at(const TopkArgs& A, int k, int64_t tile, int w) {
+  return (tile * kChunksPerTile + w) * A.K + k;
+}
 
 // Arguments of the RBGS kernels.
 struct RbgsArgs {
@@ -135,7 +141,7 @@ cudaError_t launch_finalize(Counters* step, Counters* total, unsigned long long 
 // Occupancy-derived persistent grid sizes.
 int accumulate_blocks_per_sm(int tile);
 int rbgs_blocks_per_sm();
-int accumulate_smem_bytes(int tile);
+int accumulate_smem_bytes(int tile, int K);
 cudaError_t configure_topk_kernels();
 cudaError_t configure_rbgs_kernels();
 

@@ -23,7 +23,7 @@
 namespace gmc {
 namespace {
 
-constexpr int kMaxK = 64;  // workers supported by the top-k kernels
+constexpr int kMaxK = 32;  // workers supported by the top-k kernels (one lane or mask bit each)
 
 __device__ __forceinline__ float4 load_g4(const float* __restrict__ g, int64_t j, int64_t d,
                                           int mode) {
@@ -231,9 +231,9 @@ __device__ __forceinline__ void stage_delta_warp(const TopkArgs& A, int64_t tile
       const int kk = k0 + lane;
       uint32_t base = 0, cnt = 0;
       if (kk < A.K) {
-        const int64_t c = ((int64_t)kk * A.n_tiles + tile) * kChunksPerTile + w;
-        base = A.chunk_base_prev[c];
-        cnt = A.chunk_cnt_prev[c];
+        const uint2 bc = A.chunk_prev[chunk_at(A, kk, tile, w)];
+        base = bc.x;
+        cnt = bc.y;
       }
       uint32_t total;
       const uint32_t pre = warp_excl_scan(cnt, &total);
@@ -290,9 +290,9 @@ __device__ __forceinline__ void stage_pending_warp(const TopkArgs& A, int64_t ti
     const int kk = k0 + lane;
     uint32_t base = 0, cnt = 0;
     if (kk < A.K) {
-      const int64_t c = ((int64_t)kk * A.n_tiles + tile) * kChunksPerTile + w;
-      base = A.chunk_base_prev[c];
-      cnt = A.chunk_cnt_prev[c];
+      const uint2 bc = A.chunk_prev[chunk_at(A, kk, tile, w)];
+      base = bc.x;
+      cnt = bc.y;
     }
     uint32_t total;
     const uint32_t pre = warp_excl_scan(cnt, &total);
@@ -461,11 +461,7 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
         for (int u = 0; u < U; ++u)
           write_group(v[u], s0 + u * 128 + lane * 4, bits[u], lt, pos, A.cap, ci, cv, nonfinite);
       }
-      if (lane == 0) {
-        const int64_t c = ((int64_t)k * A.n_tiles + tile) * kChunksPerTile + warp;
-        A.chunk_base[c] = base;
-        A.chunk_cnt[c] = cnt;
-      }
+      if (lane == 0) A.chunk[chunk_at(A, k, tile, warp)] = make_uint2(base, cnt);
     }
   }
   if (nonfinite) {
@@ -478,14 +474,28 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 // bulk-copy version (tiles of 4096). One persistent CTA per SM. A producer
 // thread streams each (tile, worker) item's e and g into a ring of shared-
 // memory stages with cp.async.bulk; eight consumer warps, each owning 512
-// elements of the tile, read their part, release the stage, store v over e
-// and reserve their sub-chunk in this CTA's region of the candidate buffer
-// with a shared-memory atomic. Producer and consumers meet only at mbarriers
-// and every wait is bounded.
+// elements of every tile, read their part, release the stage, store v over e
+// and append their candidates to their own part of this CTA's region of the
+// candidate buffer (one part per warp and worker). Candidates are staged in
+// shared memory and leave in whole 128-byte lines. Producer and consumers
+// meet only at mbarriers and every wait is bounded.
+//
+// Each consumer warp forms its sub-tile's w_t - w_{t-1} (and applies the
+// previous step's aggregation when it was left pending) from the previous
+// step's sent pairs. Those are reached through two dependent loads -- the
+// sub-chunk table, then the pairs -- and the pending case reads w at the
+// pairs' coordinates: a chain of three memory latencies. The warp runs that
+// chain as a pipeline over its tiles: while it works on tile n it loads w for
+// tile n+1, the pairs of tile n+2 and the sub-chunk entries of tile n+3, so
+// no latency lies on its path. A sub-tile with more than 32 pairs takes the
+// direct path (stage_pending_warp / stage_delta_warp).
 // ---------------------------------------------------------------------------
+#ifndef GMC_BULK_STAGES
+#define GMC_BULK_STAGES 4
+#endif
 namespace bulk {
 constexpr int kT = kBulkTile;
-constexpr int kStages = 6;
+constexpr int kStages = GMC_BULK_STAGES;   // shared-memory ring of (e, g) tiles
 constexpr int kConsumers = kChunksPerTile;
 constexpr int kSub = kT / kConsumers;      // 512
 constexpr int kGLen = kT + 8;              // g stage: up to 3 leading floats of misalignment
@@ -493,16 +503,121 @@ constexpr int kThreadsAll = (kConsumers + 1) * 32;
 struct Smem {
   float e[kStages][kT];
   float g[kStages][kGLen];
-  float dl[kConsumers][kSub];
+  float dl[kConsumers][kSub];              // w_t - w_{t-1} of the warp's sub-tile
   uint32_t mk[kConsumers][kSub];           // senders of the pending aggregation (bit k)
+  uint8_t own[kConsumers][32];             // scratch: worker of each listed pair
   uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
   uint64_t empty[kStages];                 // all consumer warps read the stage (8 arrivals)
   int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
-  uint32_t rcnt[kMaxK];                    // candidates this CTA wrote per worker (its region)
   uint32_t theta[kMaxK];
+  // followed by the candidate staging lines: per consumer warp and worker, 32
+  // indices then 32 values (staging_bytes)
 };
-static_assert(sizeof(Smem) <= 232448, "bulk pass shared memory above the 227 KB a block may use");
+// Dynamic shared memory of the bulk pass for K workers.
+__host__ __device__ constexpr int smem_bytes(int K) {
+  return (int)((sizeof(Smem) + 127) / 128 * 128) + kConsumers * K * 64 * 4;
+}
+static_assert(smem_bytes(kMaxK) <= 232448, "bulk pass shared memory above the 227 KB a block may use");
+
+// The first (up to 32) sent pairs of one sub-tile of the previous step, lane e
+// holding pair e of the list that runs through the workers in ascending order.
+struct Pairs {
+  uint32_t j;      // coordinate, or kUnsent for none
+  float v;         // value (pending aggregation only)
+  int kw;          // worker
+  uint32_t total;  // pairs in the sub-tile (warp-uniform)
+};
 }  // namespace bulk
+
+// Sub-chunk entry (k = lane, tile, w) of the previous step, or none.
+__device__ __forceinline__ uint2 pipe_chunk(const TopkArgs& A, int64_t tile, int w, int lane) {
+  return (A.has_prev && tile < A.n_tiles && lane < A.K) ? A.chunk_prev[chunk_at(A, lane, tile, w)]
+                                                         : make_uint2(0u, 0u);
+}
+
+// Issue the loads of a sub-tile's first 32 pairs from its sub-chunk entries.
+__device__ __forceinline__ bulk::Pairs pipe_pairs(const TopkArgs& A, uint2 cb, uint8_t* own, int lane) {
+  bulk::Pairs P;
+  const uint32_t pre = warp_excl_scan(cb.y, &P.total);
+  for (uint32_t i = 0; i < cb.y && pre + i < 32u; ++i) own[pre + i] = (uint8_t)lane;
+  __syncwarp();
+  const bool has = (uint32_t)lane < P.total;
+  const int src = has ? own[lane] : 0;
+  __syncwarp();
+  const uint32_t b = __shfl_sync(0xffffffffu, cb.x, src);
+  const uint32_t p = __shfl_sync(0xffffffffu, pre, src);
+  P.j = kUnsent;
+  P.v = 0.f;
+  P.kw = src;
+  const uint32_t at = b + ((uint32_t)lane - p);
+  if (has && at < A.cap) {
+    const int64_t q = (int64_t)src * A.cap + at;
+    P.j = A.cand_idx_prev[q];
+    if (A.pending) P.v = A.cand_val_prev[q];
+  }
+  return P;
+}
+
+// Issue the load of w (pending aggregation) or of w_t - w_{t-1} (applied) at a pair.
+__device__ __forceinline__ float pipe_w(const TopkArgs& A, const bulk::Pairs& P) {
+  if ((P.j & kUnsent) || P.j >= (uint32_t)A.d) return 0.f;
+  return A.pending ? A.w[P.j] : A.dlt[P.j];
+}
+
+// A sub-tile's w_t - w_{t-1} into dlw and the pending senders into mkw from
+// its pairs (all of them: total <= 32) and the loaded wv. Pending
+// aggregation (Alg. 1, last line): the senders' values summed in ascending
+// worker order from +0, w_{t+1} = w_t - a * sum written over w, and
+// Δ = w_{t+1} - w_t. Applied before: Δ was left in dlt; read, then cleared.
+// Returns the union coordinate this lane listed (its first sender), or ~0u.
+__device__ __forceinline__ uint32_t apply_pairs(const TopkArgs& A, uint32_t sub0, const bulk::Pairs& P,
+                                                float wv, float* dlw, uint32_t* mkw, int lane, uint32_t lt,
+                                                uint32_t& uni, uint32_t& chg) {
+  using bulk::kSub;
+  for (int i = lane; i < kSub / 4; i += 32) {
+    reinterpret_cast<float4*>(dlw)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    reinterpret_cast<uint4*>(mkw)[i] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  __syncwarp();
+  bool act = false;
+  uint32_t l = 0;
+  if (!(P.j & kUnsent)) {
+    const int64_t ll = (int64_t)P.j - sub0;
+    if (ll >= 0 && ll < kSub) {
+      act = true;
+      l = (uint32_t)ll;
+    } else {
+      atomicOr(A.status, kStatusInternal);
+    }
+  }
+  const bool first = act && atomicOr(&mkw[l], 1u << P.kw) == 0u;  // the coordinate's first sender
+  if (A.pending) {
+    // lanes holding the same coordinate add one at a time, in lane (= worker) order
+    const uint32_t peers = __match_any_sync(0xffffffffu, act ? (int)l : -1 - lane);
+    const uint32_t rk = __popc(peers & lt);
+    const uint32_t rmax = __reduce_max_sync(0xffffffffu, act ? rk : 0u);
+    for (uint32_t turn = 0; turn <= rmax; ++turn) {
+      if (act && rk == turn) dlw[l] = __fadd_rn(dlw[l], P.v);
+      __syncwarp();
+    }
+  }
+  __syncwarp();
+  if (first) {
+    if (A.pending) {
+      const float wn = __fsub_rn(wv, __fmul_rn(A.a_prev, dlw[l]));
+      A.w[P.j] = wn;
+      const float dd = __fsub_rn(wn, wv);
+      dlw[l] = dd;
+      ++uni;
+      chg += dd != 0.f;
+    } else {
+      dlw[l] = wv;          // w_t - w_{t-1}, read once
+      A.dlt[P.j] = 0.f;     // and cleared: this step's aggregate writes the next one
+    }
+  }
+  __syncwarp();
+  return first ? l : ~0u;
+}
 
 __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkArgs A) {
   using namespace bulk;
@@ -516,10 +631,8 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     }
     fence_mbar_init();
   }
-  for (int kk = threadIdx.x; kk < kMaxK; kk += blockDim.x) {
-    sm.rcnt[kk] = 0;
+  for (int kk = threadIdx.x; kk < kMaxK; kk += blockDim.x)
     sm.theta[kk] = kk < A.K ? A.sel[kk].theta : kNoCandidate;
-  }
   __syncthreads();
 
   if (warp == kConsumers) {
@@ -563,31 +676,60 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   const uint32_t lt = lanemask_lt();
   float* dlw = sm.dl[warp];
   uint32_t* mkw = sm.mk[warp];
-  const uint32_t region0 = blockIdx.x * A.cap_region;
-  const uint32_t region_end = region0 + A.cap_region;
+  uint8_t* own = sm.own[warp];
+  // this warp's part of the CTA's region, per worker: slots [part0, part0 + cap_part);
+  // lane k counts worker k's candidates so far
+  const uint32_t part0 = (blockIdx.x * kConsumers + warp) * A.cap_part;
+  uint32_t* stg = reinterpret_cast<uint32_t*>(smem_raw + (sizeof(Smem) + 127) / 128 * 128) +
+                  warp * A.K * 64;
+  uint32_t run = 0;
+  const int64_t stride = gridDim.x;
   uint32_t nonfinite = 0, uni = 0, chg = 0;
   uint32_t item = 0;
   bool ok = true;
-  for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+  // fill the pipeline: pairs of tiles 0 and 1, w of tile 0, entries of tile 2
+  Pairs p0 = pipe_pairs(A, pipe_chunk(A, blockIdx.x, warp, lane), own, lane);
+  Pairs p1 = pipe_pairs(A, pipe_chunk(A, blockIdx.x + stride, warp, lane), own, lane);
+  float w0 = pipe_w(A, p0);
+  uint2 c2 = pipe_chunk(A, blockIdx.x + 2 * stride, warp, lane);
+  for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += stride) {
     const uint32_t s0 = (uint32_t)(tile * kT) + warp * kSub;
-    // w_t - w_{t-1} of this sub-tile (and, when the previous step's
-    // aggregation is pending, its senders: their residual is +0)
-    if (A.pending) {
+    // this sub-tile's w_t - w_{t-1}, and the pending senders (their residual
+    // is +0): at most 32 union coordinates, one per lane (upos, umask), are
+    // zeroed in each worker's stage before it is read; more use per-element masks
+    uint32_t upos = ~0u;
+    bool many = false;
+    if (p0.total <= 32u) {
+      upos = apply_pairs(A, s0, p0, w0, dlw, mkw, lane, lt, uni, chg);
+    } else if (A.pending) {
       stage_pending_warp(A, tile, warp, s0, kSub, dlw, mkw, lane, uni, chg);
+      many = true;
     } else {
       stage_delta_warp(A, tile, warp, s0, kSub, dlw, lane);
     }
+    const uint32_t umask = (A.pending && upos != ~0u) ? mkw[upos] : 0u;
+    const bool patch = __any_sync(0xffffffffu, umask != 0u);
+    // the next tiles' loads, in flight while this tile is processed
+    const float w1 = pipe_w(A, p1);
+    const Pairs p2 = pipe_pairs(A, c2, own, lane);
+    const uint2 c3 = pipe_chunk(A, tile + 3 * stride, warp, lane);
     float4 dl4[kSub / 128];
     uint4 mk4[kSub / 128];
 #pragma unroll
     for (int u = 0; u < kSub / 128; ++u) {
       const int l = u * 128 + lane * 4;
       dl4[u] = *reinterpret_cast<const float4*>(dlw + l);
-      mk4[u] = A.pending ? *reinterpret_cast<const uint4*>(mkw + l) : make_uint4(0u, 0u, 0u, 0u);
+      mk4[u] = many ? *reinterpret_cast<const uint4*>(mkw + l) : make_uint4(0u, 0u, 0u, 0u);
     }
     const int64_t rem = A.d - (int64_t)s0;
     const int lim = rem < kSub ? (int)rem : kSub;
-    const bool full = lim == kSub;
+    // candidate flags of this lane's 16 values (bit 4u + i: value u*128 + lane*4 + i)
+    uint32_t valid = 0;
+#pragma unroll
+    for (int u = 0; u < kSub / 128; ++u)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) valid |= (u * 128 + lane * 4 + i < lim ? 1u : 0u) << (4 * u + i);
+    uint2 bc_lane = make_uint2(0u, 0u);
     for (int k = 0; k < A.K; ++k, ++item) {
       const uint32_t s = item % kStages, r = item / kStages;
       if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
@@ -595,13 +737,20 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         break;
       }
       const int32_t off = sm.gmeta[s];
-      const float* se = sm.e[s] + warp * kSub;
+      float* se = sm.e[s] + warp * kSub;
       const float* sg = sm.g[s] + (off > 0 ? off : 0) + warp * kSub;
+      if (patch) {
+        if ((umask >> k) & 1u) {
+          se[upos] = 0.f;
+          fence_proxy_async();  // before the stage is refilled by the bulk copy
+        }
+        __syncwarp();
+      }
       float v[kSub / 128][4];
 #pragma unroll
       for (int u = 0; u < kSub / 128; ++u) {
         const int l = u * 128 + lane * 4;
-        const float4 e4 = *reinterpret_cast<const float4*>(se + l);
+        float4 e4 = *reinterpret_cast<const float4*>(se + l);
         float4 g4;
         if (off == 0) {
           g4 = *reinterpret_cast<const float4*>(sg + l);
@@ -615,81 +764,146 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
           const float* gk = A.grads + (int64_t)k * A.d;
           g4 = load_g4(gk, (int64_t)s0 + l, A.d, g_mode(gk));
         }
-        if (!full && off >= 0) {  // past d the stage holds bytes of no meaning
+        if (lim < kSub && off >= 0) {  // past d the stage holds bytes of no meaning
           if (l >= lim) g4.x = 0.f;
           if (l + 1 >= lim) g4.y = 0.f;
           if (l + 2 >= lim) g4.z = 0.f;
           if (l + 3 >= lim) g4.w = 0.f;
         }
+        if (many) {
+          const uint4 m4 = mk4[u];
+          if ((m4.x >> k) & 1u) e4.x = 0.f;
+          if ((m4.y >> k) & 1u) e4.y = 0.f;
+          if ((m4.z >> k) & 1u) e4.z = 0.f;
+          if ((m4.w >> k) & 1u) e4.w = 0.f;
+        }
         const float4 d4 = dl4[u];
-        const uint4 m4 = mk4[u];
-        v[u][0] = accumulate(((m4.x >> k) & 1u) ? 0.f : e4.x, g4.x, A.c, d4.x);
-        v[u][1] = accumulate(((m4.y >> k) & 1u) ? 0.f : e4.y, g4.y, A.c, d4.y);
-        v[u][2] = accumulate(((m4.z >> k) & 1u) ? 0.f : e4.z, g4.z, A.c, d4.z);
-        v[u][3] = accumulate(((m4.w >> k) & 1u) ? 0.f : e4.w, g4.w, A.c, d4.w);
+        v[u][0] = accumulate(e4.x, g4.x, A.c, d4.x);
+        v[u][1] = accumulate(e4.y, g4.y, A.c, d4.y);
+        v[u][2] = accumulate(e4.z, g4.z, A.c, d4.z);
+        v[u][3] = accumulate(e4.w, g4.w, A.c, d4.w);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.empty[s]);  // this warp is done reading stage s
-      const uint32_t theta = sm.theta[k];
+      // candidates: |v| >= theta, or NaN (its key is above every threshold);
+      // theta is at most the Inf key, or kNoCandidate for none
+      const uint32_t th = sm.theta[k];
+      const float tf = __uint_as_float(th);
       float* ekt = A.e + (int64_t)k * A.ld + s0;
-      uint32_t bits[kSub / 128];
-      uint32_t nloc = 0;
+      uint32_t bits = 0;
 #pragma unroll
       for (int u = 0; u < kSub / 128; ++u) {
         const int l = u * 128 + lane * 4;
         __stcs(reinterpret_cast<float4*>(ekt + l), make_float4(v[u][0], v[u][1], v[u][2], v[u][3]));
-        bits[u] = cand_bits(v[u], l, lim, theta);
-        nloc += __popc(bits[u]);
-      }
-      const uint32_t cnt = __reduce_add_sync(0xffffffffu, nloc);
-      uint32_t base = region0;
-      if (cnt) {
-        uint32_t used = 0;
-        if (lane == 0) {
-          used = atomicAdd(&sm.rcnt[k], cnt);
-          if (used + cnt > A.cap_region) A.sel[k].dense = 1;  // region full: dense path
-        }
-        base = region0 + __shfl_sync(0xffffffffu, used, 0);
-        uint32_t pos = base;
-        uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
-        float* cv = A.cand_val + (int64_t)k * A.cap;
 #pragma unroll
-        for (int u = 0; u < kSub / 128; ++u)
-          write_group(v[u], s0 + u * 128 + lane * 4, bits[u], lt, pos, region_end, ci, cv, nonfinite);
+        for (int i = 0; i < 4; ++i) bits |= (!(fabsf(v[u][i]) < tf) ? 1u : 0u) << (4 * u + i);
       }
-      if (lane == 0) {
-        const int64_t c = ((int64_t)k * A.n_tiles + tile) * kChunksPerTile + warp;
-        A.chunk_base[c] = base;
-        A.chunk_cnt[c] = cnt;
+      bits &= th == kNoCandidate ? 0u : valid;
+      const uint32_t cnt = __reduce_add_sync(0xffffffffu, __popc(bits));
+      const uint32_t run_k = __shfl_sync(0xffffffffu, run, k);  // worker k's candidates so far
+      if (cnt) {
+        if (lane == 0 && run_k + cnt > A.cap_part) A.sel[k].dense = 1;  // part full: dense path
+        // rank in index order (group u, then lane, then value): the four
+        // groups' counts, one byte each, scanned over the lanes at once
+        uint32_t packed = 0;
+#pragma unroll
+        for (int u = 0; u < kSub / 128; ++u) packed |= (uint32_t)__popc((bits >> (4 * u)) & 0xfu) << (8 * u);
+        uint32_t incl = packed;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const uint32_t tot = __shfl_sync(0xffffffffu, incl, 31);
+        const uint32_t excl = incl - packed;
+        uint32_t gbase[kSub / 128];  // rank of the lane's first candidate in each group
+        uint32_t acc = run_k;
+#pragma unroll
+        for (int u = 0; u < kSub / 128; ++u) {
+          gbase[u] = acc + ((excl >> (8 * u)) & 0xffu);
+          acc += (tot >> (8 * u)) & 0xffu;
+        }
+        uint32_t* ci = A.cand_idx + (int64_t)k * A.cap + part0;
+        float* cv = A.cand_val + (int64_t)k * A.cap + part0;
+        uint32_t* si = stg + k * 64;
+        float* sv = reinterpret_cast<float*>(si + 32);
+        const uint32_t end = run_k + cnt;
+        for (uint32_t line = run_k >> 5; line <= (end - 1) >> 5; ++line) {
+#pragma unroll
+          for (int u = 0; u < kSub / 128; ++u) {
+            uint32_t o = gbase[u];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              if ((bits >> (4 * u + i)) & 1u) {
+                if ((o >> 5) == line && o < A.cap_part) {
+                  si[o & 31] = s0 + u * 128 + lane * 4 + i;
+                  sv[o & 31] = v[u][i];
+                }
+                ++o;
+              }
+            }
+          }
+          __syncwarp();
+          const uint32_t line_end = (line + 1) * 32;
+          if (line_end <= end && line_end <= A.cap_part) {  // a whole line: one coalesced store per array
+            const float x = sv[lane];
+            ci[line * 32 + lane] = si[lane];
+            cv[line * 32 + lane] = x;
+            nonfinite += is_nonfinite(x) ? 1u : 0u;
+          }
+          __syncwarp();
+        }
+        if (lane == k) run += cnt;
       }
+      const uint32_t base = part0 + run_k;
+      if (lane == k) bc_lane = make_uint2(base, cnt);
     }
+    // the tile's sub-chunk entries of this warp: lane k holds worker k's
+    if (ok && lane < A.K) A.chunk[chunk_at(A, lane, tile, warp)] = bc_lane;
+    p0 = p1;
+    w0 = w1;
+    p1 = p2;
+    c2 = c3;
   }
   if (!ok) atomicOr(A.status, kStatusTimeout);
-  if (nonfinite) {
-    atomicOr(A.status, kStatusNonfinite);
-    atomicAdd(&A.step_ctr->v[kNonfinite], (unsigned long long)nonfinite);
-  }
   if (A.pending) {  // the previous step's counts, straight into the totals
     const uint32_t u_w = __reduce_add_sync(0xffffffffu, uni);
     const uint32_t c_w = __reduce_add_sync(0xffffffffu, chg);
     if (lane == 0 && u_w) atomicAdd(&A.total_ctr->v[kUnion], (unsigned long long)u_w);
     if (lane == 0 && c_w) atomicAdd(&A.total_ctr->v[kChanged], (unsigned long long)c_w);
   }
-  // every consumer warp is past its last reservation: publish the region counts
-  asm volatile("bar.sync 1, %0;" ::"r"(kConsumers * 32) : "memory");
-  if (warp == 0) {
-    for (int kk = lane; kk < A.K; kk += 32) {
-      const uint32_t n = sm.rcnt[kk];
-      A.rcount[(int64_t)kk * A.regions + blockIdx.x] = n < A.cap_region ? n : A.cap_region;
-      if (n) atomicAdd(&A.sel[kk].count, n);
+  // the staged tail of each worker's part, and the part's count
+  for (int k = 0; k < A.K; ++k) {
+    const uint32_t run_k = __shfl_sync(0xffffffffu, run, k);
+    const uint32_t line = run_k >> 5;
+    if (run_k <= A.cap_part && (uint32_t)lane < (run_k & 31)) {
+      const uint32_t* si = stg + k * 64;
+      const float x = reinterpret_cast<const float*>(si + 32)[lane];
+      A.cand_idx[(int64_t)k * A.cap + part0 + line * 32 + lane] = si[lane];
+      A.cand_val[(int64_t)k * A.cap + part0 + line * 32 + lane] = x;
+      nonfinite += is_nonfinite(x) ? 1u : 0u;
     }
+  }
+  if (nonfinite) {
+    atomicOr(A.status, kStatusNonfinite);
+    atomicAdd(&A.step_ctr->v[kNonfinite], (unsigned long long)nonfinite);
+  }
+  if (lane < A.K) {
+    A.rcount[(int64_t)lane * A.regions * kConsumers + blockIdx.x * kConsumers + warp] =
+        run < A.cap_part ? run : A.cap_part;
+    if (run) atomicAdd(&A.sel[lane].count, run);
   }
 }
 
 // ---------------------------------------------------------------------------
-// Candidate ranges of a worker: one per region of the bulk pass, or [0, count)
-// split evenly when the candidates share one region. Part p of nparts.
+// Candidate ranges of a worker, visited one warp per part: the parts of the
+// bulk pass (one per CTA and warp), or [0, count) split evenly when the
+// candidates share one region. nparts = candidate_parts(A); a warp of a block
+// visits parts blockIdx.x * kWarps + warp, then every gridDim.x * kWarps.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ int candidate_parts(const TopkArgs& A) {
+  return A.regions > 1 ? A.regions * kChunksPerTile : (int)gridDim.x * kWarps;
+}
 __device__ __forceinline__ void candidate_part(const TopkArgs& A, int k, int p, int nparts,
                                                uint32_t* lo, uint32_t* hi) {
   if (A.regions == 1) {
@@ -698,8 +912,8 @@ __device__ __forceinline__ void candidate_part(const TopkArgs& A, int k, int p, 
     *lo = min(cnt, (uint32_t)p * per);
     *hi = min(cnt, *lo + per);
   } else {
-    *lo = (uint32_t)p * A.cap_region;
-    *hi = *lo + A.rcount[(int64_t)k * A.regions + p];
+    *lo = (uint32_t)p * A.cap_part;
+    *hi = *lo + A.rcount[(int64_t)k * nparts + p];
   }
 }
 
@@ -732,15 +946,16 @@ __global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
   for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) h[b] = 0;
   __syncthreads();
   const float* cv = A.cand_val + (int64_t)k * A.cap;
-  const int nparts = A.regions == 1 ? (int)gridDim.x : A.regions;
-  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+  const int nparts = candidate_parts(A);
+  const int lane = threadIdx.x & 31;
+  for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
     uint32_t lo, hi;
     candidate_part(A, k, part, nparts, &lo, &hi);
-    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * blockDim.x) {
+    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * 32) {
       uint32_t kv[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const uint32_t i = i0 + q * blockDim.x + threadIdx.x;
+        const uint32_t i = i0 + q * 32 + lane;
         kv[q] = i < hi ? mag_key(cv[i]) : 0xffffffffu;
       }
 #pragma unroll
@@ -823,12 +1038,12 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   uint32_t* bk = A.bucket + (int64_t)k * 2 * kBucketCap;  // keys, then indices
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
-  const int nparts = A.regions == 1 ? (int)gridDim.x : A.regions;
-  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+  const int nparts = candidate_parts(A);
+  for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
     uint32_t lo, hi;
     candidate_part(A, k, part, nparts, &lo, &hi);
-    for (uint32_t i0 = lo; i0 < hi; i0 += blockDim.x) {
-      const uint32_t i = i0 + threadIdx.x;
+    for (uint32_t i0 = lo; i0 < hi; i0 += 32) {
+      const uint32_t i = i0 + lane;
       uint32_t key = 0;
       bool in = false;
       if (i < hi) {
@@ -985,11 +1200,9 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
     const uint32_t in_tile = (uint32_t)(tot >> 32) + (min(eqrun + (uint32_t)tot, n_tie) - taken0);
     if (threadIdx.x == 0) sb[kChunksPerTile] = running + in_tile;
     __syncthreads();
-    if (threadIdx.x < kChunksPerTile) {
-      const int64_t c = ((int64_t)k * A.n_tiles + tile) * kChunksPerTile + threadIdx.x;
-      A.chunk_base[c] = sb[threadIdx.x];
-      A.chunk_cnt[c] = sb[threadIdx.x + 1] - sb[threadIdx.x];
-    }
+    if (threadIdx.x < kChunksPerTile)
+      A.chunk[chunk_at(A, k, tile, threadIdx.x)] =
+          make_uint2(sb[threadIdx.x], sb[threadIdx.x + 1] - sb[threadIdx.x]);
     running += in_tile;
     eqrun += (uint32_t)tot;
     __syncthreads();
@@ -1023,8 +1236,8 @@ __device__ __forceinline__ void sent_part(const TopkArgs& A, int k, int p, int n
     *lo = min(n, (uint32_t)p * per);
     *hi = min(n, *lo + per);
   } else {
-    *lo = (uint32_t)p * A.cap_region;
-    *hi = *lo + (p < A.regions ? A.rcount[(int64_t)k * A.regions + p] : 0u);
+    *lo = (uint32_t)p * A.cap_part;
+    *hi = *lo + A.rcount[(int64_t)k * nparts + p];
   }
 }
 
@@ -1034,17 +1247,18 @@ __global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A, int mode) {
   const uint32_t bit = 1u << k;
   uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
-  const int nparts = A.regions > 1 ? A.regions : (int)gridDim.x;
+  const int nparts = candidate_parts(A);
+  const int lane = threadIdx.x & 31;
   unsigned long long nnz = 0;
-  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+  for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
     uint32_t lo, hi;
     sent_part(A, k, part, nparts, &lo, &hi);
-    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * blockDim.x) {
+    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * 32) {
       uint32_t jq[4];
       float vq[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const uint32_t i = i0 + q * blockDim.x + threadIdx.x;
+        const uint32_t i = i0 + q * 32 + lane;
         jq[q] = i < hi ? ci[i] : 0xffffffffu;
         vq[q] = i < hi ? cv[i] : 0.f;
       }
@@ -1060,7 +1274,7 @@ __global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A, int mode) {
           }
           nnz += (vq[q] != 0.f);
         } else {
-          ci[i0 + q * blockDim.x + threadIdx.x] = j | kUnsent;
+          ci[i0 + q * 32 + lane] = j | kUnsent;
         }
       }
     }
@@ -1075,12 +1289,12 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
   const int k = blockIdx.y;
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const uint32_t mine = 1u << k, lower = mine - 1u;
-  const int nparts = A.regions > 1 ? A.regions : (int)gridDim.x;
+  const int nparts = candidate_parts(A);
   unsigned long long uni = 0, changed = 0;
-  for (int part = blockIdx.x; part < nparts; part += gridDim.x) {
+  for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
     uint32_t lo, hi;
     sent_part(A, k, part, nparts, &lo, &hi);
-    for (uint32_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+    for (uint32_t i = lo + (threadIdx.x & 31); i < hi; i += 32) {
       const uint32_t j = __ldcg(ci + i);
       if (j >= (uint32_t)A.d) continue;  // not sent (marked) or out of range
       const uint32_t m = A.mask[j];
@@ -1125,7 +1339,6 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
 __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uint32_t* idx_out,
                                                           float* val_out) {
   __shared__ uint32_t ws[32];
-  const int64_t row = (int64_t)k * A.n_tiles;
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
   uint32_t carry = 0;
@@ -1134,8 +1347,8 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
     uint32_t cnt = 0;
     if (tile < A.n_tiles) {
       for (int w = 0; w < kChunksPerTile; ++w) {
-        const int64_t c = (row + tile) * kChunksPerTile + w;
-        const uint32_t base = A.chunk_base[c], n = A.chunk_cnt[c];
+        const uint2 bc = A.chunk[chunk_at(A, k, tile, w)];
+        const uint32_t base = bc.x, n = bc.y;
         for (uint32_t i = 0; i < n && base + i < A.cap; ++i) cnt += (ci[base + i] & kUnsent) ? 0u : 1u;
       }
     }
@@ -1143,8 +1356,8 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
     uint32_t pos = carry + block_inclusive_scan<uint32_t>(cnt, ws, &tot) - cnt;
     if (cnt) {
       for (int w = 0; w < kChunksPerTile; ++w) {
-        const int64_t c = (row + tile) * kChunksPerTile + w;
-        const uint32_t base = A.chunk_base[c], n = A.chunk_cnt[c];
+        const uint2 bc = A.chunk[chunk_at(A, k, tile, w)];
+        const uint32_t base = bc.x, n = bc.y;
         for (uint32_t i = 0; i < n && base + i < A.cap; ++i) {
           const uint32_t j = ci[base + i];
           if (j & kUnsent) continue;
@@ -1166,8 +1379,8 @@ bool use_bulk(int tile) { return tile == bulk::kT; }
 
 }  // namespace
 
-int accumulate_smem_bytes(int tile) {
-  return use_bulk(tile) ? (int)sizeof(bulk::Smem) : tile * 12;
+int accumulate_smem_bytes(int tile, int K) {
+  return use_bulk(tile) ? bulk::smem_bytes(K) : tile * 12;
 }
 
 cudaError_t configure_topk_kernels() {
@@ -1180,7 +1393,7 @@ cudaError_t configure_topk_kernels() {
   set((const void*)k_accumulate<2>, 2048 * 12);
   set((const void*)k_accumulate<4>, 4096 * 12);
   set((const void*)k_accumulate<8>, 8192 * 12);
-  set((const void*)k_accumulate_bulk, (int)sizeof(bulk::Smem));
+  set((const void*)k_accumulate_bulk, bulk::smem_bytes(kMaxK));
   set((const void*)k_select_finish, 2 * kBucketCap * 4);
   return err;
 }
@@ -1188,7 +1401,7 @@ cudaError_t configure_topk_kernels() {
 int accumulate_blocks_per_sm(int tile) {
   if (use_bulk(tile)) return 1;  // one persistent CTA per SM
   int n = 0;
-  const int smem = accumulate_smem_bytes(tile);
+  const int smem = accumulate_smem_bytes(tile, kMaxK);
   switch (tile_u(tile)) {
     case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<1>, kThreads, smem); break;
     case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<2>, kThreads, smem); break;
@@ -1204,7 +1417,7 @@ cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
 }
 
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
-  const int smem = accumulate_smem_bytes(A.tile);
+  const int smem = accumulate_smem_bytes(A.tile, A.K);
   if (use_bulk(A.tile)) {
     k_accumulate_bulk<<<grid, bulk::kThreadsAll, smem, s>>>(A);
     return cudaGetLastError();
