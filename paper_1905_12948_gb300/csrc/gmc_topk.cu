@@ -473,14 +473,16 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 // ---------------------------------------------------------------------------
 // bulk-copy version (tiles of 4096). One persistent CTA per SM. A producer
 // thread streams each (tile, worker) item's e and g into a ring of shared-
-// memory stages with cp.async.bulk; eight consumer warps, each owning 512
-// elements of every tile, read their part, release the stage, store v over e
-// and append their candidates to their own part of this CTA's region of the
-// candidate buffer (one part per warp and worker). Candidates are staged in
-// shared memory and leave in whole 128-byte lines. Producer and consumers
-// meet only at mbarriers and every wait is bounded.
+// memory stages with cp.async.bulk; sixteen consumer warps, two per 512-
+// element sub-tile of every tile (one for the workers of even index, one for
+// the odd), read their part, release the stage, store v over e and append
+// their candidates to their sub-tile's part of this CTA's region of the
+// candidate buffer (one part per sub-tile and worker). Candidates are staged
+// in shared memory and leave in whole 128-byte lines. Producer and consumers
+// meet only at mbarriers (every wait bounded); the two warps of a sub-tile
+// meet at a named barrier twice per tile.
 //
-// Each consumer warp forms its sub-tile's w_t - w_{t-1} (and applies the
+// The even warp of a sub-tile forms its w_t - w_{t-1} (and applies the
 // previous step's aggregation when it was left pending) from the previous
 // step's sent pairs. Those are reached through two dependent loads -- the
 // sub-chunk table, then the pairs -- and the pending case reads w at the
@@ -496,16 +498,20 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 namespace bulk {
 constexpr int kT = kBulkTile;
 constexpr int kStages = GMC_BULK_STAGES;   // shared-memory ring of (e, g) tiles
-constexpr int kConsumers = kChunksPerTile;
-constexpr int kSub = kT / kConsumers;      // 512
+constexpr int kSubTiles = kChunksPerTile;  // 8 sub-tiles of 512 elements
+constexpr int kSub = kT / kSubTiles;       // 512
+constexpr int kConsumers = 2 * kSubTiles;  // warps 0..15: sub-tile w & 7, workers of parity w >> 3
 constexpr int kGLen = kT + 8;              // g stage: up to 3 leading floats of misalignment
+constexpr int kProducer = kConsumers;      // warp 16
 constexpr int kThreadsAll = (kConsumers + 1) * 32;
 struct Smem {
   float e[kStages][kT];
   float g[kStages][kGLen];
-  float dl[kConsumers][kSub];              // w_t - w_{t-1} of the warp's sub-tile
-  uint32_t mk[kConsumers][kSub];           // senders of the pending aggregation (bit k)
-  uint8_t own[kConsumers][32];             // scratch: worker of each listed pair
+  float dl[kSubTiles][kSub];               // w_t - w_{t-1} of a sub-tile
+  uint32_t mk[kSubTiles][kSub];            // senders of the pending aggregation (bit k)
+  uint8_t own[kSubTiles][32];              // scratch: worker of each listed pair
+  uint32_t upos[kSubTiles][32];            // union coordinates of a sub-tile, one per lane
+  uint32_t pflag[kSubTiles][2];            // per sub-tile: the two warps' status, many-senders flag
   uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
   uint64_t empty[kStages];                 // all consumer warps read the stage (8 arrivals)
   int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
@@ -515,7 +521,7 @@ struct Smem {
 };
 // Dynamic shared memory of the bulk pass for K workers.
 __host__ __device__ constexpr int smem_bytes(int K) {
-  return (int)((sizeof(Smem) + 127) / 128 * 128) + kConsumers * K * 64 * 4;
+  return (int)((sizeof(Smem) + 127) / 128 * 128) + kSubTiles * K * 64 * 4;
 }
 static_assert(smem_bytes(kMaxK) <= 232448, "bulk pass shared memory above the 227 KB a block may use");
 
@@ -627,7 +633,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], kConsumers);
+      mbar_init(&sm.empty[s], kSubTiles);  // the eight warps of the item's worker parity
     }
     fence_mbar_init();
   }
@@ -635,7 +641,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     sm.theta[kk] = kk < A.K ? A.sel[kk].theta : kNoCandidate;
   __syncthreads();
 
-  if (warp == kConsumers) {
+  if (warp == kProducer) {
     // ---- producer ----
     if (lane != 0) return;
     const char* g_lo = reinterpret_cast<const char*>(A.grads);
@@ -674,52 +680,73 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
 
   // ---- consumers ----
   const uint32_t lt = lanemask_lt();
-  float* dlw = sm.dl[warp];
-  uint32_t* mkw = sm.mk[warp];
-  uint8_t* own = sm.own[warp];
-  // this warp's part of the CTA's region, per worker: slots [part0, part0 + cap_part);
+  const int sw = warp & (kSubTiles - 1);  // sub-tile
+  const int gp = warp / kSubTiles;         // workers k = gp, gp + 2, ...
+  const bool lead = gp == 0;               // forms the sub-tile's w_t - w_{t-1}
+  float* dlw = sm.dl[sw];
+  uint32_t* mkw = sm.mk[sw];
+  uint8_t* own = sm.own[sw];
+  // the sub-tile's part of the CTA's region, per worker: slots [part0, part0 + cap_part);
   // lane k counts worker k's candidates so far
-  const uint32_t part0 = (blockIdx.x * kConsumers + warp) * A.cap_part;
+  const uint32_t part0 = (blockIdx.x * kSubTiles + sw) * A.cap_part;
   uint32_t* stg = reinterpret_cast<uint32_t*>(smem_raw + (sizeof(Smem) + 127) / 128 * 128) +
-                  warp * A.K * 64;
+                  sw * A.K * 64;
   uint32_t run = 0;
   const int64_t stride = gridDim.x;
   uint32_t nonfinite = 0, uni = 0, chg = 0;
-  uint32_t item = 0;
   bool ok = true;
   // fill the pipeline: pairs of tiles 0 and 1, w of tile 0, entries of tile 2
-  Pairs p0 = pipe_pairs(A, pipe_chunk(A, blockIdx.x, warp, lane), own, lane);
-  Pairs p1 = pipe_pairs(A, pipe_chunk(A, blockIdx.x + stride, warp, lane), own, lane);
-  float w0 = pipe_w(A, p0);
-  uint2 c2 = pipe_chunk(A, blockIdx.x + 2 * stride, warp, lane);
-  for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += stride) {
-    const uint32_t s0 = (uint32_t)(tile * kT) + warp * kSub;
+  Pairs p0{kUnsent, 0.f, 0, 0u}, p1{kUnsent, 0.f, 0, 0u};
+  float w0 = 0.f;
+  uint2 c2 = make_uint2(0u, 0u);
+  if (lead) {
+    p0 = pipe_pairs(A, pipe_chunk(A, blockIdx.x, sw, lane), own, lane);
+    p1 = pipe_pairs(A, pipe_chunk(A, blockIdx.x + stride, sw, lane), own, lane);
+    w0 = pipe_w(A, p0);
+    c2 = pipe_chunk(A, blockIdx.x + 2 * stride, sw, lane);
+  }
+  const uint32_t pair_bar = 1 + sw;  // named barrier of the sub-tile's two warps
+  uint32_t n = 0;                    // tiles done
+  for (int64_t tile = blockIdx.x; tile < A.n_tiles; tile += stride, ++n) {
+    const uint32_t s0 = (uint32_t)(tile * kT) + sw * kSub;
     // this sub-tile's w_t - w_{t-1}, and the pending senders (their residual
     // is +0): at most 32 union coordinates, one per lane (upos, umask), are
     // zeroed in each worker's stage before it is read; more use per-element masks
-    uint32_t upos = ~0u;
-    bool many = false;
-    if (p0.total <= 32u) {
-      upos = apply_pairs(A, s0, p0, w0, dlw, mkw, lane, lt, uni, chg);
-    } else if (A.pending) {
-      stage_pending_warp(A, tile, warp, s0, kSub, dlw, mkw, lane, uni, chg);
-      many = true;
-    } else {
-      stage_delta_warp(A, tile, warp, s0, kSub, dlw, lane);
+    if (lead) {
+      uint32_t up = ~0u;
+      bool many = false;
+      if (p0.total <= 32u) {
+        up = apply_pairs(A, s0, p0, w0, dlw, mkw, lane, lt, uni, chg);
+      } else if (A.pending) {
+        stage_pending_warp(A, tile, sw, s0, kSub, dlw, mkw, lane, uni, chg);
+        many = true;
+      } else {
+        stage_delta_warp(A, tile, sw, s0, kSub, dlw, lane);
+      }
+      sm.upos[sw][lane] = up;
+      if (lane == 0) sm.pflag[sw][1] = many ? 1u : 0u;
     }
+    if (lane == 0) sm.pflag[sw][0] = 0;  // both warps: report a timeout below
+    asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+    if (lane == 0 && !ok) atomicOr(&sm.pflag[sw][0], 1u);
+    asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+    if (sm.pflag[sw][0]) break;  // one of the two warps gave up: both leave together
+    const bool many = sm.pflag[sw][1] != 0u;
+    const uint32_t upos = sm.upos[sw][lane];
     const uint32_t umask = (A.pending && upos != ~0u) ? mkw[upos] : 0u;
     const bool patch = __any_sync(0xffffffffu, umask != 0u);
-    // the next tiles' loads, in flight while this tile is processed
-    const float w1 = pipe_w(A, p1);
-    const Pairs p2 = pipe_pairs(A, c2, own, lane);
-    const uint2 c3 = pipe_chunk(A, tile + 3 * stride, warp, lane);
     float4 dl4[kSub / 128];
-    uint4 mk4[kSub / 128];
 #pragma unroll
-    for (int u = 0; u < kSub / 128; ++u) {
-      const int l = u * 128 + lane * 4;
-      dl4[u] = *reinterpret_cast<const float4*>(dlw + l);
-      mk4[u] = many ? *reinterpret_cast<const uint4*>(mkw + l) : make_uint4(0u, 0u, 0u, 0u);
+    for (int u = 0; u < kSub / 128; ++u) dl4[u] = *reinterpret_cast<const float4*>(dlw + u * 128 + lane * 4);
+    // the lead warp rewrites the sub-tile's buffers for the next tile only after this
+    asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+    float w1 = 0.f;
+    Pairs p2{kUnsent, 0.f, 0, 0u};
+    uint2 c3 = make_uint2(0u, 0u);
+    if (lead) {  // the next tiles' loads, in flight while this tile is processed
+      w1 = pipe_w(A, p1);
+      p2 = pipe_pairs(A, c2, own, lane);
+      c3 = pipe_chunk(A, tile + 3 * stride, sw, lane);
     }
     const int64_t rem = A.d - (int64_t)s0;
     const int lim = rem < kSub ? (int)rem : kSub;
@@ -730,15 +757,16 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
 #pragma unroll
       for (int i = 0; i < 4; ++i) valid |= (u * 128 + lane * 4 + i < lim ? 1u : 0u) << (4 * u + i);
     uint2 bc_lane = make_uint2(0u, 0u);
-    for (int k = 0; k < A.K; ++k, ++item) {
+    for (int k = gp; k < A.K; k += 2) {
+      const uint32_t item = n * (uint32_t)A.K + (uint32_t)k;
       const uint32_t s = item % kStages, r = item / kStages;
       if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
         ok = false;
         break;
       }
       const int32_t off = sm.gmeta[s];
-      float* se = sm.e[s] + warp * kSub;
-      const float* sg = sm.g[s] + (off > 0 ? off : 0) + warp * kSub;
+      float* se = sm.e[s] + sw * kSub;
+      const float* sg = sm.g[s] + (off > 0 ? off : 0) + sw * kSub;
       if (patch) {
         if ((umask >> k) & 1u) {
           se[upos] = 0.f;
@@ -770,8 +798,8 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
           if (l + 2 >= lim) g4.z = 0.f;
           if (l + 3 >= lim) g4.w = 0.f;
         }
-        if (many) {
-          const uint4 m4 = mk4[u];
+        if (many) {  // more union coordinates than lanes: per-element sender masks
+          const uint4 m4 = *reinterpret_cast<const uint4*>(mkw + l);
           if ((m4.x >> k) & 1u) e4.x = 0.f;
           if ((m4.y >> k) & 1u) e4.y = 0.f;
           if ((m4.z >> k) & 1u) e4.z = 0.f;
@@ -855,15 +883,18 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         }
         if (lane == k) run += cnt;
       }
-      const uint32_t base = part0 + run_k;
-      if (lane == k) bc_lane = make_uint2(base, cnt);
+      if (lane == k) bc_lane = make_uint2(part0 + run_k, cnt);
     }
-    // the tile's sub-chunk entries of this warp: lane k holds worker k's
-    if (ok && lane < A.K) A.chunk[chunk_at(A, lane, tile, warp)] = bc_lane;
-    p0 = p1;
-    w0 = w1;
-    p1 = p2;
-    c2 = c3;
+    // the tile's sub-chunk entries of this warp's workers: lane k holds worker k's
+    if (ok && lane < A.K && (lane & 1) == gp) A.chunk[chunk_at(A, lane, tile, sw)] = bc_lane;
+    if (lead) {
+      p0 = p1;
+      w0 = w1;
+      p1 = p2;
+      c2 = c3;
+    }
+    // the per-element masks of a many-sender sub-tile stay in use until both warps are done
+    if (many) asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
   }
   if (!ok) atomicOr(A.status, kStatusTimeout);
   if (A.pending) {  // the previous step's counts, straight into the totals
@@ -873,7 +904,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     if (lane == 0 && c_w) atomicAdd(&A.total_ctr->v[kChanged], (unsigned long long)c_w);
   }
   // the staged tail of each worker's part, and the part's count
-  for (int k = 0; k < A.K; ++k) {
+  for (int k = gp; k < A.K; k += 2) {
     const uint32_t run_k = __shfl_sync(0xffffffffu, run, k);
     const uint32_t line = run_k >> 5;
     if (run_k <= A.cap_part && (uint32_t)lane < (run_k & 31)) {
@@ -888,8 +919,8 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     atomicOr(A.status, kStatusNonfinite);
     atomicAdd(&A.step_ctr->v[kNonfinite], (unsigned long long)nonfinite);
   }
-  if (lane < A.K) {
-    A.rcount[(int64_t)lane * A.regions * kConsumers + blockIdx.x * kConsumers + warp] =
+  if (lane < A.K && (lane & 1) == gp) {
+    A.rcount[(int64_t)lane * A.regions * kSubTiles + blockIdx.x * kSubTiles + sw] =
         run < A.cap_part ? run : A.cap_part;
     if (run) atomicAdd(&A.sel[lane].count, run);
   }
