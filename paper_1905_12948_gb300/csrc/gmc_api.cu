@@ -434,7 +434,9 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
 
   const int64_t streams_wide = 2 * (int64_t)h->num_sms;
   if (compressor == GMC_TOPK) {
-    int U = 4;
+    // tiles of 4096 take the bulk-copy pass, for up to kBulkMaxK workers (its
+    // shared memory grows with K); otherwise the load/store pass
+    int U = K <= kBulkMaxK ? 4 : 2;
     if (d < 4096 * streams_wide) U = 2;
     if (d < 2048 * streams_wide) U = 1;
     h->tile = 1024 * U;

@@ -118,6 +118,7 @@ cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s);
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s);
 constexpr int kBulkTile = 4096;  // tile of the bulk-copy accumulate pass (k_accumulate_bulk)
+constexpr int kBulkMaxK = 16;    // workers the bulk-copy pass takes (its shared memory grows with K)
 
 // k_mark over worker k's sent pairs; mode is a bit set of kMark*.
 constexpr int kMarkSent = 1;    // mark the candidates not sent, count the non-zero sent values

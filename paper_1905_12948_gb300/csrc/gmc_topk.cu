@@ -492,12 +492,9 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 // no latency lies on its path. A sub-tile with more than 32 pairs takes the
 // direct path (stage_pending_warp / stage_delta_warp).
 // ---------------------------------------------------------------------------
-#ifndef GMC_BULK_STAGES
-#define GMC_BULK_STAGES 4
-#endif
 namespace bulk {
 constexpr int kT = kBulkTile;
-constexpr int kStages = GMC_BULK_STAGES;   // shared-memory ring of (e, g) tiles
+constexpr int kStages = 4;                 // shared-memory ring of (e, g) tiles
 constexpr int kSubTiles = kChunksPerTile;  // 8 sub-tiles of 512 elements
 constexpr int kSub = kT / kSubTiles;       // 512
 constexpr int kConsumers = 2 * kSubTiles;  // warps 0..15: sub-tile w & 7, workers of parity w >> 3
@@ -523,7 +520,7 @@ struct Smem {
 __host__ __device__ constexpr int smem_bytes(int K) {
   return (int)((sizeof(Smem) + 127) / 128 * 128) + kSubTiles * K * 64 * 4;
 }
-static_assert(smem_bytes(kMaxK) <= 232448, "bulk pass shared memory above the 227 KB a block may use");
+static_assert(smem_bytes(kBulkMaxK) <= 232448, "bulk pass shared memory above the 227 KB a block may use");
 
 // The first (up to 32) sent pairs of one sub-tile of the previous step, lane e
 // holding pair e of the list that runs through the workers in ascending order.
@@ -1424,7 +1421,7 @@ cudaError_t configure_topk_kernels() {
   set((const void*)k_accumulate<2>, 2048 * 12);
   set((const void*)k_accumulate<4>, 4096 * 12);
   set((const void*)k_accumulate<8>, 8192 * 12);
-  set((const void*)k_accumulate_bulk, bulk::smem_bytes(kMaxK));
+  set((const void*)k_accumulate_bulk, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_select_finish, 2 * kBucketCap * 4);
   return err;
 }

@@ -74,6 +74,19 @@ def test_topk_bulk_copy_path(offset):
     assert p.gpu.check() == 0
 
 
+def test_topk_many_workers_take_load_store_pass():
+    """More workers than the bulk pass takes (17..32): the load/store pass at
+    a size that would otherwise be bulk, with the aggregate applied each step."""
+    d, K = 1_300_001, 20
+    rng = np.random.default_rng(17)
+    p = Pair(d, K, 0.9, 0.05, ratio=0.001, seed=7)
+    for t in range(2):
+        g = (rng.standard_normal((K, d)) * np.exp(rng.uniform(-3, 0, size=d))).astype(np.float32)
+        p.compare(p.step(g), residuals=(t == 1))
+    p.compare_stats()
+    assert p.gpu.check() == 0
+
+
 def test_topk_dense_tiles_unstaged_aggregate():
     """Every coordinate sent by 5 workers: more entries per tile than the
     aggregate stages in shared memory."""
