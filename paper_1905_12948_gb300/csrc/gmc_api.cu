@@ -66,7 +66,7 @@ struct gmc_ctx {
   float* cand_val[2] = {nullptr, nullptr};
   uint2* chunk[2] = {nullptr, nullptr};
   uint32_t* mask = nullptr;
-  uint32_t* smask[2] = {nullptr, nullptr};  // senders at the sampled positions, by step parity
+  uint32_t* sample_pend = nullptr;  // 2 x kSampleSlots
   // deferred aggregation (bulk top-k pass): the last step's sent pairs are
   // summed into w by the next step's bulk pass, or by flush() when state is read
   bool agg_pending = false;
@@ -228,8 +228,7 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.mask = h->mask;
   A.cand_idx_prev = h->cand_idx[prev];
   A.cand_val_prev = h->cand_val[prev];
-  A.smask_rd = h->smask[prev];
-  A.smask_wr = h->smask[cur];
+  A.sample_pend = h->sample_pend;
   A.total_ctr = h->total_ctr;
   A.pending = 0;
   A.a_prev = A.a;
@@ -302,6 +301,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager) {
     TopkArgs A = topk_args(h, grads);
     A.pending = h->agg_pending ? 1 : 0;
     A.a_prev = h->a_pending;
+    const bool defer = h->tile == kBulkTile && !eager && !h->detach_out;
     const double kk = (double)h->K * (double)h->ksel;
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
@@ -309,10 +309,8 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager) {
     h->agg_pending = false;
     GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] { return launch_select(A, h->sel_blocks, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_DENSE, 0.0, s, [&] { return launch_select_dense(A, s); }));
-    const bool defer = h->tile == kBulkTile && !eager && !h->detach_out;
     if (defer) {
-      GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 8.0 * kk, s,
-                    [&] { return launch_mark(A, kMarkSent | kMarkSample, h->grid_agg, s); }));
+      // the next step's sample and bulk pass apply the aggregation
       h->agg_pending = true;
       h->a_pending = A.a;
     } else {
@@ -320,7 +318,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager) {
       B.a_prev = A.a;
       B.total_ctr = nullptr;  // k_finalize adds the step's counts to the totals
       GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk, s, [&] {
-        cudaError_t err = launch_mark(B, kMarkSent | kMarkMask, h->grid_agg, s);
+        cudaError_t err = launch_mark(B, h->grid_agg, s);
         return err != cudaSuccess ? err : launch_owner_sum(B, h->grid_agg, s);
       }));
     }
@@ -344,8 +342,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager) {
 }
 
 // Apply a pending aggregation on stream s (ordered after the last step):
-// the senders of every coordinate into mask, then k_owner_sum; the sampled
-// senders are cleared, since the next sample must not apply them again.
+// the senders of every coordinate into mask, then k_owner_sum.
 int flush(gmc_ctx* h, cudaStream_t s) {
   if (!h->agg_pending) return GMC_OK;
   GMC_TRY(cudaStreamWaitEvent(s, h->ev_step, 0));
@@ -353,9 +350,8 @@ int flush(gmc_ctx* h, cudaStream_t s) {
   A.a_prev = h->a_pending;
   A.step_ctr = h->step_ctr;    // the counts belong to the last step
   A.total_ctr = h->total_ctr;  // which k_finalize has already added up
-  GMC_TRY(launch_mark(A, kMarkMask, h->grid_agg, s));
+  GMC_TRY(launch_mark(A, h->grid_agg, s));
   GMC_TRY(launch_owner_sum(A, h->grid_agg, s));
-  GMC_TRY(cudaMemsetAsync(A.smask_wr, 0, (size_t)kSampleSlots * sizeof(uint32_t), s));
   GMC_TRY(cudaEventRecord(h->ev_flush, s));
   h->wait_flush = true;
   h->agg_pending = false;
@@ -501,8 +497,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->big_tiles, (size_t)h->n_tiles + 1)) != cudaSuccess ||
         (err = dalloc(h, &h->rcount, (size_t)K * h->regions * kChunksPerTile)) != cudaSuccess ||
         (err = dalloc(h, &h->mask, (size_t)h->ld)) != cudaSuccess ||
-        (err = dalloc(h, &h->smask[0], (size_t)kSampleSlots)) != cudaSuccess ||
-        (err = dalloc(h, &h->smask[1], (size_t)kSampleSlots)) != cudaSuccess)
+        (err = dalloc(h, &h->sample_pend, (size_t)2 * kSampleSlots)) != cudaSuccess)
       return fail(err);
     if ((err = cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking)) != cudaSuccess ||
         (err = cudaEventCreateWithFlags(&h->ev_step, cudaEventDisableTiming)) != cudaSuccess ||
@@ -608,8 +603,6 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
       GMC_TRY(cudaMemsetAsync(h->chunk[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint2), s));
     GMC_TRY(cudaMemsetAsync(h->sel, 0, (size_t)h->K * sizeof(WorkerSel), s));
     GMC_TRY(cudaMemsetAsync(h->mask, 0, (size_t)h->ld * sizeof(uint32_t), s));
-    for (int p = 0; p < 2; ++p)
-      GMC_TRY(cudaMemsetAsync(h->smask[p], 0, (size_t)kSampleSlots * sizeof(uint32_t), s));
   } else {
     for (int p = 0; p < 2; ++p) GMC_TRY(cudaMemsetAsync(h->uflag[p], 0, (size_t)h->nb, s));
   }

@@ -48,7 +48,7 @@ constexpr unsigned kStatusNonfinite = 1u;
 constexpr unsigned kStatusInternal = 2u;
 constexpr unsigned kStatusTimeout = 4u;     // a bounded wait gave up (see wait_bounded)
 constexpr int kChunksPerTile = 8;           // candidate sub-chunks per tile: one per warp
-constexpr uint32_t kUnsent = 0x80000000u;   // index mark of a candidate that was not sent
+constexpr uint32_t kNone = 0xffffffffu;     // no coordinate
 
 __device__ __forceinline__ uint32_t mag_key(float v) {
   return __float_as_uint(v) & kKeyMask;

@@ -16,7 +16,9 @@ namespace gmc {
 // sub-chunk (k, tile, w) holds worker k's candidates of the w-th of the
 // kChunksPerTile equal parts of the tile, in ascending index order, at
 // cand_idx/cand_val[k*cap + base .. + cnt). The accumulate pass writes every
-// candidate; the aggregate marks the ones not sent (index | kUnsent).
+// candidate; the select fixes the k-th key T and the last tie kept t_idx, and
+// a candidate is sent iff selected(key, index, T, t_idx): the exact top-k, for
+// candidates and for every other coordinate alike.
 // Buffers alternate between steps:
 // the previous step's sent pairs give the non-zero positions of w_t - w_{t-1}.
 struct TopkArgs {
@@ -59,8 +61,8 @@ struct TopkArgs {
   // streams every coordinate anyway (see k_accumulate_bulk).
   int pending;               // the previous step's aggregation is still to be applied
   float a_prev;              // fl(eta/K) of that step
-  const uint32_t* smask_rd;  // kSampleSlots: senders (bit k) of the previous step at each sampled position
-  uint32_t* smask_wr;        // the same for this step (cleared by the sample kernel)
+  uint32_t* sample_pend;     // 2 x kSampleSlots: its senders' mask and w_{t+1} - w_t at the
+                             // sampled coordinates (k_sample_pending, for k_sample)
   Counters* total_ctr;       // running totals: the deferred aggregation counts there
   Counters* step_ctr;
   unsigned* status;
@@ -120,11 +122,8 @@ cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s);
 constexpr int kBulkTile = 4096;  // tile of the bulk-copy accumulate pass (k_accumulate_bulk)
 constexpr int kBulkMaxK = 16;    // workers the bulk-copy pass takes (its shared memory grows with K)
 
-// k_mark over worker k's sent pairs; mode is a bit set of kMark*.
-constexpr int kMarkSent = 1;    // mark the candidates not sent, count the non-zero sent values
-constexpr int kMarkMask = 2;    // record the senders of every coordinate in mask (for k_owner_sum)
-constexpr int kMarkSample = 4;  // record the senders at the sampled positions only (smask_wr)
-cudaError_t launch_mark(const TopkArgs& A, int mode, int grid, cudaStream_t s);
+// k_mark: the senders of every coordinate into mask (for k_owner_sum).
+cudaError_t launch_mark(const TopkArgs& A, int grid, cudaStream_t s);
 // Sum of the sent pairs into w (with a_prev), residuals to +0 where sent,
 // w_{t+1} - w_t into dlt, mask cleared; counts into step_ctr and total_ctr
 // (either may be null).

@@ -67,26 +67,51 @@ __device__ __forceinline__ uint32_t warp_excl_scan(uint32_t x, uint32_t* total) 
   return incl - x;
 }
 
-// w_{t+1}[j] - w_t[j] at a coordinate whose aggregation is still pending: the
-// senders' values are still in e (they were this step's accumulators), w
-// still holds w_t. Sum in ascending worker order from +0 (Alg. 1).
-__device__ __noinline__ float pending_delta(const TopkArgs& A, uint32_t senders, int64_t j) {
-  float sum = 0.f;
-  for (uint32_t m = senders; m; m &= m - 1u)
-    sum = __fadd_rn(sum, __ldcg(A.e + (int64_t)(__ffs(m) - 1) * A.ld + j));
-  const float wo = A.w[j];
-  return __fsub_rn(__fsub_rn(wo, __fmul_rn(A.a_prev, sum)), wo);
+// Sampled coordinate of slot i: the sample takes 8 consecutive coordinates
+// from (c * d / chunks) rounded down to a multiple of 8, c = 0 .. chunks-1
+// (every coordinate when chunks = 0).
+__device__ __forceinline__ int64_t sample_coord(const TopkArgs& A, int i) {
+  if (!A.sample_chunks) return i;
+  const int64_t ch = i >> 3;
+  return ((ch * A.d / A.sample_chunks) & ~int64_t(7)) + (i & 7);
 }
 
-// Slot of coordinate j among the sampled positions, or -1: the sample takes
-// 8 consecutive coordinates from (c * d / chunks) rounded down to a multiple
-// of 8, for c = 0 .. chunks-1 (every coordinate when chunks = 0).
-__device__ __forceinline__ int sample_slot(const TopkArgs& A, uint32_t j) {
-  if (!A.sample_chunks) return j < (uint32_t)kSampleSlots ? (int)j : -1;
-  const int64_t q = (int64_t)(j & ~7u), C = A.sample_chunks;
-  const int64_t c = (q * C + A.d - 1) / A.d;  // first chunk starting at or after q
-  if (c >= C || (((c * A.d) / C) & ~int64_t(7)) != q) return -1;
-  return (int)(c * 8 + (j & 7u));
+// The previous step's aggregation at the sampled coordinates, when it is
+// still pending, once for all workers: the senders of coordinate j are the
+// workers whose value there (still in e: it was their accumulator) was
+// selected; w still holds w_t. For slot i: the senders' mask, and
+// w_{t+1}[j] - w_t[j] -- their values summed in ascending worker order from
+// +0 (Alg. 1).
+__global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
+  __shared__ uint32_t Tp[kMaxK], tip[kMaxK];
+  for (int kk = threadIdx.x; kk < A.K; kk += blockDim.x) {  // the previous step's selections
+    Tp[kk] = A.sel[kk].T;
+    tip[kk] = A.sel[kk].t_idx;
+  }
+  __syncthreads();
+  const int n_s = A.sample_chunks ? A.sample_chunks * 8 : (int)A.d;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n_s) return;
+  const int64_t j = sample_coord(A, i);
+  float x[kMaxK];
+#pragma unroll
+  for (int b = 0; b < kMaxK; ++b) x[b] = b < A.K ? __ldcg(A.e + (int64_t)b * A.ld + j) : 0.f;
+  float sum = 0.f;
+  uint32_t m = 0;
+#pragma unroll
+  for (int b = 0; b < kMaxK; ++b) {
+    if (b < A.K && selected(mag_key(x[b]), (uint32_t)j, Tp[b], tip[b])) {
+      sum = __fadd_rn(sum, x[b]);
+      m |= 1u << b;
+    }
+  }
+  float dd = 0.f;
+  if (m) {
+    const float wo = A.w[j];
+    dd = __fsub_rn(__fsub_rn(wo, __fmul_rn(A.a_prev, sum)), wo);
+  }
+  A.sample_pend[i] = m;
+  A.sample_pend[kSampleSlots + i] = __float_as_uint(dd);
 }
 
 // ---------------------------------------------------------------------------
@@ -102,10 +127,6 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
   if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) A.big_tiles[0] = 0;
-  if (k == 0) {  // this step's sampled-position senders start empty
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < kSampleSlots; i += gridDim.x * blockDim.x)
-      A.smask_wr[i] = 0u;
-  }
   if (A.dense_mode) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       S.theta = kNoCandidate;
@@ -130,18 +151,14 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
       const int i = i0 + q * blockDim.x + threadIdx.x;
       ev[q] = gv[q] = dv[q] = 0.f;
       if (i < i_hi) {
-        int64_t j = i;
-        if (A.sample_chunks) {
-          const int64_t ch = i >> 3;
-          j = ((ch * A.d / A.sample_chunks) & ~int64_t(7)) + (i & 7);
-        }
+        const int64_t j = sample_coord(A, i);
         ev[q] = ek[j];
         gv[q] = gk[j];
         dv[q] = A.dlt[j];
-        const uint32_t m = A.smask_rd[i];
-        if (m) {  // the previous step's aggregation is still pending at j
+        if (A.pending) {  // as if the previous step's aggregation were applied at j
+          const uint32_t m = A.sample_pend[i];
           if ((m >> k) & 1u) ev[q] = 0.f;
-          dv[q] = pending_delta(A, m, j);
+          if (m) dv[q] = __uint_as_float(A.sample_pend[kSampleSlots + i]);
         }
       }
     }
@@ -251,8 +268,10 @@ __device__ __forceinline__ void stage_delta_warp(const TopkArgs& A, int64_t tile
         if (e < total) {
           const uint32_t at = b + (e - p);
           if (at < A.cap) {
-            const uint32_t j = A.cand_idx_prev[(int64_t)(k0 + src) * A.cap + at];
-            if (!(j & kUnsent)) {
+            const int64_t q = (int64_t)(k0 + src) * A.cap + at;
+            const uint32_t j = A.cand_idx_prev[q];
+            const WorkerSel& Sp = A.sel[k0 + src];  // the previous step's selection
+            if (selected(mag_key(A.cand_val_prev[q]), j, Sp.T, Sp.t_idx)) {
               const int64_t l = (int64_t)j - sub0;
               if (l >= 0 && l < n) dlw[l] = A.dlt[j];
               else atomicOr(A.status, kStatusInternal);
@@ -316,12 +335,14 @@ __device__ __forceinline__ void stage_pending_warp(const TopkArgs& A, int64_t ti
         if (at < A.cap) {
           const int64_t q = (int64_t)(k0 + src) * A.cap + at;
           const uint32_t j = A.cand_idx_prev[q];
-          if (!(j & kUnsent)) {
+          const float vq = A.cand_val_prev[q];
+          const WorkerSel& Sp = A.sel[k0 + src];  // the previous step's selection
+          if (selected(mag_key(vq), j, Sp.T, Sp.t_idx)) {
             const int64_t ll = (int64_t)j - sub0;
             if (ll >= 0 && ll < n) {
               act = true;
               l = (uint32_t)ll;
-              v = A.cand_val_prev[q];
+              v = vq;
               atomicOr(&mkw[l], 1u << (k0 + src));
             } else {
               atomicOr(A.status, kStatusInternal);
@@ -513,6 +534,7 @@ struct Smem {
   uint64_t empty[kStages];                 // all consumer warps read the stage (8 arrivals)
   int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
   uint32_t theta[kMaxK];
+  uint32_t Tp[kMaxK], tip[kMaxK];          // the previous step's selection (T, t_idx) per worker
   // followed by the candidate staging lines: per consumer warp and worker, 32
   // indices then 32 values (staging_bytes)
 };
@@ -525,8 +547,8 @@ static_assert(smem_bytes(kBulkMaxK) <= 232448, "bulk pass shared memory above th
 // The first (up to 32) sent pairs of one sub-tile of the previous step, lane e
 // holding pair e of the list that runs through the workers in ascending order.
 struct Pairs {
-  uint32_t j;      // coordinate, or kUnsent for none
-  float v;         // value (pending aggregation only)
+  uint32_t j;      // coordinate, or kNone
+  float v;         // value
   int kw;          // worker
   uint32_t total;  // pairs in the sub-tile (warp-uniform)
 };
@@ -549,21 +571,27 @@ __device__ __forceinline__ bulk::Pairs pipe_pairs(const TopkArgs& A, uint2 cb, u
   __syncwarp();
   const uint32_t b = __shfl_sync(0xffffffffu, cb.x, src);
   const uint32_t p = __shfl_sync(0xffffffffu, pre, src);
-  P.j = kUnsent;
+  P.j = kNone;
   P.v = 0.f;
   P.kw = src;
   const uint32_t at = b + ((uint32_t)lane - p);
   if (has && at < A.cap) {
     const int64_t q = (int64_t)src * A.cap + at;
     P.j = A.cand_idx_prev[q];
-    if (A.pending) P.v = A.cand_val_prev[q];
+    P.v = A.cand_val_prev[q];
   }
   return P;
 }
 
-// Issue the load of w (pending aggregation) or of w_t - w_{t-1} (applied) at a pair.
-__device__ __forceinline__ float pipe_w(const TopkArgs& A, const bulk::Pairs& P) {
-  if ((P.j & kUnsent) || P.j >= (uint32_t)A.d) return 0.f;
+// The pair was sent: selected under its worker's selection of the previous step.
+__device__ __forceinline__ bool pair_sent(const bulk::Pairs& P, const uint32_t* Tp, const uint32_t* tip) {
+  return P.j != kNone && selected(mag_key(P.v), P.j, Tp[P.kw], tip[P.kw]);
+}
+
+// Issue the load of w (pending aggregation) or of w_t - w_{t-1} (applied) at a sent pair.
+__device__ __forceinline__ float pipe_w(const TopkArgs& A, const bulk::Pairs& P, const uint32_t* Tp,
+                                        const uint32_t* tip) {
+  if (!pair_sent(P, Tp, tip) || P.j >= (uint32_t)A.d) return 0.f;
   return A.pending ? A.w[P.j] : A.dlt[P.j];
 }
 
@@ -574,7 +602,8 @@ __device__ __forceinline__ float pipe_w(const TopkArgs& A, const bulk::Pairs& P)
 // Δ = w_{t+1} - w_t. Applied before: Δ was left in dlt; read, then cleared.
 // Returns the union coordinate this lane listed (its first sender), or ~0u.
 __device__ __forceinline__ uint32_t apply_pairs(const TopkArgs& A, uint32_t sub0, const bulk::Pairs& P,
-                                                float wv, float* dlw, uint32_t* mkw, int lane, uint32_t lt,
+                                                const uint32_t* Tp, const uint32_t* tip, float wv,
+                                                float* dlw, uint32_t* mkw, int lane, uint32_t lt,
                                                 uint32_t& uni, uint32_t& chg) {
   using bulk::kSub;
   for (int i = lane; i < kSub / 4; i += 32) {
@@ -584,7 +613,7 @@ __device__ __forceinline__ uint32_t apply_pairs(const TopkArgs& A, uint32_t sub0
   __syncwarp();
   bool act = false;
   uint32_t l = 0;
-  if (!(P.j & kUnsent)) {
+  if (pair_sent(P, Tp, tip)) {
     const int64_t ll = (int64_t)P.j - sub0;
     if (ll >= 0 && ll < kSub) {
       act = true;
@@ -634,8 +663,11 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     }
     fence_mbar_init();
   }
-  for (int kk = threadIdx.x; kk < kMaxK; kk += blockDim.x)
+  for (int kk = threadIdx.x; kk < kMaxK; kk += blockDim.x) {
     sm.theta[kk] = kk < A.K ? A.sel[kk].theta : kNoCandidate;
+    sm.Tp[kk] = kk < A.K ? A.sel[kk].T : 0u;  // this step's select runs after this pass
+    sm.tip[kk] = kk < A.K ? A.sel[kk].t_idx : 0u;
+  }
   __syncthreads();
 
   if (warp == kProducer) {
@@ -693,13 +725,13 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   uint32_t nonfinite = 0, uni = 0, chg = 0;
   bool ok = true;
   // fill the pipeline: pairs of tiles 0 and 1, w of tile 0, entries of tile 2
-  Pairs p0{kUnsent, 0.f, 0, 0u}, p1{kUnsent, 0.f, 0, 0u};
+  Pairs p0{kNone, 0.f, 0, 0u}, p1{kNone, 0.f, 0, 0u};
   float w0 = 0.f;
   uint2 c2 = make_uint2(0u, 0u);
   if (lead) {
     p0 = pipe_pairs(A, pipe_chunk(A, blockIdx.x, sw, lane), own, lane);
     p1 = pipe_pairs(A, pipe_chunk(A, blockIdx.x + stride, sw, lane), own, lane);
-    w0 = pipe_w(A, p0);
+    w0 = pipe_w(A, p0, sm.Tp, sm.tip);
     c2 = pipe_chunk(A, blockIdx.x + 2 * stride, sw, lane);
   }
   const uint32_t pair_bar = 1 + sw;  // named barrier of the sub-tile's two warps
@@ -713,7 +745,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
       uint32_t up = ~0u;
       bool many = false;
       if (p0.total <= 32u) {
-        up = apply_pairs(A, s0, p0, w0, dlw, mkw, lane, lt, uni, chg);
+        up = apply_pairs(A, s0, p0, sm.Tp, sm.tip, w0, dlw, mkw, lane, lt, uni, chg);
       } else if (A.pending) {
         stage_pending_warp(A, tile, sw, s0, kSub, dlw, mkw, lane, uni, chg);
         many = true;
@@ -738,10 +770,10 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     // the lead warp rewrites the sub-tile's buffers for the next tile only after this
     asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
     float w1 = 0.f;
-    Pairs p2{kUnsent, 0.f, 0, 0u};
+    Pairs p2{kNone, 0.f, 0, 0u};
     uint2 c3 = make_uint2(0u, 0u);
     if (lead) {  // the next tiles' loads, in flight while this tile is processed
-      w1 = pipe_w(A, p1);
+      w1 = pipe_w(A, p1, sm.Tp, sm.tip);
       p2 = pipe_pairs(A, c2, own, lane);
       c3 = pipe_chunk(A, tile + 3 * stride, sw, lane);
     }
@@ -1140,6 +1172,9 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
     S.n_tie = n_tie;
     S.ties = ties;
     S.t_idx = t_idx;
+    // ||C_k||_0: every key sent is >= T; only when T is the zero key are the
+    // n_tie ties kept zeros
+    atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(A.ksel - (T == 0u ? n_tie : 0u)));
   }
 }
 
@@ -1215,6 +1250,7 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
         const float v = vk[j];
         const uint32_t key = mag_key(v);
         const bool take = key > T || (key == T && qg < n_tie);
+        if (key == T && qg + 1 == n_tie) S.t_idx = (uint32_t)j;  // the last tie kept
         if (key == T) ++qg;
         if (take) {
           if (o < A.ksel && o < A.cap) {
@@ -1237,22 +1273,25 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
   }
   if (threadIdx.x == 0) {
     if (running != A.ksel) atomicOr(A.status, kStatusInternal);
-    // the sub-chunks now hold exactly C(v): the aggregate keeps all of them
-    S.T = 0;
-    S.t_idx = 0xffffffffu;
+    // the sub-chunks now hold exactly C(v), [0, k) of the candidate buffer
+    S.T = T;
+    S.n_tie = n_tie;
     S.dense = 1;
     atomicAdd(&A.step_ctr->v[kFallbacks], 1ull);
+    atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(A.ksel - (T == 0u ? n_tie : 0u)));
   }
 }
 
 // ---------------------------------------------------------------------------
-// aggregate + update, over all candidates in parallel (no per-tile order):
-//   mark  a candidate not sent gets its index marked (index | kUnsent); a sent
-//         one sets its worker's bit in the coordinate's mask
+// aggregate + update, over all candidates in parallel (no per-tile order),
+// when it is applied at once (an eager step, or reading the state):
+//   mark  a sent candidate sets its worker's bit in the coordinate's mask
 //   sum   the sent candidate of the lowest worker in the mask (the owner) adds
 //         the workers' values in ascending worker order from +0 -- each value
 //         is still in e[k][j], where the accumulate pass wrote it -- sets those
 //         e to +0, and applies w -= (eta/K) * sum, keeping w_{t+1} - w_t.
+// A candidate is sent iff selected(key, index, T, t_idx) under its worker's
+// selection of that step.
 // ---------------------------------------------------------------------------
 // Candidates of worker k, part p of nparts: the dense path's [0, k) when it
 // decided this worker, else a region of the bulk pass or a slice of [0, count).
@@ -1269,15 +1308,14 @@ __device__ __forceinline__ void sent_part(const TopkArgs& A, int k, int p, int n
   }
 }
 
-__global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A, int mode) {
+__global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A) {
   const int k = blockIdx.y;
   const uint32_t T = A.sel[k].T, tidx = A.sel[k].t_idx;
   const uint32_t bit = 1u << k;
-  uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
   const int nparts = candidate_parts(A);
   const int lane = threadIdx.x & 31;
-  unsigned long long nnz = 0;
   for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
     uint32_t lo, hi;
     sent_part(A, k, part, nparts, &lo, &hi);
@@ -1287,35 +1325,23 @@ __global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A, int mode) {
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const uint32_t i = i0 + q * 32 + lane;
-        jq[q] = i < hi ? ci[i] : 0xffffffffu;
+        jq[q] = i < hi ? ci[i] : kNone;
         vq[q] = i < hi ? cv[i] : 0.f;
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const uint32_t j = jq[q];
-        if (j >= (uint32_t)A.d) continue;  // beyond the part, or marked not sent already
-        if (!(mode & kMarkSent) || selected(mag_key(vq[q]), j, T, tidx)) {
-          if (mode & kMarkMask) atomicOr(&A.mask[j], bit);
-          if (mode & kMarkSample) {
-            const int slot = sample_slot(A, j);
-            if (slot >= 0) atomicOr(&A.smask_wr[slot], bit);
-          }
-          nnz += (vq[q] != 0.f);
-        } else {
-          ci[i0 + q * 32 + lane] = j | kUnsent;
-        }
+        if (j < (uint32_t)A.d && selected(mag_key(vq[q]), j, T, tidx)) atomicOr(&A.mask[j], bit);
       }
     }
-  }
-  if (mode & kMarkSent) {
-    nnz = warp_sum(nnz);
-    if ((threadIdx.x & 31) == 0 && nnz) atomicAdd(&A.step_ctr->v[kNnz], nnz);
   }
 }
 
 __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
   const int k = blockIdx.y;
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const float* cv = A.cand_val + (int64_t)k * A.cap;
+  const uint32_t T = A.sel[k].T, tidx = A.sel[k].t_idx;
   const uint32_t mine = 1u << k, lower = mine - 1u;
   const int nparts = candidate_parts(A);
   unsigned long long uni = 0, changed = 0;
@@ -1324,7 +1350,7 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
     sent_part(A, k, part, nparts, &lo, &hi);
     for (uint32_t i = lo + (threadIdx.x & 31); i < hi; i += 32) {
       const uint32_t j = __ldcg(ci + i);
-      if (j >= (uint32_t)A.d) continue;  // not sent (marked) or out of range
+      if (j >= (uint32_t)A.d || !selected(mag_key(__ldcg(cv + i)), j, T, tidx)) continue;  // not sent
       const uint32_t m = A.mask[j];
       if (!(m & mine) || (m & lower)) continue;  // a lower worker owns j (or done)
       // every sender's value is still in e[b][j]: load them all at once, then
@@ -1369,6 +1395,7 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
   __shared__ uint32_t ws[32];
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
+  const uint32_t T = A.sel[k].T, tidx = A.sel[k].t_idx;
   uint32_t carry = 0;
   for (int64_t t0 = 0; t0 < A.n_tiles; t0 += blockDim.x) {
     const int64_t tile = t0 + threadIdx.x;
@@ -1377,7 +1404,8 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
       for (int w = 0; w < kChunksPerTile; ++w) {
         const uint2 bc = A.chunk[chunk_at(A, k, tile, w)];
         const uint32_t base = bc.x, n = bc.y;
-        for (uint32_t i = 0; i < n && base + i < A.cap; ++i) cnt += (ci[base + i] & kUnsent) ? 0u : 1u;
+        for (uint32_t i = 0; i < n && base + i < A.cap; ++i)
+          cnt += selected(mag_key(cv[base + i]), ci[base + i], T, tidx) ? 1u : 0u;
       }
     }
     uint32_t tot;
@@ -1388,7 +1416,7 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
         const uint32_t base = bc.x, n = bc.y;
         for (uint32_t i = 0; i < n && base + i < A.cap; ++i) {
           const uint32_t j = ci[base + i];
-          if (j & kUnsent) continue;
+          if (!selected(mag_key(cv[base + i]), j, T, tidx)) continue;
           if (pos < A.ksel) {
             idx_out[pos] = j;
             val_out[pos] = cv[base + i];
@@ -1440,6 +1468,12 @@ int accumulate_blocks_per_sm(int tile) {
 }
 
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
+  if (A.pending && !A.dense_mode) {
+    const int n_s = A.sample_chunks ? A.sample_chunks * 8 : (int)A.d;
+    k_sample_pending<<<(n_s + kThreads - 1) / kThreads, kThreads, 0, s>>>(A);
+    const cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+  }
   k_sample<<<dim3(A.sample_blocks, A.K), kThreads, 0, s>>>(A);
   return cudaGetLastError();
 }
@@ -1473,8 +1507,8 @@ cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_mark(const TopkArgs& A, int mode, int grid, cudaStream_t s) {
-  k_mark<<<dim3(grid, A.K), kThreads, 0, s>>>(A, mode);
+cudaError_t launch_mark(const TopkArgs& A, int grid, cudaStream_t s) {
+  k_mark<<<dim3(grid, A.K), kThreads, 0, s>>>(A);
   return cudaGetLastError();
 }
 
