@@ -155,12 +155,15 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream);
  * one stream and a later gmc_step on another are ordered by the library. */
 int gmc_step(gmc_t h, const float* grads_dev, void* stream);
 
-/* gmc_step_host -- gmc_step from host memory: copies grads_host (K x d fp32,
- * row-major; pinned host memory gives an asynchronous copy) into a library
- * staging buffer (allocated on the first call), runs the step, and copies the
- * step's counters (GMC_STAT_COUNT uint64 slots, GMC_STAT_STEPS slot = 1) into
- * step_stats_host, which must then be pinned host memory valid until the
- * stream has passed the call (or NULL to skip the read-back). */
+/* gmc_step_host -- gmc_step from host memory grads_host (K x d fp32,
+ * row-major), borrowed until the stream has passed the call. Page-locked
+ * (pinned) host memory is read in place by the step's kernels over the host
+ * link; other host memory is first copied into a library staging buffer
+ * (allocated on the first such call). The step's aggregation is applied
+ * within the call, and its counters (GMC_STAT_COUNT uint64 slots,
+ * GMC_STAT_STEPS slot = 1) are copied into step_stats_host, which must then be
+ * pinned host memory valid until the stream has passed the call (or NULL to
+ * skip the read-back). */
 int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, void* stream);
 
 /* gmc_get_params -- copy w_t (d floats) into w_dev_out (applying a pending

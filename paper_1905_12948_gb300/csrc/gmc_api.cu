@@ -218,6 +218,7 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.sel_shift = h->sel_shift;
   A.sample_keys = h->sample_keys;
   A.big_tiles = h->big_tiles;
+  A.g_direct = 0;
   A.regions = h->regions;
   A.cap_region = h->cap_region;
   A.cap_part = h->cap_part;
@@ -292,13 +293,15 @@ cudaError_t order_after_flush(gmc_ctx* h, cudaStream_t s, bool clear) {
 // step's aggregation (sum of the sent pairs into w, residuals to +0 where
 // sent) is left pending unless `eager`: the next step's bulk pass applies it
 // while it streams the tile, or flush() does when the state is read.
-int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager) {
+// `direct`: grads is mapped host memory, read in place by the kernels.
+int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, bool direct = false) {
   const double Kd = (double)h->K * (double)h->d;
   GMC_TRY(order_after_flush(h, s, true));
   GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
   unsigned long long pairs_add = 0;
   if (h->compressor == GMC_TOPK) {
     TopkArgs A = topk_args(h, grads);
+    A.g_direct = direct ? 1 : 0;
     A.pending = h->agg_pending ? 1 : 0;
     A.a_prev = h->a_pending;
     const bool defer = h->tile == kBulkTile && !eager && !h->detach_out;
@@ -626,13 +629,23 @@ int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, v
   if (!h->initialized) return GMC_ESTATE;
   DeviceGuard g(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const size_t n = (size_t)h->K * (size_t)h->d;
-  if (!h->gstage) {
-    cudaError_t err = dalloc(h, &h->gstage, n);
-    if (err != cudaSuccess) return status_of(err);
+  // page-locked host memory is mapped into the device's address space: the
+  // kernels read the gradients in place, each crossing the host link once
+  // while the pass runs; other host memory is copied to a staging buffer first
+  const float* mapped = nullptr;
+  int st;
+  if (cudaHostGetDevicePointer((void**)&mapped, const_cast<float*>(grads_host), 0) == cudaSuccess) {
+    st = enqueue_step(h, mapped, s, true, true);
+  } else {
+    cudaGetLastError();
+    const size_t n = (size_t)h->K * (size_t)h->d;
+    if (!h->gstage) {
+      cudaError_t err = dalloc(h, &h->gstage, n);
+      if (err != cudaSuccess) return status_of(err);
+    }
+    GMC_TRY(cudaMemcpyAsync(h->gstage, grads_host, n * sizeof(float), cudaMemcpyHostToDevice, s));
+    st = enqueue_step(h, h->gstage, s, true);
   }
-  GMC_TRY(cudaMemcpyAsync(h->gstage, grads_host, n * sizeof(float), cudaMemcpyHostToDevice, s));
-  const int st = enqueue_step(h, h->gstage, s, true);
   if (st != GMC_OK) return st;
   if (step_stats_host)
     GMC_TRY(cudaMemcpyAsync(step_stats_host, h->step_ctr, sizeof(Counters), cudaMemcpyDeviceToHost, s));

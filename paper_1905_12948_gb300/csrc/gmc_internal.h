@@ -53,6 +53,7 @@ struct TopkArgs {
   float* cand_val;
   uint2* chunk;              // sub-chunk (base, count): n_tiles x kChunksPerTile x K, see chunk_at
   uint32_t* mask;            // d: workers that sent each coordinate (bit k), zero between steps
+  int g_direct;              // grads is mapped host memory: read it with loads, not bulk copies
   const uint32_t* cand_idx_prev;    // previous step's sub-chunks
   const float* cand_val_prev;
   const uint2* chunk_prev;

@@ -691,7 +691,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         const uint32_t off = (uint32_t)(ga & 15) >> 2;
         const char* gsrc = reinterpret_cast<const char*>(ga - off * 4);
         const uint32_t gbytes = (uint32_t)(((nvalid + off) * 4 + 15) & ~int64_t(15));
-        const bool gbulk = (ga & 3) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
+        const bool gbulk = !A.g_direct && (ga & 3) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
         sm.gmeta[s] = gbulk ? (int32_t)off : -1;
         mbar_arrive_expect_tx(&sm.full[s], kT * 4 + (gbulk ? gbytes : 0));
         bulk_load(sm.e[s], esrc, kT * 4, &sm.full[s]);

@@ -87,3 +87,32 @@ def test_deferred_steps_mixed_with_host_steps_and_detach():
         p.compare(r, state=False)
     p.compare(r)
     p.compare_stats()
+
+
+@pytest.mark.parametrize("pinned", [True, False])
+def test_host_steps_pinned_and_pageable(pinned):
+    """gmc_step_host on the bulk pass: pinned (mapped) host gradients are read
+    in place by the kernels, pageable ones copied to a staging buffer first.
+    Several host steps in a row, then device steps, against the oracle."""
+    import torch
+    K = 5
+    rng = np.random.default_rng(34 + pinned)
+    p = Pair(D_BULK, K, 0.9, 0.1, ratio=0.003, seed=8)
+    stats = torch.zeros(8, dtype=torch.int64).pin_memory()
+    for t in range(3):
+        g = _grads(rng, K, D_BULK)
+        host = torch.from_numpy(g)
+        if pinned:
+            host = host.pin_memory()
+        p.gpu.step_host(host, stats)
+        r = p.ref.step(g)
+        torch.cuda.synchronize()
+        assert int(stats[1]) == r.stats["pairs"] and int(stats[2]) == r.stats["nnz"]
+        assert int(stats[3]) == r.stats["union"] and int(stats[4]) == r.stats["changed"]
+        p.compare(r, residuals=(t == 2))
+    for t in range(2):
+        r = p.step(_grads(rng, K, D_BULK))
+        p.compare(r, state=(t == 1))
+    p.compare_stats()
+    assert p.gpu.stats()["fallbacks"] == 0
+    assert p.gpu.check() == 0
