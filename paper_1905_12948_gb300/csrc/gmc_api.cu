@@ -54,6 +54,7 @@ struct gmc_ctx {
   float* dlt = nullptr;
   WorkerSel* sel = nullptr;
   uint32_t* ghist = nullptr;
+  uint32_t* chist = nullptr;
   uint32_t* bucket = nullptr;  // K x 2*kBucketCap
   int sel_shift = 20;
   uint32_t* sample_keys = nullptr;
@@ -214,6 +215,7 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.dense_mode = h->select_mode == GMC_SELECT_DENSE;
   A.sel = h->sel;
   A.ghist = h->ghist;
+  A.chist = h->chist;
   A.bucket = h->bucket;
   A.sel_shift = h->sel_shift;
   A.sample_keys = h->sample_keys;
@@ -495,6 +497,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->dlt, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->sel, (size_t)K)) != cudaSuccess ||
         (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess ||
+        (err = dalloc(h, &h->chist, (size_t)K * kRelBins)) != cudaSuccess ||
         (err = dalloc(h, &h->bucket, (size_t)K * 2 * kBucketCap)) != cudaSuccess ||
         (err = dalloc(h, &h->sample_keys, (size_t)K * 8 * kSampleChunks)) != cudaSuccess ||
         (err = dalloc(h, &h->big_tiles, (size_t)h->n_tiles + 1)) != cudaSuccess ||

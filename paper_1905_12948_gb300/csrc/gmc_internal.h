@@ -44,7 +44,8 @@ struct TopkArgs {
   int has_prev;              // a previous step exists (t > 0)
   int dense_mode;            // GMC_SELECT_DENSE
   WorkerSel* sel;            // K entries
-  uint32_t* ghist;           // K x kHistBins (zero between uses)
+  uint32_t* ghist;           // K x kHistBins: the sample's histogram (zero between uses)
+  uint32_t* chist;           // K x kRelBins: the candidates' relative histogram (zeroed by the sample)
   uint32_t* bucket;          // K x 2*kBucketCap: keys, then indices of the k-th key's bin
   int sel_shift;             // log2 of the relative-histogram bin width (in keys)
   uint32_t* sample_keys;     // K x 8*kSampleChunks

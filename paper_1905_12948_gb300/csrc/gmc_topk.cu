@@ -114,6 +114,13 @@ __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
   A.sample_pend[kSampleSlots + i] = __float_as_uint(dd);
 }
 
+// Bin of a candidate key in the relative histogram: (key - theta) >> shift,
+// the top bin also taking everything further up (candidate keys are >= theta).
+__device__ __forceinline__ int rel_bin(uint32_t key, uint32_t theta, int shift) {
+  const uint32_t b = (key > theta ? key - theta : 0u) >> shift;
+  return b < (uint32_t)kRelBins ? (int)b : kRelBins - 1;
+}
+
 // ---------------------------------------------------------------------------
 // sample: blocks spread over the workers' samples; the last block of a worker
 // fixes two radix digits of the sample's r-th largest key. Where the previous
@@ -127,6 +134,8 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
   if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) A.big_tiles[0] = 0;
+  if (blockIdx.x == 0)  // this step's candidate histogram starts empty
+    for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) A.chist[(int64_t)k * kRelBins + b] = 0u;
   if (A.dense_mode) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       S.theta = kNoCandidate;
@@ -907,6 +916,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
             ci[line * 32 + lane] = si[lane];
             cv[line * 32 + lane] = x;
             nonfinite += is_nonfinite(x) ? 1u : 0u;
+            atomicAdd(&A.chist[(int64_t)k * kRelBins + rel_bin(mag_key(x), th, A.sel_shift)], 1u);
           }
           __syncwarp();
         }
@@ -942,6 +952,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
       A.cand_idx[(int64_t)k * A.cap + part0 + line * 32 + lane] = si[lane];
       A.cand_val[(int64_t)k * A.cap + part0 + line * 32 + lane] = x;
       nonfinite += is_nonfinite(x) ? 1u : 0u;
+      atomicAdd(&A.chist[(int64_t)k * kRelBins + rel_bin(mag_key(x), sm.theta[k], A.sel_shift)], 1u);
     }
   }
   if (nonfinite) {
@@ -988,17 +999,10 @@ __device__ __forceinline__ void candidate_part(const TopkArgs& A, int k, int p, 
 //           equal T are kept, and -- when fewer are kept than there are -- the
 //           largest index kept (ties go to the lower index)
 // ---------------------------------------------------------------------------
-// Bin of a candidate key in the relative histogram: (key - theta) >> shift,
-// the top bin also taking everything further up (candidate keys are >= theta).
-__device__ __forceinline__ int rel_bin(uint32_t key, uint32_t theta, int shift) {
-  const uint32_t b = (key > theta ? key - theta : 0u) >> shift;
-  return b < (uint32_t)kRelBins ? (int)b : kRelBins - 1;
-}
-
+// The candidate histogram of the load/store pass (the bulk pass counts its
+// candidates into chist as they leave its staging lines).
 __global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
   __shared__ uint32_t h[kRelBins];
-  __shared__ uint32_t ws[32];
-  __shared__ uint32_t s_last, s_bin, s_rank;
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
   if (needs_dense(S, A.ksel, A.cap)) return;
@@ -1023,31 +1027,9 @@ __global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
     }
   }
   __syncthreads();
-  uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
+  uint32_t* gh = A.chist + (int64_t)k * kRelBins;
   for (int b = threadIdx.x; b < kRelBins; b += blockDim.x)
     if (h[b]) atomicAdd(&gh[b], h[b]);
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[0], 1u) == gridDim.x - 1) ? 1u : 0u;
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) {
-    h[b] = __ldcg(&gh[b]);
-    gh[b] = 0;
-  }
-  if (threadIdx.x == 0) {
-    s_bin = 0;
-    s_rank = 0;
-    S.done[0] = 0;
-  }
-  __syncthreads();
-  block_find_from_top(h, kRelBins, A.ksel, ws, &s_bin, &s_rank);
-  if (threadIdx.x == 0) {
-    if (s_rank == 0) atomicOr(A.status, kStatusInternal);
-    S.prefix = s_bin;  // relative bin of the k-th key
-    S.rank = s_rank;   // its rank inside that bin
-  }
 }
 
 // Radix select in shared memory: the r-th largest of n values (digits 11/10/10).
@@ -1092,7 +1074,20 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   WorkerSel& S = A.sel[k];
   if (needs_dense(S, A.ksel, A.cap)) return;
   const uint32_t theta = S.theta;
-  const int want = (int)S.prefix;
+  // the bin holding the k-th key, and its rank there (every block, from the histogram)
+  for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) h[b] = __ldcg(&A.chist[(int64_t)k * kRelBins + b]);
+  if (threadIdx.x == 0) {
+    s_bin = 0;
+    s_rank = 0;
+  }
+  __syncthreads();
+  block_find_from_top(h, kRelBins, A.ksel, ws, &s_bin, &s_rank);
+  const int want = (int)s_bin;
+  const uint32_t want_rank = s_rank;
+  if (want_rank == 0) {  // fewer candidates than k counted: the dense path decides
+    if (blockIdx.x == 0 && threadIdx.x == 0) S.dense = 1;
+    return;
+  }
   const int lane = threadIdx.x & 31;
   const uint32_t lt = lanemask_lt();
   uint32_t* bk = A.bucket + (int64_t)k * 2 * kBucketCap;  // keys, then indices
@@ -1148,7 +1143,7 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   }
   __syncthreads();
   uint32_t n_tie;
-  const uint32_t T = smem_select(keys, n, S.rank, h, ws, &s_bin, &s_rank, &n_tie);
+  const uint32_t T = smem_select(keys, n, want_rank, h, ws, &s_bin, &s_rank, &n_tie);
   // ties: gather the indices of the keys equal to T over the keys, in place;
   // a round writes below the end of what the block has read so far
   if (threadIdx.x == 0) s_n = 0;
@@ -1495,9 +1490,11 @@ cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
 
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s) {
   const dim3 grid(blocks_per_worker, A.K);
-  k_select_hist<<<grid, kThreads, 0, s>>>(A);
-  cudaError_t err = cudaGetLastError();
-  if (err != cudaSuccess) return err;
+  if (A.regions == 1) {  // the bulk pass histogrammed its candidates already
+    k_select_hist<<<grid, kThreads, 0, s>>>(A);
+    const cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+  }
   k_select_finish<<<grid, kThreads, 2 * kBucketCap * 4, s>>>(A);
   return cudaGetLastError();
 }
