@@ -538,7 +538,7 @@ struct Smem {
   uint32_t mk[kSubTiles][kSub];            // senders of the pending aggregation (bit k)
   uint8_t own[kSubTiles][32];              // scratch: worker of each listed pair
   uint32_t upos[kSubTiles][32];            // union coordinates of a sub-tile, one per lane
-  uint32_t pflag[kSubTiles][2];            // per sub-tile: the two warps' status, many-senders flag
+  uint32_t pflag[kSubTiles];               // per sub-tile: more than 32 pairs (per-element masks)
   uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
   uint64_t empty[kStages];                 // all consumer warps read the stage (8 arrivals)
   int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
@@ -732,7 +732,8 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   uint32_t run = 0;
   const int64_t stride = gridDim.x;
   uint32_t nonfinite = 0, uni = 0, chg = 0;
-  bool ok = true;
+  bool ok = true;  // false after a bounded wait gave up: the items are skipped, the tile loop
+                   // still runs (its named barriers need both warps of the sub-tile)
   // fill the pipeline: pairs of tiles 0 and 1, w of tile 0, entries of tile 2
   Pairs p0{kNone, 0.f, 0, 0u}, p1{kNone, 0.f, 0, 0u};
   float w0 = 0.f;
@@ -762,14 +763,10 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         stage_delta_warp(A, tile, sw, s0, kSub, dlw, lane);
       }
       sm.upos[sw][lane] = up;
-      if (lane == 0) sm.pflag[sw][1] = many ? 1u : 0u;
+      if (lane == 0) sm.pflag[sw] = many ? 1u : 0u;
     }
-    if (lane == 0) sm.pflag[sw][0] = 0;  // both warps: report a timeout below
     asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
-    if (lane == 0 && !ok) atomicOr(&sm.pflag[sw][0], 1u);
-    asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
-    if (sm.pflag[sw][0]) break;  // one of the two warps gave up: both leave together
-    const bool many = sm.pflag[sw][1] != 0u;
+    const bool many = sm.pflag[sw] != 0u;
     const uint32_t upos = sm.upos[sw][lane];
     const uint32_t umask = (A.pending && upos != ~0u) ? mkw[upos] : 0u;
     const bool patch = __any_sync(0xffffffffu, umask != 0u);
@@ -795,7 +792,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
 #pragma unroll
       for (int i = 0; i < 4; ++i) valid |= (u * 128 + lane * 4 + i < lim ? 1u : 0u) << (4 * u + i);
     uint2 bc_lane = make_uint2(0u, 0u);
-    for (int k = gp; k < A.K; k += 2) {
+    for (int k = gp; ok && k < A.K; k += 2) {
       const uint32_t item = n * (uint32_t)A.K + (uint32_t)k;
       const uint32_t s = item % kStages, r = item / kStages;
       if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
