@@ -116,3 +116,43 @@ def test_host_steps_pinned_and_pageable(pinned):
     p.compare_stats()
     assert p.gpu.stats()["fallbacks"] == 0
     assert p.gpu.check() == 0
+
+
+def test_dense_sub_tiles_and_ties_on_the_bulk_pass():
+    """Many sent pairs per 512-coordinate sub-tile (more than one per lane:
+    the per-element sender masks), K = 1 and an odd K, ties across tiles,
+    deferred and host (applied at once) steps alternating."""
+    import torch
+    for K, ratio in ((1, 0.05), (7, 0.02)):
+        rng = np.random.default_rng(40 + K)
+        p = Pair(D_BULK, K, 0.9, 0.1, ratio=ratio, seed=9)
+        stats = torch.zeros(8, dtype=torch.int64).pin_memory()
+        for t in range(4):
+            g = _grads(rng, K, D_BULK)
+            g[:, rng.integers(0, D_BULK, size=4000)] = np.float32(0.75)  # ties across tiles
+            if t % 2:
+                p.gpu.step_host(torch.from_numpy(g).pin_memory(), stats)
+                r = p.ref.step(g)
+                torch.cuda.synchronize()
+            else:
+                r = p.step(g)
+            p.compare(r, state=(t == 3))
+        p.compare_stats()
+        assert p.gpu.check() == 0
+        p.gpu.close()
+
+
+def test_bulk_pass_reports_non_finite_values():
+    """NaN and Inf gradients on the bulk pass: the step completes, counts
+    them, and gmc_check reports GMC_ENONFINITE."""
+    import torch
+    K = 2
+    rng = np.random.default_rng(44)
+    p = Pair(D_BULK, K, 0.9, 0.1, ratio=0.002, seed=10)
+    g = _grads(rng, K, D_BULK)
+    g[0, 12345] = np.nan
+    g[1, 999_999] = np.inf
+    p.gpu.step(torch.from_numpy(g).to(p.dev))
+    torch.cuda.synchronize()
+    assert p.gpu.stats()["nonfinite"] == 2
+    assert p.gpu.check() == 4  # GMC_ENONFINITE
