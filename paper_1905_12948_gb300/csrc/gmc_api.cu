@@ -46,6 +46,7 @@ struct gmc_ctx {
   int64_t nb = 0, m = 0;
   uint32_t B_shift = 0xffffffffu;
   int grid_acc = 1, grid_agg = 1, grid_rbgs = 1, sel_blocks = 1;
+  bool rbgs_bulk = false;
   // state
   int64_t t = 0;
   bool initialized = false;
@@ -256,6 +257,7 @@ RbgsArgs rbgs_args(gmc_ctx* h, const float* grads) {
   A.c = h->beta / h->eta;
   A.a = h->eta / (float)h->K;
   A.K = h->K;
+  A.bulk = h->rbgs_bulk ? 1 : 0;
   A.n_tiles = h->n_tiles;
   A.B = h->block;
   A.B_shift = h->B_shift;
@@ -329,7 +331,8 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
     }
     pairs_add = (unsigned long long)h->K * h->ksel;
   } else {
-    const RbgsArgs A = rbgs_args(h, grads);
+    RbgsArgs A = rbgs_args(h, grads);
+    A.g_direct = direct ? 1 : 0;
     GMC_TRY(cudaMemsetAsync(A.uflag_cur, 0, (size_t)h->nb, s));
     GMC_TRY(timed(h, GMC_KERNEL_RBGS_PICK, 0.0, s, [&] { return launch_rbgs_pick(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_RBGS_STEP, 12.0 * Kd, s,
@@ -527,7 +530,10 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
       while ((int64_t(1) << sh) < block) ++sh;
       h->B_shift = sh;
     }
-    h->grid_rbgs = (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * rbgs_blocks_per_sm());
+    // enough tiles for one per SM: the bulk-copy kernel (one persistent CTA per SM)
+    h->rbgs_bulk = h->n_tiles >= h->num_sms;
+    h->grid_rbgs = h->rbgs_bulk ? h->num_sms
+                                : (int)std::min<int64_t>(h->n_tiles, (int64_t)h->num_sms * rbgs_blocks_per_sm());
     const int64_t nbw = (h->nb + 31) / 32;
     if ((err = dalloc(h, &h->e, (size_t)K * h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->w, (size_t)h->ld)) != cudaSuccess ||

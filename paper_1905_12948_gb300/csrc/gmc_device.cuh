@@ -77,6 +77,13 @@ __device__ __forceinline__ void warp_hist_add(uint32_t* hist, int bin) {
   const int leader = __ffs(peers) - 1;
   if (bin >= 0 && (int)(threadIdx.x & 31) == leader) atomicAdd(&hist[bin], (uint32_t)__popc(peers));
 }
+// Sum over the 32 lanes of a warp (all lanes must call it).
+template <typename V>
+__device__ __forceinline__ V warp_sum(V x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
 __device__ __forceinline__ uint32_t lanemask_lt() {
   uint32_t m;
   asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));

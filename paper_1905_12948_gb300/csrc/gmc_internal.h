@@ -101,6 +101,8 @@ struct RbgsArgs {
   uint8_t* uflag_cur;        // nb: union of this step's blocks
   float* slab;               // K x (m*B): C(e_{t+1/2,k}) values, block slot major
   int has_prev;
+  int bulk;                  // k_rbgs_bulk (bulk copies through shared memory), else k_rbgs_step
+  int g_direct;              // grads is mapped host memory: read it with loads, not bulk copies
   Counters* step_ctr;
   unsigned* status;
 };

@@ -269,11 +269,235 @@ __global__ void k_finalize(Counters* step, Counters* total, unsigned long long p
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// The same step as k_rbgs_step, with e and g streamed through a shared-memory
+// ring by bulk copies. One persistent CTA per SM: a producer thread issues
+// each (tile, worker) item's cp.async.bulk copies of e and g into the ring;
+// sixteen consumer warps each own 256 elements of every tile and run through
+// the K workers in ascending order (the aggregate adds in that order).
+// Producer and consumers meet only at mbarriers; every wait is bounded.
+// ---------------------------------------------------------------------------
+namespace rbulk {
+constexpr int kT = kRbgsTile;
+constexpr int kStages = 4;
+constexpr int kConsumers = 16;
+constexpr int kSub = kT / kConsumers;      // 256 elements per consumer warp
+constexpr int kGLen = kT + 8;              // g stage: up to 3 leading floats of misalignment
+constexpr int kThreadsAll = (kConsumers + 1) * 32;
+constexpr int kG = kSub / 128;             // float4 groups per lane
+struct Smem {
+  float e[kStages][kT];
+  float g[kStages][kGLen];
+  uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
+  uint64_t empty[kStages];                 // all consumer warps read the stage
+  int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
+};
+}  // namespace rbulk
+
+__global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A) {
+  using namespace rbulk;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kConsumers);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumers) {
+    // ---- producer ----
+    if (lane != 0) return;
+    const char* g_lo = reinterpret_cast<const char*>(A.grads);
+    const char* g_hi = reinterpret_cast<const char*>(A.grads + (int64_t)A.K * A.d);
+    uint32_t item = 0;
+    bool ok = true;
+    for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+      const int64_t j0 = tile * kT;
+      const int64_t nvalid = A.d - j0 < kT ? A.d - j0 : kT;
+      for (int k = 0; k < A.K; ++k, ++item) {
+        const uint32_t s = item % kStages, r = item / kStages;
+        if (r > 0 && !wait_bounded(&sm.empty[s], (r - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        const float* esrc = A.e + (int64_t)k * A.ld + j0;
+        const uintptr_t ga = reinterpret_cast<uintptr_t>(A.grads + (int64_t)k * A.d + j0);
+        const uint32_t off = (uint32_t)(ga & 15) >> 2;
+        const char* gsrc = reinterpret_cast<const char*>(ga - off * 4);
+        const uint32_t gbytes = (uint32_t)(((nvalid + off) * 4 + 15) & ~int64_t(15));
+        const bool gbulk = !A.g_direct && (ga & 3) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
+        sm.gmeta[s] = gbulk ? (int32_t)off : -1;
+        mbar_arrive_expect_tx(&sm.full[s], kT * 4 + (gbulk ? gbytes : 0));
+        bulk_load(sm.e[s], esrc, kT * 4, &sm.full[s]);
+        if (gbulk) bulk_load(sm.g[s], gsrc, gbytes, &sm.full[s]);
+      }
+    }
+    if (!ok) {
+      atomicOr(A.status, kStatusTimeout);
+      // let the copies already issued land before the CTA's shared memory goes away
+      const uint32_t first = item > (uint32_t)kStages ? item - kStages : 0u;
+      for (uint32_t i = first; i < item; ++i) wait_bounded(&sm.full[i % kStages], (i / kStages) & 1);
+    }
+    return;
+  }
+
+  // ---- consumers ----
+  const int64_t slab_ld = A.m * A.B;
+  uint32_t nonfinite = 0;
+  unsigned long long pairs = 0, nnz = 0, uni = 0, changed = 0;
+  uint32_t item = 0;
+  bool ok = true;
+  for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+    const int64_t s0 = tile * kT + warp * kSub;
+    const int64_t rem = A.d - s0;
+    const int lim = rem < kSub ? (rem > 0 ? (int)rem : 0) : kSub;
+    // does the sub-tile touch the last step's union (tp) or this step's (tc)?
+    int tp = 0, tc = 0;
+    if (lim > 0) {
+      const int64_t b_lo = block_of(s0, A), b_hi = block_of(s0 + lim - 1, A);
+      for (int64_t b = b_lo + lane; b <= b_hi; b += 32) {
+        tp |= A.has_prev ? A.uflag_prev[b] : 0;
+        tc |= A.uflag_cur[b];
+      }
+    }
+    tp = __any_sync(0xffffffffu, tp);
+    tc = __any_sync(0xffffffffu, tc);
+    float dl[kG][4], acc[kG][4];
+    uint32_t bid[kG][4];
+    uint32_t inU = 0;  // bit (u*4+i): coordinate in this step's union
+#pragma unroll
+    for (int u = 0; u < kG; ++u) {
+      const int l = u * 128 + lane * 4;
+      float4 d4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (tp && l < lim) d4 = *reinterpret_cast<const float4*>(A.dlt + s0 + l);
+      dl[u][0] = d4.x; dl[u][1] = d4.y; dl[u][2] = d4.z; dl[u][3] = d4.w;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        acc[u][i] = 0.f;
+        const bool in = l + i < lim;
+        bid[u][i] = (in && tc) ? block_of(s0 + l + i, A) : 0u;
+        if (in && tc && A.uflag_cur[bid[u][i]]) inU |= 1u << (u * 4 + i);
+      }
+    }
+    for (int k = 0; k < A.K; ++k, ++item) {
+      const uint32_t s = item % kStages, r = item / kStages;
+      if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
+        ok = false;
+        break;
+      }
+      const int32_t off = sm.gmeta[s];
+      const float* se = sm.e[s] + warp * kSub;
+      const float* sg = sm.g[s] + (off > 0 ? off : 0) + warp * kSub;
+      float v[kG][4];
+#pragma unroll
+      for (int u = 0; u < kG; ++u) {
+        const int l = u * 128 + lane * 4;
+        const float4 e4 = *reinterpret_cast<const float4*>(se + l);
+        float4 g4;
+        if (off == 0) {
+          g4 = *reinterpret_cast<const float4*>(sg + l);
+        } else if (off == 2) {
+          const float2 a = *reinterpret_cast<const float2*>(sg + l);
+          const float2 b = *reinterpret_cast<const float2*>(sg + l + 2);
+          g4 = make_float4(a.x, a.y, b.x, b.y);
+        } else if (off > 0) {
+          g4 = make_float4(sg[l], sg[l + 1], sg[l + 2], sg[l + 3]);
+        } else {
+          const float* gk = A.grads + (int64_t)k * A.d;
+          g4 = load_g4(gk, s0 + l, A.d, g_mode(gk));
+        }
+        if (lim < kSub && off >= 0) {  // past d the stage holds bytes of no meaning
+          if (l >= lim) g4.x = 0.f;
+          if (l + 1 >= lim) g4.y = 0.f;
+          if (l + 2 >= lim) g4.z = 0.f;
+          if (l + 3 >= lim) g4.w = 0.f;
+        }
+        v[u][0] = accumulate(e4.x, g4.x, A.c, dl[u][0]);
+        v[u][1] = accumulate(e4.y, g4.y, A.c, dl[u][1]);
+        v[u][2] = accumulate(e4.z, g4.z, A.c, dl[u][2]);
+        v[u][3] = accumulate(e4.w, g4.w, A.c, dl[u][3]);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.empty[s]);  // this warp is done reading stage s
+      float* ek = A.e + (int64_t)k * A.ld + s0;
+      const int32_t* rk = A.rank + (A.per_worker ? (int64_t)k * A.nb : 0);
+      float* sk = A.slab + (int64_t)k * slab_ld;
+#pragma unroll
+      for (int u = 0; u < kG; ++u) {
+        const int l = u * 128 + lane * 4;
+        float en[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          en[i] = v[u][i];
+          if (l + i < lim) {
+            nonfinite += is_nonfinite(v[u][i]) ? 1u : 0u;
+            if (tc) {
+              const int32_t q = rk[bid[u][i]];
+              if (q >= 0) {  // in one of worker k's chosen blocks: sent
+                acc[u][i] = __fadd_rn(acc[u][i], v[u][i]);
+                sk[(int64_t)q * A.B + (s0 + l + i - (int64_t)bid[u][i] * A.B)] = v[u][i];
+                en[i] = 0.f;  // e_{t+1,k} = +0 where sent
+                ++pairs;
+                nnz += (v[u][i] != 0.f);
+              }
+            }
+          }
+        }
+        __stcs(reinterpret_cast<float4*>(ek + l), make_float4(en[0], en[1], en[2], en[3]));
+      }
+    }
+    if (ok && (tp || tc)) {  // the union: w_{t+1} = w_t - a * sum, and w_{t+1} - w_t for the next step
+#pragma unroll
+      for (int u = 0; u < kG; ++u) {
+        const int l = u * 128 + lane * 4;
+        if (l >= lim) continue;
+        float dd[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          if (inU & (1u << (u * 4 + i))) {
+            const float wo = A.w[s0 + l + i];
+            const float wn = __fsub_rn(wo, __fmul_rn(A.a, acc[u][i]));
+            A.w[s0 + l + i] = wn;
+            dd[i] = __fsub_rn(wn, wo);
+            changed += (dd[i] != 0.f);
+            ++uni;
+          }
+        }
+        *reinterpret_cast<float4*>(A.dlt + s0 + l) = make_float4(dd[0], dd[1], dd[2], dd[3]);
+      }
+    }
+  }
+  if (!ok) atomicOr(A.status, kStatusTimeout);
+  pairs = warp_sum(pairs);
+  nnz = warp_sum(nnz);
+  uni = warp_sum(uni);
+  changed = warp_sum(changed);
+  if (lane == 0) {
+    if (pairs) atomicAdd(&A.step_ctr->v[kPairs], pairs);
+    if (nnz) atomicAdd(&A.step_ctr->v[kNnz], nnz);
+    if (uni) atomicAdd(&A.step_ctr->v[kUnion], uni);
+    if (changed) atomicAdd(&A.step_ctr->v[kChanged], changed);
+  }
+  if (nonfinite) {
+    atomicOr(A.status, kStatusNonfinite);
+    atomicAdd(&A.step_ctr->v[kNonfinite], (unsigned long long)nonfinite);
+  }
+}
+
 }  // namespace
 
 cudaError_t configure_rbgs_kernels() {
-  return cudaFuncSetAttribute((const void*)k_rbgs_pick,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, kPickSmemWords * 4);
+  cudaError_t err = cudaFuncSetAttribute((const void*)k_rbgs_pick,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kPickSmemWords * 4);
+  const cudaError_t e2 = cudaFuncSetAttribute((const void*)k_rbgs_bulk,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)sizeof(rbulk::Smem));
+  return err != cudaSuccess ? err : e2;
 }
 
 int rbgs_blocks_per_sm() {
@@ -290,7 +514,11 @@ cudaError_t launch_rbgs_pick(const RbgsArgs& A, cudaStream_t s) {
 }
 
 cudaError_t launch_rbgs_step(const RbgsArgs& A, int grid, cudaStream_t s) {
-  k_rbgs_step<<<grid, kThreads, 0, s>>>(A);
+  if (A.bulk) {
+    k_rbgs_bulk<<<grid, rbulk::kThreadsAll, (int)sizeof(rbulk::Smem), s>>>(A);
+  } else {
+    k_rbgs_step<<<grid, kThreads, 0, s>>>(A);
+  }
   return cudaGetLastError();
 }
 

@@ -48,12 +48,6 @@ __device__ __forceinline__ int g_mode(const float* p) {
   return (a & 15) == 0 ? 4 : ((a & 7) == 0 ? 2 : 1);
 }
 
-template <typename V>
-__device__ __forceinline__ V warp_sum(V x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-  return x;
-}
 
 __device__ __forceinline__ uint32_t warp_excl_scan(uint32_t x, uint32_t* total) {
   const int lane = threadIdx.x & 31;
