@@ -1088,23 +1088,31 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
     uint32_t lo, hi;
     candidate_part(A, k, part, nparts, &lo, &hi);
-    for (uint32_t i0 = lo; i0 < hi; i0 += 32) {
-      const uint32_t i = i0 + lane;
-      uint32_t key = 0;
-      bool in = false;
-      if (i < hi) {
-        key = mag_key(cv[i]);
-        in = rel_bin(key, theta, A.sel_shift) == want;
+    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * 32) {  // 128 candidates a round, one reservation
+      uint32_t key[4], m[4], n = 0;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t i = i0 + q * 32 + lane;
+        key[q] = i < hi ? mag_key(cv[i]) : 0u;
       }
-      const uint32_t m = __ballot_sync(0xffffffffu, in);
-      if (m) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t i = i0 + q * 32 + lane;
+        m[q] = __ballot_sync(0xffffffffu, i < hi && rel_bin(key[q], theta, A.sel_shift) == want);
+        n += __popc(m[q]);
+      }
+      if (n) {
         uint32_t base = 0;
-        if (lane == 0) base = atomicAdd(&S.count_bucket, (uint32_t)__popc(m));
+        if (lane == 0) base = atomicAdd(&S.count_bucket, n);
         base = __shfl_sync(0xffffffffu, base, 0);
-        const uint32_t o = base + __popc(m & lt);
-        if (in && o < (uint32_t)kBucketCap) {
-          bk[o] = key;
-          bk[kBucketCap + o] = ci[i];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const uint32_t o = base + __popc(m[q] & lt);
+          if (((m[q] >> lane) & 1u) && o < (uint32_t)kBucketCap) {
+            bk[o] = key[q];
+            bk[kBucketCap + o] = ci[i0 + q * 32 + lane];
+          }
+          base += __popc(m[q]);
         }
       }
     }
