@@ -15,7 +15,11 @@ Communication in Distributed Learning", arXiv 1905.12948):
         w_{t+1,k}   = w_{t+1} - lambda*eta*e_{t+1,k},   w_{0,k} = w_0.
     Gradients are inputs here, so the detached points are an output only.
   * Compressors (Sec. 4): top-s (the s components of largest magnitude) and
-    RBGS (random blocks chosen with one seed shared by all workers, Sec. 5.2).
+    RBGS (random blocks chosen with one seed shared by all workers, Sec. 5.2);
+    the approximate top-s of Sec. 5.1 (after DGC): a threshold theta taken
+    from a random sample S of d/100 components, such that |S|/1024 -- the
+    compression ratio times |S| -- sampled magnitudes reach it; every
+    component with |a| >= theta is sent.
   * Relative communication cost (Sec. 5, RCC), halved for RBGS (Sec. 5.2).
 
 Precision. The paper fixes none. Top-s turns floating-point magnitudes into an
@@ -38,7 +42,15 @@ Readings where the paper is silent:
     sampling (Bentley & Floyd, CACM 1987) from a SplitMix64 counter stream
     (Steele, Lea & Flood, OOPSLA 2014) keyed by (seed, t) -- or (seed, t, k)
     in the per-worker mode -- with multiply-shift range reduction;
-  * the residual at a sent coordinate is +0 exactly (v - v for finite v).
+  * the residual at a sent coordinate is +0 exactly (v - v for finite v);
+  * approximate top-s: |S| = max(1, floor(d/100)); S is drawn afresh each
+    step, the same for all workers, one component from each of |S| strata
+    [floor(i d/|S|), floor((i+1) d/|S|)), picked by the i-th draw of the
+    SplitMix64 stream keyed by (seed, t) with multiply-shift reduction;
+    theta is the r-th largest sampled magnitude key, r = max(1,
+    floor(ratio |S|)); a component is sent iff its key is >= theta's; when
+    more than M = min(d, 4 s + 4096) components reach theta (s the nominal
+    count of top-s), the exact top-M is sent instead.
 """
 from __future__ import annotations
 
@@ -52,6 +64,9 @@ U32 = np.uint32
 
 TOPK = "topk"
 RBGS = "rbgs"
+TOPK_APPROX = "topk_approx"
+
+APPROX_SAMPLE_DIV = 100  # |S| = d/100 (Sec. 5.1)
 
 # ---------------------------------------------------------------------------
 # Compressors
@@ -138,6 +153,51 @@ def floyd_blocks(key: int, nb: int, m: int) -> np.ndarray:
     return np.array(sorted(chosen), np.int64)
 
 
+def approx_sample_size(d: int) -> int:
+    """|S| = max(1, floor(d/100)), the sample of the approximate top-s (Sec. 5.1)."""
+    return max(1, d // APPROX_SAMPLE_DIV)
+
+
+def approx_rank(n_sample: int, ratio: float) -> int:
+    """r = max(1, floor(ratio * |S|)): how many sampled magnitudes reach theta
+    (|S|/1024 in Sec. 5.1, where the ratio is 1/1024)."""
+    return max(1, math.floor(ratio * n_sample))
+
+
+def approx_limit(d: int, ratio: float) -> int:
+    """M = min(d, 4 s + 4096): the most components the approximate top-s sends
+    (beyond it, the exact top-M)."""
+    return min(d, 4 * topk_count(d, ratio) + 4096)
+
+
+def approx_sample_positions(seed: int, t: int, d: int, n_sample: int) -> np.ndarray:
+    """The sample S of step t: stratum i = [floor(i d/n), floor((i+1) d/n))
+    contributes the component lo_i + below(draw_i, hi_i - lo_i), draw_i being
+    the i-th draw of the stream keyed by (seed, t) (the shared RBGS stream).
+    Ascending, one per stratum. Python integers throughout."""
+    key = rbgs_stream_key(seed, t, 0)
+    out = np.empty(n_sample, np.int64)
+    for i in range(n_sample):
+        lo = i * d // n_sample
+        hi = (i + 1) * d // n_sample
+        out[i] = lo + below(rbgs_draw(key, i), hi - lo)
+    return out
+
+
+def approx_top_s_support(x: np.ndarray, sample: np.ndarray, r: int, limit: int):
+    """Support of the approximate top-s (Sec. 5.1) and its threshold key:
+    theta = the r-th largest magnitude key among x[sample]; every component
+    whose key is >= theta is sent, unless more than `limit` are, in which case
+    the exact top-`limit` is. Returned in ascending index order."""
+    key = magnitude_key(x)
+    sampled = np.sort(key[sample])[::-1]
+    theta = int(sampled[r - 1])
+    support = np.flatnonzero(key >= U32(theta))
+    if support.size > limit:
+        support = top_s_support(x, limit)
+    return support, theta
+
+
 def rbgs_support(blocks: np.ndarray, B: int, d: int) -> np.ndarray:
     """Coordinates covered by the chosen blocks, ascending."""
     if blocks.size == 0:
@@ -153,7 +213,10 @@ def rbgs_support(blocks: np.ndarray, B: int, d: int) -> np.ndarray:
 class StepResult:
     """What one step produced (kept for the tests)."""
 
-    def __init__(self, e_half, supports, values, w_next, blocks, stats):
+    def __init__(self, e_half, supports, values, w_next, blocks, stats, sample=None,
+                 thresholds=None):
+        self.sample = sample          # approximate top-s: the sampled positions S
+        self.thresholds = thresholds  # approximate top-s: theta's key per worker
         self.e_half = e_half          # e_{t+1/2,k}, float32 [K, d]
         self.supports = supports      # list of K int64 index arrays (ascending)
         self.values = values          # list of K float32 arrays: C(e_{t+1/2,k}) on its support
@@ -176,7 +239,7 @@ class GMC:
             raise ValueError("eta must be > 0")
         if not 0.0 < ratio <= 1.0:
             raise ValueError("ratio must be in (0, 1]")
-        if compressor not in (TOPK, RBGS):
+        if compressor not in (TOPK, RBGS, TOPK_APPROX):
             raise ValueError("unknown compressor")
         self.d, self.K = d, K
         self.beta = F32(beta)
@@ -187,6 +250,11 @@ class GMC:
         self.per_worker = per_worker
         if compressor == TOPK:
             self.s = topk_count(d, ratio)
+        elif compressor == TOPK_APPROX:
+            self.s = topk_count(d, ratio)
+            self.n_sample = approx_sample_size(d)
+            self.r_sample = approx_rank(self.n_sample, ratio)
+            self.limit = approx_limit(d, ratio)
         else:
             if block < 1:
                 raise ValueError("block must be >= 1")
@@ -234,9 +302,15 @@ class GMC:
         e_half = (self.e + g) - momentum
 
         # workers: C(e_{t+1/2,k}) -- its support and values
-        blocks = None
+        blocks = sample = thresholds = None
         if self.compressor == TOPK:
             supports = [top_s_support(e_half[k], self.s) for k in range(K)]
+        elif self.compressor == TOPK_APPROX:
+            sample = approx_sample_positions(self.seed, self.t, self.d, self.n_sample)
+            picked = [approx_top_s_support(e_half[k], sample, self.r_sample, self.limit)
+                      for k in range(K)]
+            supports = [p[0] for p in picked]
+            thresholds = [p[1] for p in picked]
         else:
             blocks = self._blocks()
             per_stream = [rbgs_support(b, self.B, self.d) for b in blocks]
@@ -269,7 +343,7 @@ class GMC:
 
         self.w_prev, self.w, self.e = self.w, w_next, e_next
         self.t += 1
-        return StepResult(e_half, supports, values, w_next, blocks, stats)
+        return StepResult(e_half, supports, values, w_next, blocks, stats, sample, thresholds)
 
     def worker_params(self, k: int) -> np.ndarray:
         """GMC+ detached point of worker k: w_{t,k} = w_t - lambda*eta*e_{t,k}."""

@@ -17,7 +17,7 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle import GMC, RBGS, TOPK
+from oracle import GMC, RBGS, TOPK, TOPK_APPROX
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 U = 2.0 ** -24  # unit roundoff of fp32
@@ -127,7 +127,7 @@ def test_p2_constant_gradient_against_closed_form():
 # P3: C(v) + e = v exactly, for every worker, coordinate and step (Alg. 1)
 # ---------------------------------------------------------------------------
 
-@pytest.mark.parametrize("compressor", [TOPK, RBGS])
+@pytest.mark.parametrize("compressor", [TOPK, RBGS, TOPK_APPROX])
 def test_p3_exact_split(compressor):
     rng = np.random.default_rng(3)
     d, K, T = 1000, 4, 12
@@ -256,7 +256,7 @@ def _update_rule_residual(o, grads):
         w_prev = w_t
 
 
-@pytest.mark.parametrize("compressor", [TOPK, RBGS])
+@pytest.mark.parametrize("compressor", [TOPK, RBGS, TOPK_APPROX])
 def test_p5_update_rule(compressor):
     rng = np.random.default_rng(5)
     d, K, T = 600, 4, 30
@@ -266,7 +266,7 @@ def test_p5_update_rule(compressor):
         np.testing.assert_array_less(np.abs(lhs - rhs), budget + 1e-30)
 
 
-@pytest.mark.parametrize("compressor", [TOPK, RBGS])
+@pytest.mark.parametrize("compressor", [TOPK, RBGS, TOPK_APPROX])
 def test_p6_lemma1_z_sequence(compressor):
     """z_t = w_t + beta/(1-beta)(w_t - w_{t-1}) - eta/(1-beta) ebar_t obeys
     z_{t+1} = z_t - eta/(1-beta) gbar_t for any compressor (Lemma 1)."""
@@ -287,7 +287,7 @@ def test_p6_lemma1_z_sequence(compressor):
 # P6b, P7: GMC+ (Alg. 2) -- the mean-iterate recursion and lambda = 0
 # ---------------------------------------------------------------------------
 
-@pytest.mark.parametrize("compressor", [RBGS, TOPK])
+@pytest.mark.parametrize("compressor", [RBGS, TOPK, TOPK_APPROX])
 def test_p6b_gmcplus_mean_iterate(compressor):
     """With wbar_t = mean_k w_{t,k} (the detached points), Sec. 4's
     zbar_t = wbar_t + beta/(1-beta)(wbar_t - wbar_{t-1})
@@ -423,6 +423,125 @@ def test_rcc_dense_pairs():
     for _ in range(4):
         o.step((rng.standard_normal((K, d)) + 5.0).astype(np.float32))
     assert o.rcc() == 2.0
+
+
+# ---------------------------------------------------------------------------
+# Approximate top-s (Sec. 5.1): sample, threshold, selection
+# ---------------------------------------------------------------------------
+
+def test_approx_sizes():
+    """|S| = d/100 and r = |S|/1024 at the paper's ratio s/d = 1/1024."""
+    d = 102_400 * 13
+    n = oracle.approx_sample_size(d)
+    assert n == d // 100 == 13_312
+    assert oracle.approx_rank(n, 1 / 1024) == 13
+    assert oracle.approx_sample_size(99) == 1 and oracle.approx_rank(1, 1 / 1024) == 1
+    assert oracle.approx_limit(138_357_544, 0.001) == 4 * 138_357 + 4096
+    assert oracle.approx_limit(1000, 0.001) == 1000
+
+
+def test_approx_sample_positions_from_the_generator():
+    """One position per stratum, at the offset the published generator's
+    outputs give (the stream's draws are SplitMix64 outputs from its key)."""
+    for d, n, seed, t in ((1000, 10, 0, 0), (1_000_003, 10_000, 99, 7), (77, 1, 5, 3), (100, 1, 0, 1)):
+        pos = oracle.approx_sample_positions(seed, t, d, n)
+        key = oracle.rbgs_stream_key(seed, t, 0)
+        draws = oracle.splitmix64_sequence(key, n)
+        assert pos.size == n
+        for i in range(n):
+            lo, hi = i * d // n, (i + 1) * d // n
+            assert lo <= pos[i] < hi
+            assert pos[i] == lo + (((draws[i] >> 32) * (hi - lo)) >> 32)
+    a = oracle.approx_sample_positions(1, 0, 10_000, 100)
+    assert not np.array_equal(a, oracle.approx_sample_positions(1, 1, 10_000, 100))
+    assert not np.array_equal(a, oracle.approx_sample_positions(2, 0, 10_000, 100))
+
+
+def test_approx_sample_offsets_uniform():
+    """The offset inside a stratum of 100 is uniform (chi-square over 100 cells)."""
+    counts = np.zeros(100, np.int64)
+    d, n = 100 * 4000, 4000
+    for t in range(5):
+        pos = oracle.approx_sample_positions(31, t, d, n)
+        np.add.at(counts, pos - np.arange(n) * 100, 1)
+    expected = counts.sum() / 100
+    chi2 = float(((counts - expected) ** 2 / expected).sum())
+    assert chi2 < 180.0  # 99 degrees of freedom; p < 1e-5 beyond this
+
+
+def _brute_approx(x, sample, r, limit):
+    mags = sorted((abs(float(x[p])) for p in sample), reverse=True)
+    theta = mags[r - 1]
+    sup = [j for j in range(x.size) if abs(float(x[j])) >= theta]
+    if len(sup) > limit:
+        sup = sorted(sorted(range(x.size), key=lambda j: (-abs(float(x[j])), j))[:limit])
+    return np.array(sup, np.int64)
+
+
+def test_approx_brute_force():
+    """Theta and the support against a plain loop over |x| (ties, signed
+    zeros and the exact top-M beyond the limit included)."""
+    rng = np.random.default_rng(12)
+    for case, (x, _) in enumerate(_tiny_inputs(rng, 3_000)):
+        d = x.size
+        n = int(rng.integers(1, d + 1))
+        sample = np.sort(rng.choice(d, size=n, replace=False))
+        r = int(rng.integers(1, n + 1))
+        limit = int(rng.integers(1, d + 1)) if case % 3 == 0 else d
+        got, theta = oracle.approx_top_s_support(x, sample, r, limit)
+        np.testing.assert_array_equal(got, _brute_approx(x, sample, r, limit))
+        mags = sorted((abs(float(x[p])) for p in sample), reverse=True)
+        assert abs(float(np.array([theta], np.uint32).view(np.float32)[0])) == mags[r - 1]
+
+
+def test_approx_threshold_properties():
+    """A threshold set: everything sent is at least as large as everything
+    kept back, and at least r sampled components are sent (below the limit)."""
+    rng = np.random.default_rng(13)
+    for _ in range(200):
+        d = int(rng.integers(200, 5000))
+        x = (rng.standard_normal(d) * np.exp(rng.uniform(-3, 3, d))).astype(np.float32)
+        n = oracle.approx_sample_size(d)
+        r = oracle.approx_rank(n, 0.05)
+        sample = oracle.approx_sample_positions(int(rng.integers(0, 2 ** 63)), 0, d, n)
+        S, _ = oracle.approx_top_s_support(x, sample, r, d)
+        keep = np.zeros(d, bool)
+        keep[S] = True
+        a = np.abs(x.astype(np.float64))
+        if not keep.all():
+            assert a[keep].min() >= a[~keep].max()
+        assert np.count_nonzero(keep[sample]) >= r
+
+
+def test_approx_count_near_ratio():
+    """On Gaussian data the number sent is ratio*d up to the sample's spread
+    (about 1/sqrt(r)): within 40% per draw, within 8% on average."""
+    rng = np.random.default_rng(14)
+    d, ratio = 1 << 20, 0.01
+    n = oracle.approx_sample_size(d)
+    r = oracle.approx_rank(n, ratio)
+    assert r == 104
+    rel = []
+    for t in range(20):
+        x = rng.standard_normal(d).astype(np.float32)
+        S, _ = oracle.approx_top_s_support(x, oracle.approx_sample_positions(3, t, d, n), r, d)
+        rel.append(S.size / (ratio * d))
+    assert all(0.6 < q < 1.4 for q in rel)
+    assert abs(np.mean(rel) - 1.0) < 0.08
+
+
+def test_approx_limit_takes_exact_top():
+    """All-zero accumulators: theta is the zero key, every component reaches
+    it, and the limit leaves the M lowest indices (ties to the lower index)."""
+    d, K = 20_000, 2
+    o = GMC(d, K, beta=0.0, eta=0.1, compressor=TOPK_APPROX, ratio=0.001)
+    assert o.limit == 4 * 20 + 4096
+    o.set_params(np.zeros(d, np.float32))
+    r = o.step(np.zeros((K, d), np.float32))
+    for k in range(K):
+        np.testing.assert_array_equal(r.supports[k], np.arange(o.limit))
+        assert r.thresholds[k] == 0
+    assert r.stats["pairs"] == K * o.limit and r.stats["nnz"] == 0
 
 
 # ---------------------------------------------------------------------------
