@@ -5,6 +5,7 @@ Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU baseline
 computes and which passages of the paper each part follows.
 """
 from .gmc_oracle import (GMC, RBGS, TOPK, TOPK_APPROX, approx_limit, approx_rank,  # noqa: F401
+                         approx_runs,
                          approx_sample_positions, approx_sample_size, approx_top_s_support,
                          below, floyd_blocks, magnitude_key, rbgs_draw, rbgs_stream_key,
                          rbgs_support, splitmix64_mix, splitmix64_sequence, top_s_support,

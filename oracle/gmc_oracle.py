@@ -43,10 +43,12 @@ Readings where the paper is silent:
     (Steele, Lea & Flood, OOPSLA 2014) keyed by (seed, t) -- or (seed, t, k)
     in the per-worker mode -- with multiply-shift range reduction;
   * the residual at a sent coordinate is +0 exactly (v - v for finite v);
-  * approximate top-s: |S| = max(1, floor(d/100)); S is drawn afresh each
-    step, the same for all workers, one component from each of |S| strata
-    [floor(i d/|S|), floor((i+1) d/|S|)), picked by the i-th draw of the
-    SplitMix64 stream keyed by (seed, t) with multiply-shift reduction;
+  * approximate top-s: S is drawn afresh each step, the same for all
+    workers, as n = max(1, floor(d/800)) runs of 8 consecutive components
+    (|S| = 8n, about d/100), one run per stratum [floor(i d/n),
+    floor((i+1) d/n)), starting at a multiple of 8 inside it picked by the
+    i-th draw of the SplitMix64 stream keyed by (seed, t) with
+    multiply-shift reduction (d < 8: S = [0, d));
     theta is the r-th largest sampled magnitude key, r = max(1,
     floor(ratio |S|)); a component is sent iff its key is >= theta's; when
     more than M = min(d, 4 s + 4096) components reach theta (s the nominal
@@ -153,9 +155,17 @@ def floyd_blocks(key: int, nb: int, m: int) -> np.ndarray:
     return np.array(sorted(chosen), np.int64)
 
 
+APPROX_RUN = 8  # consecutive components per run of the sample
+
+
+def approx_runs(d: int) -> int:
+    """Runs of the sample: max(1, floor(d/800)), so that |S| is about d/100."""
+    return max(1, d // (APPROX_SAMPLE_DIV * APPROX_RUN))
+
+
 def approx_sample_size(d: int) -> int:
-    """|S| = max(1, floor(d/100)), the sample of the approximate top-s (Sec. 5.1)."""
-    return max(1, d // APPROX_SAMPLE_DIV)
+    """|S| = 8 * runs (all of [0, d) when d < 8), about d/100 (Sec. 5.1)."""
+    return d if d < APPROX_RUN else APPROX_RUN * approx_runs(d)
 
 
 def approx_rank(n_sample: int, ratio: float) -> int:
@@ -170,17 +180,24 @@ def approx_limit(d: int, ratio: float) -> int:
     return min(d, 4 * topk_count(d, ratio) + 4096)
 
 
-def approx_sample_positions(seed: int, t: int, d: int, n_sample: int) -> np.ndarray:
-    """The sample S of step t: stratum i = [floor(i d/n), floor((i+1) d/n))
-    contributes the component lo_i + below(draw_i, hi_i - lo_i), draw_i being
-    the i-th draw of the stream keyed by (seed, t) (the shared RBGS stream).
-    Ascending, one per stratum. Python integers throughout."""
+def approx_sample_positions(seed: int, t: int, d: int) -> np.ndarray:
+    """The sample S of step t, ascending. Stratum i = [floor(i d/n),
+    floor((i+1) d/n)) of the n runs contributes the 8 components from
+    a_i + 8 * below(draw_i, m_i), where a_i is lo_i rounded up to a multiple of
+    8, m_i the number of whole runs of 8 from a_i inside the stratum, and
+    draw_i the i-th draw of the stream keyed by (seed, t) (the shared RBGS
+    stream). d < 8: all of [0, d). Python integers throughout."""
+    if d < APPROX_RUN:
+        return np.arange(d, dtype=np.int64)
+    n = approx_runs(d)
     key = rbgs_stream_key(seed, t, 0)
-    out = np.empty(n_sample, np.int64)
-    for i in range(n_sample):
-        lo = i * d // n_sample
-        hi = (i + 1) * d // n_sample
-        out[i] = lo + below(rbgs_draw(key, i), hi - lo)
+    out = np.empty(APPROX_RUN * n, np.int64)
+    for i in range(n):
+        lo, hi = i * d // n, (i + 1) * d // n
+        a = -(-lo // APPROX_RUN) * APPROX_RUN
+        m = (hi - a) // APPROX_RUN
+        start = a + APPROX_RUN * below(rbgs_draw(key, i), m)
+        out[APPROX_RUN * i: APPROX_RUN * (i + 1)] = np.arange(start, start + APPROX_RUN)
     return out
 
 
@@ -306,7 +323,7 @@ class GMC:
         if self.compressor == TOPK:
             supports = [top_s_support(e_half[k], self.s) for k in range(K)]
         elif self.compressor == TOPK_APPROX:
-            sample = approx_sample_positions(self.seed, self.t, self.d, self.n_sample)
+            sample = approx_sample_positions(self.seed, self.t, self.d)
             picked = [approx_top_s_support(e_half[k], sample, self.r_sample, self.limit)
                       for k in range(K)]
             supports = [p[0] for p in picked]

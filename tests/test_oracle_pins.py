@@ -430,40 +430,51 @@ def test_rcc_dense_pairs():
 # ---------------------------------------------------------------------------
 
 def test_approx_sizes():
-    """|S| = d/100 and r = |S|/1024 at the paper's ratio s/d = 1/1024."""
+    """|S| is about d/100 in runs of 8 (|S| = 8 floor(d/800)); r = ratio |S|,
+    |S|/1024 at the paper's ratio s/d = 1/1024 (Sec. 5.1)."""
     d = 102_400 * 13
     n = oracle.approx_sample_size(d)
-    assert n == d // 100 == 13_312
+    assert n == 8 * (d // 800) == 13_312
+    assert abs(n - d / 100) <= 8
     assert oracle.approx_rank(n, 1 / 1024) == 13
-    assert oracle.approx_sample_size(99) == 1 and oracle.approx_rank(1, 1 / 1024) == 1
+    assert oracle.approx_sample_size(799) == 8 and oracle.approx_sample_size(5) == 5
+    assert oracle.approx_rank(8, 1 / 1024) == 1
     assert oracle.approx_limit(138_357_544, 0.001) == 4 * 138_357 + 4096
     assert oracle.approx_limit(1000, 0.001) == 1000
 
 
 def test_approx_sample_positions_from_the_generator():
-    """One position per stratum, at the offset the published generator's
-    outputs give (the stream's draws are SplitMix64 outputs from its key)."""
-    for d, n, seed, t in ((1000, 10, 0, 0), (1_000_003, 10_000, 99, 7), (77, 1, 5, 3), (100, 1, 0, 1)):
-        pos = oracle.approx_sample_positions(seed, t, d, n)
+    """One run of 8 per stratum, starting on a multiple of 8 at the offset the
+    published generator's outputs give (the stream's draws are SplitMix64
+    outputs from its key)."""
+    for d, seed, t in ((1000, 0, 0), (1_000_003, 99, 7), (8_000, 5, 3), (15, 0, 1), (805, 2, 2)):
+        pos = oracle.approx_sample_positions(seed, t, d)
+        n = oracle.approx_runs(d)
         key = oracle.rbgs_stream_key(seed, t, 0)
         draws = oracle.splitmix64_sequence(key, n)
-        assert pos.size == n
+        assert pos.size == oracle.approx_sample_size(d) == 8 * n
         for i in range(n):
             lo, hi = i * d // n, (i + 1) * d // n
-            assert lo <= pos[i] < hi
-            assert pos[i] == lo + (((draws[i] >> 32) * (hi - lo)) >> 32)
-    a = oracle.approx_sample_positions(1, 0, 10_000, 100)
-    assert not np.array_equal(a, oracle.approx_sample_positions(1, 1, 10_000, 100))
-    assert not np.array_equal(a, oracle.approx_sample_positions(2, 0, 10_000, 100))
+            run = pos[8 * i: 8 * i + 8]
+            a = -(-lo // 8) * 8
+            m = (hi - a) // 8
+            assert m >= 1 and run[0] % 8 == 0 and lo <= run[0] and run[-1] < hi
+            assert run[0] == a + 8 * (((draws[i] >> 32) * m) >> 32)
+            np.testing.assert_array_equal(run, np.arange(run[0], run[0] + 8))
+    np.testing.assert_array_equal(oracle.approx_sample_positions(3, 0, 5), np.arange(5))
+    a = oracle.approx_sample_positions(1, 0, 100_000)
+    assert not np.array_equal(a, oracle.approx_sample_positions(1, 1, 100_000))
+    assert not np.array_equal(a, oracle.approx_sample_positions(2, 0, 100_000))
 
 
 def test_approx_sample_offsets_uniform():
-    """The offset inside a stratum of 100 is uniform (chi-square over 100 cells)."""
+    """The run's slot inside a stratum of 100 slots is uniform (chi-square
+    over 100 cells)."""
     counts = np.zeros(100, np.int64)
-    d, n = 100 * 4000, 4000
+    d = 800 * 4000
     for t in range(5):
-        pos = oracle.approx_sample_positions(31, t, d, n)
-        np.add.at(counts, pos - np.arange(n) * 100, 1)
+        pos = oracle.approx_sample_positions(31, t, d)[::8]
+        np.add.at(counts, (pos - np.arange(pos.size) * 800) // 8, 1)
     expected = counts.sum() / 100
     chi2 = float(((counts - expected) ** 2 / expected).sum())
     assert chi2 < 180.0  # 99 degrees of freedom; p < 1e-5 beyond this
@@ -503,7 +514,7 @@ def test_approx_threshold_properties():
         x = (rng.standard_normal(d) * np.exp(rng.uniform(-3, 3, d))).astype(np.float32)
         n = oracle.approx_sample_size(d)
         r = oracle.approx_rank(n, 0.05)
-        sample = oracle.approx_sample_positions(int(rng.integers(0, 2 ** 63)), 0, d, n)
+        sample = oracle.approx_sample_positions(int(rng.integers(0, 2 ** 63)), 0, d)
         S, _ = oracle.approx_top_s_support(x, sample, r, d)
         keep = np.zeros(d, bool)
         keep[S] = True
@@ -524,7 +535,7 @@ def test_approx_count_near_ratio():
     rel = []
     for t in range(20):
         x = rng.standard_normal(d).astype(np.float32)
-        S, _ = oracle.approx_top_s_support(x, oracle.approx_sample_positions(3, t, d, n), r, d)
+        S, _ = oracle.approx_top_s_support(x, oracle.approx_sample_positions(3, t, d), r, d)
         rel.append(S.size / (ratio * d))
     assert all(0.6 < q < 1.4 for q in rel)
     assert abs(np.mean(rel) - 1.0) < 0.08
