@@ -273,7 +273,7 @@ def run_reference(args, wl, world, rank):
 
 def config_of(wl, args):
     return {"workload": f"{wl.name}: d={wl.d:,}, K={wl.K}, {wl.compressor}"
-                        + (f" ratio {wl.ratio}" if wl.compressor == "topk"
+                        + (f" ratio {wl.ratio:.6g}" if wl.compressor != "rbgs"
                            else f" block {wl.block}, {wl.ratio:.0%} of blocks, lambda {wl.lam}")
                         + f", beta {wl.beta}, eta {wl.eta}",
             "d": wl.d, "K": wl.K, "compressor": wl.compressor, "ratio": wl.ratio,
@@ -328,7 +328,7 @@ def run_gmc(args, wl, world, rank, local):
     ms_max = max_over_ranks(ms, world, dev)
     value = wl.K * wl.d * args.steps * world / (ms_max / 1e3)
 
-    dom = "accumulate" if wl.compressor == "topk" else "rbgs_step"
+    dom = "rbgs_step" if wl.compressor == "rbgs" else "accumulate"
     p = prof.get(dom, {"ms": float("nan"), "launches": 1, "bytes": float("nan")})
     per_launch_bytes = p["bytes"] / p["launches"]
     avg_s = p["ms"] / p["launches"] / 1e3

@@ -11,8 +11,9 @@
  *   with w_{-1} = w_0 and e_{0,k} = 0.
  *   Algorithm 2 (GMC+, Sec. 4) adds the detached point
  *     w_{t+1,k} = w_{t+1} - lambda*eta*e_{t+1,k}.
- *   Compressors (Sec. 4, Sec. 5.2): exact top-s ("top-k"), and RBGS (random
- *   blocks chosen with one seed shared by all workers).
+ *   Compressors (Sec. 4, Sec. 5.1, Sec. 5.2): exact top-s ("top-k"), the
+ *   approximate top-s of Sec. 5.1 (a threshold taken from a random sample),
+ *   and RBGS (random blocks chosen with one seed shared by all workers).
  *
  * Arithmetic: fp32, one IEEE round-to-nearest-even rounding per operation in
  * the order written above: v = (e + g) - (c * (w_t - w_{t-1})), c = fl(beta/eta);
@@ -59,6 +60,17 @@ typedef struct gmc_ctx* gmc_t;
 /* Compressors C(.). */
 #define GMC_TOPK 0 /* exact top-k by magnitude, ties to the lower index (Sec. 4 top-s) */
 #define GMC_RBGS 1 /* random aligned blocks of `block` components (Sec. 4, Sec. 5.2) */
+#define GMC_TOPK_APPROX 2 /* approximate top-s (Sec. 5.1): a sample S of about d/100
+                             components -- n = max(1, floor(d/800)) runs of 8
+                             consecutive ones, one per stratum [floor(i d/n),
+                             floor((i+1) d/n)) starting on a multiple of 8 picked by
+                             the SplitMix64 stream of (seed, t), drawn afresh each
+                             step and shared by all workers (d < 8: all of [0, d)) --
+                             gives theta, the r-th largest sampled |v| with
+                             r = max(1, floor(ratio*|S|)); every component with
+                             |v| >= theta is sent (the count varies), unless more
+                             than min(d, 4 s + 4096) do (s = max(1, floor(ratio*d))):
+                             then the exact top of that many */
 
 /* Top-k selection engines; both give identical results. */
 #define GMC_SELECT_SAMPLED 0 /* default: a sampled threshold filters candidates in the one
@@ -96,8 +108,9 @@ typedef struct gmc_ctx* gmc_t;
  * Inputs of Algorithm 1 (Sec. 3.1): d parameters, K workers, momentum beta in
  * [0,1), learning rate eta > 0, compressor C; ratio in (0,1] is the kept share
  * (top-k: k = max(1, floor(ratio*d)); RBGS: m = max(1, floor(ratio*nb)) of the
- * nb = ceil(d/block) blocks); block >= 1 is the RBGS block size (ignored for
- * top-k). Requires 1 <= d < 2^31 - 2^16 and 1 <= K <= 32.
+ * nb = ceil(d/block) blocks; approximate top-s: ratio*|S| sampled components
+ * reach theta); block >= 1 is the RBGS block size (ignored otherwise).
+ * Requires 1 <= d < 2^31 - 2^16 and 1 <= K <= 32.
  * GMC+'s lambda defaults to 0 (plain GMC) for top-k and 0.5 for RBGS (Sec. 5.2
  * uses 0.5 for GMC+). Returns GMC_EINVAL, GMC_ENOMEM or GMC_ECUDA on failure,
  * with *out set to NULL. The state must be initialised with gmc_set_params.
@@ -116,14 +129,16 @@ int gmc_set_lambda(gmc_t h, float lambda);
 int gmc_set_rbgs_mode(gmc_t h, int32_t per_worker);
 
 /* gmc_set_seed -- seed of the RBGS block choice (SplitMix64 counter stream
- * keyed by (seed, t[, k]); Floyd's sampling). Default 0. */
+ * keyed by (seed, t[, k]); Floyd's sampling) and of the approximate top-s
+ * sample (the stream of (seed, t)). Default 0. */
 int gmc_set_seed(gmc_t h, uint64_t seed);
 
 /* gmc_set_eta -- change eta between steps (e.g. the cosine schedule of Sec. 5.1);
  * takes effect at the next gmc_step. */
 int gmc_set_eta(gmc_t h, float eta);
 
-/* gmc_set_select_mode -- GMC_SELECT_SAMPLED (default) or GMC_SELECT_DENSE. */
+/* gmc_set_select_mode -- GMC_SELECT_SAMPLED (default) or GMC_SELECT_DENSE (exact
+ * top-k only: GMC_EINVAL for GMC_TOPK_APPROX, which its sample defines). */
 int gmc_set_select_mode(gmc_t h, int32_t mode);
 
 /* gmc_set_detach_output -- GMC+ (Alg. 2 detach): when out_dev is not NULL, every
@@ -183,7 +198,8 @@ int gmc_get_selected(gmc_t h, int32_t k, uint32_t* idx_dev, float* val_dev,
                      int64_t capacity, int64_t* count_host, void* stream);
 
 /* gmc_selected_capacity -- the largest number of pairs one worker can send per
- * step (k for top-k, m*block for RBGS), or -1 for an invalid handle. */
+ * step (k for top-k, min(d, 4 s + 4096) for the approximate top-s, m*block for
+ * RBGS), or -1 for an invalid handle. */
 int64_t gmc_selected_capacity(gmc_t h);
 
 /* gmc_get_worker_params -- GMC+ detached point of worker k at the current step,

@@ -68,7 +68,10 @@ struct gmc_ctx {
   float* cand_val[2] = {nullptr, nullptr};
   uint2* chunk[2] = {nullptr, nullptr};
   uint32_t* mask = nullptr;
-  uint32_t* sample_pend = nullptr;  // 2 x kSampleSlots
+  uint32_t* sample_pend = nullptr;  // 3 x sample_stride
+  // sample geometry; approximate top-s: its limit and theta blocks
+  uint32_t n_sample = 0, sample_stride = 0, limit = 0;
+  int theta_blocks = 1;
   // deferred aggregation (bulk top-k pass): the last step's sent pairs are
   // summed into w by the next step's bulk pass, or by flush() when state is read
   bool agg_pending = false;
@@ -220,6 +223,13 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.bucket = h->bucket;
   A.sel_shift = h->sel_shift;
   A.sample_keys = h->sample_keys;
+  A.n_sample = h->n_sample;
+  A.sample_stride = h->sample_stride;
+  A.approx = h->compressor == GMC_TOPK_APPROX ? 1 : 0;
+  A.seed = h->seed;
+  A.t = t;
+  A.limit = h->limit;
+  A.theta_blocks = h->theta_blocks;
   A.big_tiles = h->big_tiles;
   A.g_direct = 0;
   A.regions = h->regions;
@@ -303,7 +313,8 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
   GMC_TRY(order_after_flush(h, s, true));
   GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
   unsigned long long pairs_add = 0;
-  if (h->compressor == GMC_TOPK) {
+  if (h->compressor != GMC_RBGS) {
+    const bool approx = h->compressor == GMC_TOPK_APPROX;
     TopkArgs A = topk_args(h, grads);
     A.g_direct = direct ? 1 : 0;
     A.pending = h->agg_pending ? 1 : 0;
@@ -314,7 +325,9 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
     GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
                   [&] { return launch_accumulate(A, h->grid_acc, s); }));
     h->agg_pending = false;
-    GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] { return launch_select(A, h->sel_blocks, s); }));
+    GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] {
+      return approx ? launch_select_approx(A, s) : launch_select(A, h->sel_blocks, s);
+    }));
     GMC_TRY(timed(h, GMC_KERNEL_DENSE, 0.0, s, [&] { return launch_select_dense(A, s); }));
     if (defer) {
       // the next step's sample and bulk pass apply the aggregation
@@ -329,7 +342,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
         return err != cudaSuccess ? err : launch_owner_sum(B, h->grid_agg, s);
       }));
     }
-    pairs_add = (unsigned long long)h->K * h->ksel;
+    pairs_add = approx ? 0ull : (unsigned long long)h->K * h->ksel;  // approximate: counted on the device
   } else {
     RbgsArgs A = rbgs_args(h, grads);
     A.g_direct = direct ? 1 : 0;
@@ -408,7 +421,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
   if (!finite_f(beta) || !(beta >= 0.f) || !(beta < 1.f)) return GMC_EINVAL;
   if (!finite_f(eta) || !(eta > 0.f)) return GMC_EINVAL;
   if (!std::isfinite(ratio) || !(ratio > 0.0) || !(ratio <= 1.0)) return GMC_EINVAL;
-  if (compressor != GMC_TOPK && compressor != GMC_RBGS) return GMC_EINVAL;
+  if (compressor != GMC_TOPK && compressor != GMC_RBGS && compressor != GMC_TOPK_APPROX) return GMC_EINVAL;
   if (compressor == GMC_RBGS && block < 1) return GMC_EINVAL;
   if (K > 32) return GMC_EINVAL;
 
@@ -437,7 +450,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
   if (err != cudaSuccess) return fail(err);
 
   const int64_t streams_wide = 2 * (int64_t)h->num_sms;
-  if (compressor == GMC_TOPK) {
+  if (compressor != GMC_RBGS) {
     // tiles of 4096 take the bulk-copy pass, for up to kBulkMaxK workers (its
     // shared memory grows with K); otherwise the load/store pass
     int U = K <= kBulkMaxK ? 4 : 2;
@@ -448,7 +461,20 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     h->ld = h->n_tiles * h->tile;
     const int64_t ks = std::max<int64_t>(1, (int64_t)std::floor(ratio * (double)d));
     h->ksel = (uint32_t)ks;
-    if (d <= kSampleAll) {
+    if (compressor == GMC_TOPK_APPROX) {
+      // Sec. 5.1: |S| = about d/100 sampled components (runs of 8, one per
+      // stratum of d / floor(d/800)), theta such that ratio*|S| of them reach
+      // it; at most limit = min(d, 4 s + 4096) are sent
+      h->sample_chunks = 0;
+      h->n_sample = d < 8 ? (uint32_t)d : (uint32_t)(8 * std::max<int64_t>(1, d / 800));
+      h->sample_rank = (uint32_t)std::max<int64_t>(1, (int64_t)std::floor(ratio * (double)h->n_sample));
+      h->limit = (uint32_t)std::min<int64_t>(d, 4 * ks + 4096);
+      // candidate parts: the expected count s with a 5-sigma margin of the
+      // sample's spread (relative sd 1/sqrt(r)); the dense path rewrites up to limit
+      const double r = (double)h->sample_rank;
+      const double capd = std::ceil((double)ks * (1.0 + 5.0 / std::sqrt(r))) + 4096.0;
+      h->cap = (uint32_t)std::min<double>((double)d, capd);
+    } else if (d <= kSampleAll) {
       h->sample_chunks = 0;
       h->sample_rank = h->ksel;
       h->cap = (uint32_t)d;
@@ -477,7 +503,8 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
       h->cap_region = (cap0 + 3) & ~3u;
       h->cap_part = h->cap_region;
     }
-    h->cap = (uint32_t)std::min<uint64_t>((uint64_t)h->regions * h->cap_region, 0xfffffff0ull);
+    h->cap = (uint32_t)std::min<uint64_t>(
+        std::max<uint64_t>((uint64_t)h->regions * h->cap_region, h->limit), 0xfffffff0ull);
     const int64_t per = (h->cap + 8191) / 8192;
     h->grid_agg = h->regions > 1 ? h->regions : (int)std::max<int64_t>(1, 4 * (int64_t)h->num_sms / K);
     // select passes: about 2048 expected candidates per block
@@ -485,7 +512,11 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     const int64_t want = std::max<int64_t>(1, (int64_t)(expect / 2048.0));
     h->sel_blocks = h->regions > 1 ? (int)std::min<int64_t>(h->regions, want)
                                    : (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
-    h->sample_blocks = (int)std::max<int64_t>(1, ((h->sample_chunks ? 8 * kSampleChunks : d) + 2047) / 2048);
+    if (compressor == GMC_TOPK) h->n_sample = (uint32_t)(h->sample_chunks ? 8 * kSampleChunks : d);
+    h->sample_stride = std::max<uint32_t>(kSampleSlots, (h->n_sample + 3) & ~3u);
+    h->sample_blocks = (int)std::max<int64_t>(1, ((int64_t)h->n_sample + 2047) / 2048);
+    h->theta_blocks = (int)std::max<int64_t>(1, std::min<int64_t>(2 * h->num_sms / K + 1,
+                                                                  ((int64_t)h->n_sample + 8191) / 8192));
     // relative-histogram bin width 2^sel_shift keys: near the k-th key a key
     // step of 2^23 is an octave of |v|, and a Gaussian-like tail puts about
     // 11 ln2 * k * 2^s / 2^23 candidates in one bin; aim at 2048 (the bin is
@@ -502,11 +533,11 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess ||
         (err = dalloc(h, &h->chist, (size_t)K * kRelBins)) != cudaSuccess ||
         (err = dalloc(h, &h->bucket, (size_t)K * 2 * kBucketCap)) != cudaSuccess ||
-        (err = dalloc(h, &h->sample_keys, (size_t)K * 8 * kSampleChunks)) != cudaSuccess ||
+        (err = dalloc(h, &h->sample_keys, (size_t)K * h->sample_stride)) != cudaSuccess ||
         (err = dalloc(h, &h->big_tiles, (size_t)h->n_tiles + 1)) != cudaSuccess ||
         (err = dalloc(h, &h->rcount, (size_t)K * h->regions * kChunksPerTile)) != cudaSuccess ||
         (err = dalloc(h, &h->mask, (size_t)h->ld)) != cudaSuccess ||
-        (err = dalloc(h, &h->sample_pend, (size_t)2 * kSampleSlots)) != cudaSuccess)
+        (err = dalloc(h, &h->sample_pend, (size_t)3 * h->sample_stride)) != cudaSuccess)
       return fail(err);
     if ((err = cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking)) != cudaSuccess ||
         (err = cudaEventCreateWithFlags(&h->ev_step, cudaEventDisableTiming)) != cudaSuccess ||
@@ -589,6 +620,8 @@ int gmc_set_eta(gmc_t h, float eta) {
 
 int gmc_set_select_mode(gmc_t h, int32_t mode) {
   if (!h || (mode != GMC_SELECT_SAMPLED && mode != GMC_SELECT_DENSE)) return GMC_EINVAL;
+  // the approximate top-s is defined by its sample: it has no dense engine
+  if (h->compressor == GMC_TOPK_APPROX && mode != GMC_SELECT_SAMPLED) return GMC_EINVAL;
   h->select_mode = mode;
   return GMC_OK;
 }
@@ -610,7 +643,7 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
   GMC_TRY(cudaMemcpyAsync(h->w, w0_dev, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice, s));
   GMC_TRY(cudaMemsetAsync(h->e, 0, (size_t)h->K * h->ld * sizeof(float), s));
   GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
-  if (h->compressor == GMC_TOPK) {
+  if (h->compressor != GMC_RBGS) {
     for (int p = 0; p < 2; ++p)
       GMC_TRY(cudaMemsetAsync(h->chunk[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint2), s));
     GMC_TRY(cudaMemsetAsync(h->sel, 0, (size_t)h->K * sizeof(WorkerSel), s));
@@ -685,6 +718,7 @@ int gmc_get_residual(gmc_t h, int32_t k, float* e_dev_out, void* stream) {
 
 int64_t gmc_selected_capacity(gmc_t h) {
   if (!h) return -1;
+  if (h->compressor == GMC_TOPK_APPROX) return (int64_t)h->limit;
   return h->compressor == GMC_TOPK ? (int64_t)h->ksel : h->m * h->block;
 }
 
@@ -694,9 +728,16 @@ int gmc_get_selected(gmc_t h, int32_t k, uint32_t* idx_dev, float* val_dev, int6
   if (!h->initialized || h->t == 0) return GMC_ESTATE;
   DeviceGuard g(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (h->compressor == GMC_TOPK) {
-    *count_host = h->ksel;
-    if (capacity < (int64_t)h->ksel) return GMC_EINVAL;
+  if (h->compressor != GMC_RBGS) {
+    int64_t count = h->ksel;
+    if (h->compressor == GMC_TOPK_APPROX) {  // the count varies by step: read it
+      uint32_t nsel = 0;
+      GMC_TRY(cudaMemcpyAsync(&nsel, &h->sel[k].nsel, sizeof(uint32_t), cudaMemcpyDeviceToHost, s));
+      GMC_TRY(cudaStreamSynchronize(s));
+      count = nsel;
+    }
+    *count_host = count;
+    if (capacity < count) return GMC_EINVAL;
     const TopkArgs A = topk_args_at(h, nullptr, h->t - 1);
     GMC_TRY(launch_gather_selected(A, k, idx_dev, val_dev, s));
   } else {

@@ -33,7 +33,8 @@ struct WorkerSel {
   uint32_t dense;    // 1: this worker's selection is made by the dense path
   uint32_t done[4];  // finished-block counters: the two select passes, -, the sample
   uint32_t count_bucket;  // candidates collected from the k-th key's bin
-  uint32_t pad[2];
+  uint32_t nsel;     // approximate top-s: components sent (the count varies by step)
+  uint32_t pad;
 };
 
 // Step counters (see GMC_STAT_* in gmc.h), unsigned 64-bit slots.
@@ -64,6 +65,25 @@ __device__ __forceinline__ float accumulate(float e, float g, float c, float dl)
 // fewer candidates than k, a candidate region overflowed, or too many ties.
 __device__ __forceinline__ bool needs_dense(const WorkerSel& s, uint32_t ksel, uint32_t cap) {
   return s.count < ksel || s.count > cap || s.dense != 0;
+}
+// SplitMix64 (Steele, Lea & Flood, OOPSLA 2014): output function, the key of
+// step t's stream (stream 0 = shared by all workers, k+1 = worker k), the
+// stream's i-th draw, and [0, n) from a draw's top 32 bits by multiply-shift.
+constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
+__device__ __forceinline__ uint64_t sm64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+__device__ __forceinline__ uint64_t stream_key(uint64_t seed, int64_t t, uint64_t stream) {
+  const uint64_t k1 = sm64_mix(seed + kGamma * (uint64_t)(t + 1));
+  return sm64_mix(k1 + kGamma * (stream + 1));
+}
+__device__ __forceinline__ uint64_t draw(uint64_t key, uint64_t i) {
+  return sm64_mix(key + kGamma * (i + 1));
+}
+__device__ __forceinline__ uint32_t below(uint64_t x, uint64_t n) {
+  return (uint32_t)(((x >> 32) * n) >> 32);
 }
 // Membership of a candidate in C(v): above the k-th key, or equal to it with
 // an index no larger than the last tie kept (ties go to the lower index).

@@ -39,8 +39,19 @@ struct TopkArgs {
   uint32_t cap_part;         // slots per warp part (a multiple of 32: whole 128-byte lines)
   uint32_t* rcount;          // K x regions x kChunksPerTile: candidates written in each part
   uint32_t sample_rank;      // rank of the sampled threshold
-  int sample_chunks;         // 0 = sample every element
+  int sample_chunks;         // 0 = sample every element (or the approximate top-s sample)
   int sample_blocks;         // blocks per worker of the sample kernel
+  uint32_t n_sample;         // sampled positions per worker
+  uint32_t sample_stride;    // per-worker stride of sample_keys; offset of the delta half of sample_pend
+  // Approximate top-s (Sec. 5.1): the sample is one position per stratum of
+  // d / n_sample drawn from the shared SplitMix64 stream of (seed, t); theta
+  // is the exact sample_rank-th largest sampled key and C(v) = {key >= theta},
+  // or the exact top-`limit` when more than `limit` components reach theta.
+  int approx;
+  uint64_t seed;
+  int64_t t;
+  uint32_t limit;
+  int theta_blocks;          // blocks per worker of k_sample_theta
   int has_prev;              // a previous step exists (t > 0)
   int dense_mode;            // GMC_SELECT_DENSE
   WorkerSel* sel;            // K entries
@@ -48,7 +59,7 @@ struct TopkArgs {
   uint32_t* chist;           // K x kRelBins: the candidates' relative histogram (zeroed by the sample)
   uint32_t* bucket;          // K x 2*kBucketCap: keys, then indices of the k-th key's bin
   int sel_shift;             // log2 of the relative-histogram bin width (in keys)
-  uint32_t* sample_keys;     // K x 8*kSampleChunks
+  uint32_t* sample_keys;     // K x sample_stride
   uint32_t* big_tiles;       // [0]: count, then tile ids left to the block aggregate
   uint32_t* cand_idx;        // current chunks: K x cap
   float* cand_val;
@@ -63,8 +74,9 @@ struct TopkArgs {
   // streams every coordinate anyway (see k_accumulate_bulk).
   int pending;               // the previous step's aggregation is still to be applied
   float a_prev;              // fl(eta/K) of that step
-  uint32_t* sample_pend;     // 2 x kSampleSlots: its senders' mask and w_{t+1} - w_t at the
-                             // sampled coordinates (k_sample_pending, for k_sample)
+  uint32_t* sample_pend;     // 3 x sample_stride: its senders' mask and w_{t+1} - w_t at the
+                             // sampled coordinates (k_sample_pending, for k_sample); the
+                             // approximate top-s adds the coordinates
   Counters* total_ctr;       // running totals: the deferred aggregation counts there
   Counters* step_ctr;
   unsigned* status;
@@ -122,6 +134,8 @@ struct DetachArgs {
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s);
+// Approximate top-s: T = theta, every tie kept, the count; or the dense path.
+cudaError_t launch_select_approx(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s);
 constexpr int kBulkTile = 4096;  // tile of the bulk-copy accumulate pass (k_accumulate_bulk)
 constexpr int kBulkMaxK = 16;    // workers the bulk-copy pass takes (its shared memory grows with K)

@@ -16,27 +16,7 @@
 namespace gmc {
 namespace {
 
-constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
 constexpr int kPickSmemWords = 12288;  // bitmap words kept in shared memory
-
-// SplitMix64 output function (Steele, Lea & Flood, OOPSLA 2014).
-__device__ __forceinline__ uint64_t sm64_mix(uint64_t z) {
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
-// Key of step t's block-choice stream; stream 0 = shared, k+1 = worker k.
-__device__ __forceinline__ uint64_t stream_key(uint64_t seed, int64_t t, uint64_t stream) {
-  const uint64_t k1 = sm64_mix(seed + kGamma * (uint64_t)(t + 1));
-  return sm64_mix(k1 + kGamma * (stream + 1));
-}
-__device__ __forceinline__ uint64_t draw(uint64_t key, uint64_t i) {
-  return sm64_mix(key + kGamma * (i + 1));
-}
-// [0, n) from the top 32 bits of a draw (multiply-shift).
-__device__ __forceinline__ uint32_t below(uint64_t x, uint64_t n) {
-  return (uint32_t)(((x >> 32) * n) >> 32);
-}
 
 __device__ __forceinline__ float4 load_g4(const float* __restrict__ g, int64_t j, int64_t d,
                                           int mode) {

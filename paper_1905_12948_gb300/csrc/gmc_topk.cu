@@ -61,13 +61,26 @@ __device__ __forceinline__ uint32_t warp_excl_scan(uint32_t x, uint32_t* total) 
   return incl - x;
 }
 
-// Sampled coordinate of slot i: the sample takes 8 consecutive coordinates
-// from (c * d / chunks) rounded down to a multiple of 8, c = 0 .. chunks-1
-// (every coordinate when chunks = 0).
-__device__ __forceinline__ int64_t sample_coord(const TopkArgs& A, int i) {
+// Sampled coordinate of slot i. Exact top-k: 8 consecutive coordinates from
+// (c * d / chunks) rounded down to a multiple of 8, c = 0 .. chunks-1 (every
+// coordinate when chunks = 0). Approximate top-s (Sec. 5.1): run i/8 of the
+// n = n_sample/8 runs of 8 consecutive coordinates, one per stratum
+// [r d / n, (r+1) d / n), starting on a multiple of 8 inside it at the slot
+// the r-th draw of the step's shared stream `key` picks (d < 8: slot i).
+__device__ __forceinline__ int64_t sample_coord(const TopkArgs& A, uint64_t key, int i) {
+  if (A.approx) {
+    if (A.d < 8) return i;
+    const uint64_t n = A.n_sample >> 3, d = (uint64_t)A.d, run = (uint64_t)i >> 3;
+    const uint64_t lo = run * d / n, hi = (run + 1) * d / n;
+    const uint64_t a = (lo + 7) & ~uint64_t(7);
+    return (int64_t)(a + 8 * (uint64_t)below(draw(key, run), (hi - a) >> 3) + (i & 7));
+  }
   if (!A.sample_chunks) return i;
   const int64_t ch = i >> 3;
   return ((ch * A.d / A.sample_chunks) & ~int64_t(7)) + (i & 7);
+}
+__device__ __forceinline__ uint64_t sample_key(const TopkArgs& A) {
+  return A.approx ? stream_key(A.seed, A.t, 0) : 0ull;
 }
 
 // The previous step's aggregation at the sampled coordinates, when it is
@@ -75,7 +88,9 @@ __device__ __forceinline__ int64_t sample_coord(const TopkArgs& A, int i) {
 // workers whose value there (still in e: it was their accumulator) was
 // selected; w still holds w_t. For slot i: the senders' mask, and
 // w_{t+1}[j] - w_t[j] -- their values summed in ascending worker order from
-// +0 (Alg. 1).
+// +0 (Alg. 1). The approximate top-s runs it every step: it also stores each
+// slot's coordinate, and the step's w_t - w_{t-1} there (from dlt when no
+// aggregation is pending), for k_sample to read in order.
 __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
   __shared__ uint32_t Tp[kMaxK], tip[kMaxK];
   for (int kk = threadIdx.x; kk < A.K; kk += blockDim.x) {  // the previous step's selections
@@ -83,29 +98,35 @@ __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
     tip[kk] = A.sel[kk].t_idx;
   }
   __syncthreads();
-  const int n_s = A.sample_chunks ? A.sample_chunks * 8 : (int)A.d;
+  const int n_s = (int)A.n_sample;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n_s) return;
-  const int64_t j = sample_coord(A, i);
-  float x[kMaxK];
-#pragma unroll
-  for (int b = 0; b < kMaxK; ++b) x[b] = b < A.K ? __ldcg(A.e + (int64_t)b * A.ld + j) : 0.f;
-  float sum = 0.f;
+  const int64_t j = sample_coord(A, sample_key(A), i);
   uint32_t m = 0;
+  float dd = 0.f;
+  if (A.pending) {
+    float x[kMaxK];
 #pragma unroll
-  for (int b = 0; b < kMaxK; ++b) {
-    if (b < A.K && selected(mag_key(x[b]), (uint32_t)j, Tp[b], tip[b])) {
-      sum = __fadd_rn(sum, x[b]);
-      m |= 1u << b;
+    for (int b = 0; b < kMaxK; ++b) x[b] = b < A.K ? __ldcg(A.e + (int64_t)b * A.ld + j) : 0.f;
+    float sum = 0.f;
+#pragma unroll
+    for (int b = 0; b < kMaxK; ++b) {
+      if (b < A.K && selected(mag_key(x[b]), (uint32_t)j, Tp[b], tip[b])) {
+        sum = __fadd_rn(sum, x[b]);
+        m |= 1u << b;
+      }
+    }
+    if (m) {
+      const float wo = A.w[j];
+      dd = __fsub_rn(__fsub_rn(wo, __fmul_rn(A.a_prev, sum)), wo);
     }
   }
-  float dd = 0.f;
-  if (m) {
-    const float wo = A.w[j];
-    dd = __fsub_rn(__fsub_rn(wo, __fmul_rn(A.a_prev, sum)), wo);
+  if (A.approx) {
+    if (!m) dd = A.dlt[j];
+    A.sample_pend[2 * A.sample_stride + i] = (uint32_t)j;
   }
   A.sample_pend[i] = m;
-  A.sample_pend[kSampleSlots + i] = __float_as_uint(dd);
+  A.sample_pend[A.sample_stride + i] = __float_as_uint(dd);
 }
 
 // Bin of a candidate key in the relative histogram: (key - theta) >> shift,
@@ -140,8 +161,9 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   }
   const float* ek = A.e + (int64_t)k * A.ld;
   const float* gk = A.grads + (int64_t)k * A.d;
-  uint32_t* keys = A.sample_keys + (int64_t)k * (8 * kSampleChunks);
-  const int n_s = A.sample_chunks ? A.sample_chunks * 8 : (int)A.d;
+  uint32_t* keys = A.sample_keys + (int64_t)k * A.sample_stride;
+  const int n_s = (int)A.n_sample;
+  const uint64_t skey = sample_key(A);
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0;
   __syncthreads();
   const int per = (n_s + gridDim.x - 1) / gridDim.x;
@@ -153,15 +175,21 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
     for (int q = 0; q < 8; ++q) {
       const int i = i0 + q * blockDim.x + threadIdx.x;
       ev[q] = gv[q] = dv[q] = 0.f;
-      if (i < i_hi) {
-        const int64_t j = sample_coord(A, i);
+      if (i < i_hi && A.approx) {  // coordinate, senders and w_t - w_{t-1} from k_sample_pending
+        const int64_t j = A.sample_pend[2 * A.sample_stride + i];
+        const uint32_t m = A.sample_pend[i];
+        ev[q] = ((m >> k) & 1u) ? 0.f : ek[j];
+        gv[q] = gk[j];
+        dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
+      } else if (i < i_hi) {
+        const int64_t j = sample_coord(A, skey, i);
         ev[q] = ek[j];
         gv[q] = gk[j];
         dv[q] = A.dlt[j];
         if (A.pending) {  // as if the previous step's aggregation were applied at j
           const uint32_t m = A.sample_pend[i];
           if ((m >> k) & 1u) ev[q] = 0.f;
-          if (m) dv[q] = __uint_as_float(A.sample_pend[kSampleSlots + i]);
+          if (m) dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
         }
       }
     }
@@ -181,6 +209,7 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
     if (hist[b]) atomicAdd(&gh[b], hist[b]);
+  if (A.approx) return;  // k_sample_theta fixes theta exactly
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[3], 1u) == gridDim.x - 1) ? 1u : 0u;
@@ -231,6 +260,149 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
     S.theta = min((b1 << 20) | (s_bin << 10), 0x7f800000u);
     S.count = 0;
     S.dense = 0;
+  }
+}
+
+// Radix select in shared memory: the r-th largest of n values (digits 11/10/10).
+__device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, uint32_t r,
+                                                uint32_t* h, uint32_t* ws, uint32_t* s_bin,
+                                                uint32_t* s_rank, uint32_t* rank_out) {
+  uint32_t prefix = 0;
+  for (int pass = 0; pass < 3; ++pass) {
+    const int nbins = pass == 0 ? 2048 : 1024;
+    const int shift = pass == 0 ? 20 : (pass == 1 ? 10 : 0);
+    for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
+    if (threadIdx.x == 0) {
+      *s_bin = 0;
+      *s_rank = 0;
+    }
+    __syncthreads();
+    for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
+      const uint32_t i = i0 + threadIdx.x;
+      int bin = -1;
+      if (i < n) {
+        const uint32_t v = x[i];
+        if (pass == 0 || (v >> (shift + 10)) == prefix) bin = (int)((v >> shift) & (uint32_t)(nbins - 1));
+      }
+      warp_hist_add(h, bin);
+    }
+    __syncthreads();
+    block_find_from_top(h, nbins, r, ws, s_bin, s_rank);
+    prefix = pass == 0 ? *s_bin : ((prefix << 10) | *s_bin);
+    r = *s_rank;
+    __syncthreads();
+  }
+  *rank_out = r;
+  return prefix;
+}
+
+// ---------------------------------------------------------------------------
+// Approximate top-s (Sec. 5.1): theta is the exact r-th largest sampled key.
+// Every block finds, from the sample's first-digit histogram, the bin that
+// holds it and collects that bin's keys from its slice of the sample (128 a
+// round, one bucket reservation); the last block ranks the bucket in shared
+// memory. A bin too crowded for the bucket is resolved by the last block's
+// two remaining radix digits over the whole sample.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_sample_theta(TopkArgs A) {
+  extern __shared__ __align__(16) uint32_t fin[];  // kBucketCap keys
+  __shared__ uint32_t h[kHistBins];
+  __shared__ uint32_t ws[32];
+  __shared__ uint32_t s_last, s_bin, s_rank, s_n;
+  const int k = blockIdx.y;
+  WorkerSel& S = A.sel[k];
+  uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) h[b] = __ldcg(&gh[b]);
+  if (threadIdx.x == 0) {
+    s_bin = 0;
+    s_rank = 0;
+  }
+  __syncthreads();
+  const uint32_t n_s = A.n_sample;
+  const uint32_t r = A.sample_rank < n_s ? A.sample_rank : n_s;
+  block_find_from_top(h, kHistBins, r, ws, &s_bin, &s_rank);
+  const uint32_t b1 = s_bin, r1 = s_rank;
+  const uint32_t* keys = A.sample_keys + (int64_t)k * A.sample_stride;
+  uint32_t* bk = A.bucket + (int64_t)k * 2 * kBucketCap;
+  const int lane = threadIdx.x & 31;
+  const uint32_t lt = lanemask_lt();
+  const uint32_t per = (n_s + gridDim.x - 1) / gridDim.x;
+  const uint32_t i_lo = min(n_s, blockIdx.x * per), i_hi = min(n_s, i_lo + per);
+  for (uint32_t i0 = i_lo + (threadIdx.x >> 5) * 128; i0 < i_hi; i0 += kWarps * 128) {
+    uint32_t key[4], m[4], n = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t i = i0 + q * 32 + lane;
+      key[q] = i < i_hi ? __ldcg(keys + i) : 0u;
+      m[q] = __ballot_sync(0xffffffffu, i < i_hi && (key[q] >> 20) == b1);
+      n += __popc(m[q]);
+    }
+    if (n) {
+      uint32_t base = 0;
+      if (lane == 0) base = atomicAdd(&S.count_bucket, n);
+      base = __shfl_sync(0xffffffffu, base, 0);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t o = base + __popc(m[q] & lt);
+        if (((m[q] >> lane) & 1u) && o < (uint32_t)kBucketCap) bk[o] = key[q];
+        base += __popc(m[q]);
+      }
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[2], 1u) == gridDim.x - 1) ? 1u : 0u;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (threadIdx.x == 0) {
+    s_n = __ldcg(&S.count_bucket);
+    S.count_bucket = 0;
+    S.done[2] = 0;
+  }
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) gh[b] = 0;  // zero between uses
+  __syncthreads();
+  const uint32_t n = s_n;
+  uint32_t theta;
+  if (n <= (uint32_t)kBucketCap) {
+    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) fin[i] = __ldcg(&bk[i]);
+    __syncthreads();
+    uint32_t unused;
+    theta = smem_select(fin, n, r1, h, ws, &s_bin, &s_rank, &unused);
+  } else {
+    // the remaining digits (bits 19..10, then 9..0) over every sampled key
+    uint32_t prefix = b1, rr = r1;
+    for (int pass = 1; pass < 3; ++pass) {
+      const int shift = pass == 1 ? 10 : 0;
+      for (int b = threadIdx.x; b < 1024; b += blockDim.x) h[b] = 0;
+      if (threadIdx.x == 0) {
+        s_bin = 0;
+        s_rank = 0;
+      }
+      __syncthreads();
+      for (uint32_t i0 = 0; i0 < n_s; i0 += blockDim.x) {
+        const uint32_t i = i0 + threadIdx.x;
+        int bin = -1;
+        if (i < n_s) {
+          const uint32_t v = __ldcg(keys + i);
+          if ((v >> (shift + 10)) == prefix) bin = (int)((v >> shift) & 1023u);
+        }
+        warp_hist_add(h, bin);
+      }
+      __syncthreads();
+      block_find_from_top(h, 1024, rr, ws, &s_bin, &s_rank);
+      prefix = (prefix << 10) | s_bin;
+      rr = s_rank;
+      __syncthreads();
+    }
+    theta = prefix;
+  }
+  if (threadIdx.x == 0) {
+    // capped at the Inf key: every non-finite value is a candidate (and counted there)
+    S.theta = min(theta, 0x7f800000u);
+    S.count = 0;
+    S.dense = 0;
+    S.nsel = 0;
   }
 }
 
@@ -1023,39 +1195,6 @@ __global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
     if (h[b]) atomicAdd(&gh[b], h[b]);
 }
 
-// Radix select in shared memory: the r-th largest of n values (digits 11/10/10).
-__device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, uint32_t r,
-                                                uint32_t* h, uint32_t* ws, uint32_t* s_bin,
-                                                uint32_t* s_rank, uint32_t* rank_out) {
-  uint32_t prefix = 0;
-  for (int pass = 0; pass < 3; ++pass) {
-    const int nbins = pass == 0 ? 2048 : 1024;
-    const int shift = pass == 0 ? 20 : (pass == 1 ? 10 : 0);
-    for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
-    if (threadIdx.x == 0) {
-      *s_bin = 0;
-      *s_rank = 0;
-    }
-    __syncthreads();
-    for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
-      const uint32_t i = i0 + threadIdx.x;
-      int bin = -1;
-      if (i < n) {
-        const uint32_t v = x[i];
-        if (pass == 0 || (v >> (shift + 10)) == prefix) bin = (int)((v >> shift) & (uint32_t)(nbins - 1));
-      }
-      warp_hist_add(h, bin);
-    }
-    __syncthreads();
-    block_find_from_top(h, nbins, r, ws, s_bin, s_rank);
-    prefix = pass == 0 ? *s_bin : ((prefix << 10) | *s_bin);
-    r = *s_rank;
-    __syncthreads();
-  }
-  *rank_out = r;
-  return prefix;
-}
-
 __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   extern __shared__ __align__(16) uint32_t fin[];  // kBucketCap keys + kBucketCap indices
   __shared__ uint32_t h[kHistBins];
@@ -1173,21 +1312,89 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
 }
 
 // ---------------------------------------------------------------------------
+// Approximate top-s (Sec. 5.1): the candidates are C(v) itself -- every key
+// >= theta, all ties kept. One block per worker records T = theta and the
+// count, and counts the pairs and the non-zero ones (zeros are sent only when
+// theta is the zero key). More than `limit` candidates, or a part that
+// overflowed, leaves the worker to the dense path.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_select_approx(TopkArgs A) {
+  __shared__ uint32_t s_zero;
+  const int k = blockIdx.y;
+  WorkerSel& S = A.sel[k];
+  const uint32_t count = S.count;
+  if (S.dense || count > A.limit || count > A.cap) {
+    if (threadIdx.x == 0) S.dense = 1;
+    return;
+  }
+  const uint32_t T = S.theta;
+  if (threadIdx.x == 0) s_zero = 0;
+  __syncthreads();
+  if (T == 0u) {
+    const float* cv = A.cand_val + (int64_t)k * A.cap;
+    const int nparts = candidate_parts(A);
+    uint32_t z = 0;
+    for (int part = threadIdx.x >> 5; part < nparts; part += kWarps) {
+      uint32_t lo, hi;
+      candidate_part(A, k, part, nparts, &lo, &hi);
+      for (uint32_t i = lo + (threadIdx.x & 31); i < hi; i += 32) z += mag_key(cv[i]) == 0u;
+    }
+    if (z) atomicAdd(&s_zero, z);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    S.T = T;
+    S.t_idx = 0xffffffffu;
+    S.n_tie = 0;
+    S.nsel = count;
+    atomicAdd(&A.step_ctr->v[kPairs], (unsigned long long)count);
+    atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(count - s_zero));
+  }
+}
+
+// ---------------------------------------------------------------------------
 // dense exact select + chunk rewrite for workers whose filter missed; one
-// block per worker (a rare path: correct for any input, not fast).
+// block per worker (a rare path: correct for any input, not fast). For the
+// approximate top-s: every key >= theta when at most `limit` reach it, else
+// the exact top-`limit`.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
   const int k = blockIdx.x;
   WorkerSel& S = A.sel[k];
-  if (!needs_dense(S, A.ksel, A.cap)) return;
+  if (A.approx ? S.dense == 0 : !needs_dense(S, A.ksel, A.cap)) return;
   __shared__ uint32_t h[kHistBins];
   __shared__ uint32_t ws[32];
   __shared__ unsigned long long ws64[32];
   __shared__ uint32_t s_bin, s_rank;
+  __shared__ unsigned long long s_reach;
   const float* vk = A.e + (int64_t)k * A.ld;
   const int64_t d = A.d;
   uint32_t r = A.ksel, prefix = 0;
-  for (int pass = 0; pass < 3; ++pass) {
+  uint32_t nsel = A.ksel;
+  bool all_ties = false;  // approximate top-s below its limit: T = theta, every tie kept
+  unsigned long long reach = 0;  // approximate: (components above theta) << 32 | (equal to it)
+  if (A.approx) {
+    const uint32_t theta = S.theta;
+    unsigned long long x = 0;
+    for (int64_t j = threadIdx.x; j < d; j += blockDim.x) {
+      const uint32_t key = mag_key(vk[j]);
+      x += key > theta ? (1ull << 32) : (key == theta ? 1ull : 0ull);
+    }
+    unsigned long long tot;
+    block_inclusive_scan<unsigned long long>(x, ws64, &tot);
+    if (threadIdx.x == 0) s_reach = tot;
+    __syncthreads();
+    reach = s_reach;
+    const unsigned long long n_reach = (reach >> 32) + (reach & 0xffffffffull);
+    if (n_reach <= A.limit) {
+      all_ties = true;
+      nsel = (uint32_t)n_reach;
+    } else {
+      r = A.limit;
+      nsel = A.limit;
+    }
+  }
+  for (int pass = 0; pass < 3 && !all_ties; ++pass) {
     const int nbins = pass == 0 ? 2048 : 1024;
     const int shift = pass == 0 ? 20 : (pass == 1 ? 10 : 0);
     for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
@@ -1212,7 +1419,9 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
     r = s_rank;
     __syncthreads();
   }
-  const uint32_t T = prefix, n_tie = r;
+  const uint32_t T = all_ties ? S.theta : prefix;
+  const uint32_t n_tie = all_ties ? 0xffffffffu : r;
+  if (all_ties && threadIdx.x == 0) S.t_idx = 0xffffffffu;
 
   const int P = A.tile / (int)blockDim.x;  // consecutive elements per thread
   const int per_sub = (int)blockDim.x / kChunksPerTile;  // threads per sub-tile
@@ -1247,7 +1456,7 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
         if (key == T && qg + 1 == n_tie) S.t_idx = (uint32_t)j;  // the last tie kept
         if (key == T) ++qg;
         if (take) {
-          if (o < A.ksel && o < A.cap) {
+          if (o < nsel && o < A.cap) {
             oi[o] = (uint32_t)j;
             ov[o] = v;
           }
@@ -1266,13 +1475,17 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
     __syncthreads();
   }
   if (threadIdx.x == 0) {
-    if (running != A.ksel) atomicOr(A.status, kStatusInternal);
-    // the sub-chunks now hold exactly C(v), [0, k) of the candidate buffer
+    if (running != nsel) atomicOr(A.status, kStatusInternal);
+    // the sub-chunks now hold exactly C(v), [0, nsel) of the candidate buffer;
+    // zeros are sent only when T is the zero key: n_tie of them, or every tie
+    const uint32_t zeros = T != 0u ? 0u : (all_ties ? (uint32_t)(reach & 0xffffffffull) : n_tie);
     S.T = T;
     S.n_tie = n_tie;
+    S.nsel = nsel;
     S.dense = 1;
     atomicAdd(&A.step_ctr->v[kFallbacks], 1ull);
-    atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(A.ksel - (T == 0u ? n_tie : 0u)));
+    atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(nsel - zeros));
+    if (A.approx) atomicAdd(&A.step_ctr->v[kPairs], (unsigned long long)nsel);
   }
 }
 
@@ -1292,7 +1505,7 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
 __device__ __forceinline__ void sent_part(const TopkArgs& A, int k, int p, int nparts,
                                           uint32_t* lo, uint32_t* hi) {
   if (A.sel[k].dense || A.regions == 1) {
-    const uint32_t n = A.sel[k].dense ? A.ksel : min(A.sel[k].count, A.cap);
+    const uint32_t n = A.sel[k].dense ? (A.approx ? A.sel[k].nsel : A.ksel) : min(A.sel[k].count, A.cap);
     const uint32_t per = (n + nparts - 1) / nparts;
     *lo = min(n, (uint32_t)p * per);
     *hi = min(n, *lo + per);
@@ -1390,6 +1603,7 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
   const uint32_t T = A.sel[k].T, tidx = A.sel[k].t_idx;
+  const uint32_t want = A.approx ? A.sel[k].nsel : A.ksel;
   uint32_t carry = 0;
   for (int64_t t0 = 0; t0 < A.n_tiles; t0 += blockDim.x) {
     const int64_t tile = t0 + threadIdx.x;
@@ -1411,7 +1625,7 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
         for (uint32_t i = 0; i < n && base + i < A.cap; ++i) {
           const uint32_t j = ci[base + i];
           if (!selected(mag_key(cv[base + i]), j, T, tidx)) continue;
-          if (pos < A.ksel) {
+          if (pos < want) {
             idx_out[pos] = j;
             val_out[pos] = cv[base + i];
           }
@@ -1421,7 +1635,7 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
     }
     carry += tot;
   }
-  if (threadIdx.x == 0 && carry != A.ksel) atomicOr(A.status, kStatusInternal);
+  if (threadIdx.x == 0 && carry != want) atomicOr(A.status, kStatusInternal);
 }
 
 int tile_u(int tile) { return tile / (kWarps * 128); }
@@ -1445,6 +1659,7 @@ cudaError_t configure_topk_kernels() {
   set((const void*)k_accumulate<8>, 8192 * 12);
   set((const void*)k_accumulate_bulk, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_select_finish, 2 * kBucketCap * 4);
+  set((const void*)k_sample_theta, kBucketCap * 4);
   return err;
 }
 
@@ -1462,13 +1677,18 @@ int accumulate_blocks_per_sm(int tile) {
 }
 
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
-  if (A.pending && !A.dense_mode) {
-    const int n_s = A.sample_chunks ? A.sample_chunks * 8 : (int)A.d;
+  if ((A.pending || A.approx) && !A.dense_mode) {
+    const int n_s = (int)A.n_sample;
     k_sample_pending<<<(n_s + kThreads - 1) / kThreads, kThreads, 0, s>>>(A);
     const cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
   }
   k_sample<<<dim3(A.sample_blocks, A.K), kThreads, 0, s>>>(A);
+  if (A.approx) {
+    const cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    k_sample_theta<<<dim3(A.theta_blocks, A.K), kThreads, kBucketCap * 4, s>>>(A);
+  }
   return cudaGetLastError();
 }
 
@@ -1495,6 +1715,11 @@ cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t
     if (err != cudaSuccess) return err;
   }
   k_select_finish<<<grid, kThreads, 2 * kBucketCap * 4, s>>>(A);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select_approx(const TopkArgs& A, cudaStream_t s) {
+  k_select_approx<<<dim3(1, A.K), kThreads, 0, s>>>(A);
   return cudaGetLastError();
 }
 

@@ -15,7 +15,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libgmc.so")
 
 GMC_OK, GMC_EINVAL, GMC_ENOMEM, GMC_ECUDA, GMC_ENONFINITE, GMC_ESTATE, GMC_EINTERNAL, GMC_ETOOBIG = range(8)
-GMC_TOPK, GMC_RBGS = 0, 1
+GMC_TOPK, GMC_RBGS, GMC_TOPK_APPROX = 0, 1, 2
 GMC_SELECT_SAMPLED, GMC_SELECT_DENSE = 0, 1
 STAT_NAMES = ["steps", "pairs", "nnz", "union", "changed", "fallbacks", "nonfinite", "reserved"]
 GMC_STAT_COUNT = 8
@@ -120,7 +120,7 @@ class GMC:
         self.d, self.K = int(d), int(K)
         self.compressor = compressor
         self.device = torch.device(device if device is not None else "cuda")
-        comp = {"topk": GMC_TOPK, "rbgs": GMC_RBGS}[compressor]
+        comp = {"topk": GMC_TOPK, "rbgs": GMC_RBGS, "topk_approx": GMC_TOPK_APPROX}[compressor]
         h = _c_p()
         with torch.cuda.device(self.device):
             _check(self.lib.gmc_create(ctypes.byref(h), self.d, self.K, beta, eta, comp,

@@ -21,6 +21,7 @@ pytestmark = pytest.mark.gpu
     ("resnet50", 2, False, False),  # d = 25,557,032, K = 32, RBGS B = 4096, shared blocks, GMC+
     ("resnet50", 2, True, False),   # same, per-worker blocks
     ("vgg16", 3, False, True),      # d = 138,357,544, K = 8, top-k 0.1%
+    ("vgg16_approx", 3, False, True),  # the same under the approximate top-s of Sec. 5.1
 ])
 def test_fullsize_parity(name, steps, per_worker, deferred):
     import torch

@@ -36,7 +36,7 @@ class Workload:
     name: str
     d: int                      # parameters
     K: int                      # simulated workers
-    compressor: str             # "topk" or "rbgs"
+    compressor: str             # "topk", "topk_approx" or "rbgs"
     ratio: float                # top-k: k = max(1, floor(ratio*d)); rbgs: share of blocks
     beta: float
     eta: float
@@ -70,6 +70,10 @@ WORKLOADS = [
              eta=0.1, steps=20, block=4096, lam=0.5, n_segments=161, noniid=0.02),
     Workload("vgg16", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
              eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
+             scale_lo=1e-4, scale_hi=1e-1, noniid=0.02),
+    # the vgg16 configuration under the approximate top-s of Sec. 5.1 (s = d/1024)
+    Workload("vgg16_approx", d=138_357_544, K=8, compressor="topk_approx", ratio=1 / 1024,
+             beta=0.9, eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
              scale_lo=1e-4, scale_hi=1e-1, noniid=0.02),
 ]
 
