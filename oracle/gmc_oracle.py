@@ -21,6 +21,13 @@ Communication in Distributed Learning", arXiv 1905.12948):
     compression ratio times |S| -- sampled magnitudes reach it; every
     component with |a| >= theta is sent.
   * Relative communication cost (Sec. 5, RCC), halved for RBGS (Sec. 5.2).
+  * The appendix's other ways to combine momentum and error feedback, as
+    variants of the same step:
+      Alg. 3 (momentum on the server): e_{t+1/2,k} = e_{t,k} + g_{t,k};
+        w_{t+1} = w_t - (eta/K) sum_k C(e_{t+1/2,k}) + beta (w_t - w_{t-1});
+      Alg. 4 (learning rate inside the residual):
+        e_{t+1/2,k} = e_{t,k} + eta g_{t,k} - beta (w_t - w_{t-1});
+        w_{t+1} = w_t - (1/K) sum_k C(e_{t+1/2,k}).
 
 Precision. The paper fixes none. Top-s turns floating-point magnitudes into an
 integer decision (which indices are sent), so that decision is taken in the
@@ -67,6 +74,10 @@ U32 = np.uint32
 TOPK = "topk"
 RBGS = "rbgs"
 TOPK_APPROX = "topk_approx"
+
+ALG1 = "gmc"               # Algorithm 1 (the method)
+ALG3 = "server_momentum"   # Algorithm 3: momentum term on the server
+ALG4 = "lr_in_residual"    # Algorithm 4: learning rate inside the residual
 
 APPROX_SAMPLE_DIV = 100  # |S| = d/100 (Sec. 5.1)
 
@@ -247,7 +258,7 @@ class GMC:
 
     def __init__(self, d: int, K: int, beta: float, eta: float, compressor: str = TOPK,
                  ratio: float = 0.01, block: int = 4096, lam: float = 0.0, seed: int = 0,
-                 per_worker: bool = False):
+                 per_worker: bool = False, variant: str = ALG1):
         if d < 1 or K < 1:
             raise ValueError("d and K must be >= 1")
         if not 0.0 <= beta < 1.0:
@@ -258,6 +269,11 @@ class GMC:
             raise ValueError("ratio must be in (0, 1]")
         if compressor not in (TOPK, RBGS, TOPK_APPROX):
             raise ValueError("unknown compressor")
+        if variant not in (ALG1, ALG3, ALG4):
+            raise ValueError("unknown variant")
+        if variant != ALG1 and (compressor == RBGS or lam != 0.0):
+            raise ValueError("the appendix variants are GMC with a top-s compressor")
+        self.variant = variant
         self.d, self.K = d, K
         self.beta = F32(beta)
         self.lam = F32(lam)
@@ -282,10 +298,13 @@ class GMC:
         self.w = None
 
     def set_eta(self, eta: float) -> None:
-        """Constants of the step, each one fp32 rounding of the paper's ratio."""
+        """Constants of the step, each one fp32 rounding of the paper's ratio.
+        Alg. 4 scales the residual update by 1/K instead of eta/K."""
         self.eta = F32(eta)
         self.c = F32(self.beta / self.eta)          # beta / eta
         self.a = F32(self.eta / F32(self.K))        # eta / K
+        if self.variant == ALG4:
+            self.a = F32(F32(1.0) / F32(self.K))    # 1 / K
         self.b = F32(self.lam * self.eta)           # lambda * eta
 
     def set_params(self, w0: np.ndarray) -> None:
@@ -315,8 +334,12 @@ class GMC:
         K = self.K
 
         # workers: e_{t+1/2,k} = e_{t,k} + g_{t,k} - (beta/eta)(w_t - w_{t-1})
-        momentum = self.c * (self.w - self.w_prev)
-        e_half = (self.e + g) - momentum
+        if self.variant == ALG1:
+            e_half = (self.e + g) - self.c * (self.w - self.w_prev)
+        elif self.variant == ALG3:   # e_{t,k} + g_{t,k}
+            e_half = self.e + g
+        else:                        # e_{t,k} + eta g_{t,k} - beta (w_t - w_{t-1})
+            e_half = (self.e + self.eta * g) - self.beta * (self.w - self.w_prev)
 
         # workers: C(e_{t+1/2,k}) -- its support and values
         blocks = sample = thresholds = None
@@ -340,10 +363,13 @@ class GMC:
             e_next[k, supports[k]] = F32(0.0)
 
         # server: w_{t+1} = w_t - (eta/K) sum_k C(e_{t+1/2,k}), workers summed in order
+        # (Alg. 4: 1/K in a; Alg. 3 adds beta (w_t - w_{t-1}))
         total = np.zeros(self.d, F32)
         for k in range(K):
             total[supports[k]] = total[supports[k]] + values[k]
         w_next = self.w - self.a * total
+        if self.variant == ALG3:
+            w_next = w_next + self.beta * (self.w - self.w_prev)
 
         in_union = np.zeros(self.d, bool)
         for k in range(K):

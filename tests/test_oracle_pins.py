@@ -426,6 +426,118 @@ def test_rcc_dense_pairs():
 
 
 # ---------------------------------------------------------------------------
+# The appendix variants: Alg. 3 (momentum on the server) and Alg. 4 (learning
+# rate inside the residual)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("variant", [oracle.ALG3, oracle.ALG4])
+def test_variants_without_compression_are_heavy_ball(variant):
+    """ratio = 1: both variants leave e = 0 exactly and follow the heavy-ball
+    recursion of eq. (2) in float64 (the appendix: they differ from GMC only
+    in how the compression error is fed back)."""
+    rng = np.random.default_rng(21)
+    d, K, T, eta, beta = 129, 3, 40, 0.05, 0.9
+    o = GMC(d, K, beta=beta, eta=eta, compressor=TOPK, ratio=1.0, variant=variant)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    o.set_params(w0)
+    grads = _grads(rng, T, K, d)
+    eta32, beta32 = float(np.float32(eta)), float(np.float32(beta))
+    ref = _heavy_ball(w0.astype(np.float64), [g.astype(np.float64) for g in grads], eta32, beta32)
+    budget = np.zeros(d)
+    w_prev = w0.astype(np.float64)
+    for t, g in enumerate(grads):
+        w_t = o.w.astype(np.float64)
+        o.step(g)
+        assert not np.any(o.e)
+        w_next = o.w.astype(np.float64)
+        dlt = np.abs(w_t - w_prev)
+        local = 6 * U * (np.abs(w_next) + np.abs(w_t) + (K + 3) * eta32 / K *
+                         (np.abs(g.astype(np.float64)).sum(0) + K * beta32 / eta32 * dlt) + beta32 * dlt)
+        budget += local
+        np.testing.assert_array_less(np.abs(w_next - ref[t + 1]), 2 * budget / (1 - beta32) + 1e-30)
+        w_prev = w_t
+
+
+def test_alg3_update_rule_is_gmcs():
+    """Eliminating C from Alg. 3 gives GMC's update rule (the appendix): the
+    P5 identity holds for Alg. 3's residuals."""
+    rng = np.random.default_rng(22)
+    d, K, T = 600, 4, 30
+    o = GMC(d, K, beta=0.9, eta=0.1, compressor=TOPK, ratio=0.05, variant=oracle.ALG3)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    for lhs, rhs, budget, *_ in _update_rule_residual(o, _grads(rng, T, K, d)):
+        np.testing.assert_array_less(np.abs(lhs - rhs), budget + 1e-30)
+
+
+def test_alg4_update_rule():
+    """Alg. 4 with C eliminated: w_{t+1} - w_t = -eta gbar - ebar_t + ebar_{t+1}
+    + beta (w_t - w_{t-1}) (its residual carries the learning rate)."""
+    rng = np.random.default_rng(23)
+    d, K, T, eta, beta = 600, 4, 30, 0.1, 0.9
+    o = GMC(d, K, beta=beta, eta=eta, compressor=TOPK, ratio=0.05, variant=oracle.ALG4)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    eta32, beta32 = float(np.float32(eta)), float(np.float32(beta))
+    w_prev = o.w.astype(np.float64)
+    for g in _grads(rng, T, K, d):
+        w_t, e_t = o.w.astype(np.float64), o.e.astype(np.float64)
+        r = o.step(g)
+        w_n, e_n, g64 = o.w.astype(np.float64), o.e.astype(np.float64), g.astype(np.float64)
+        lhs = w_n - w_t
+        rhs = -eta32 * g64.mean(0) - e_t.mean(0) + e_n.mean(0) + beta32 * (w_t - w_prev)
+        dl = np.abs(w_t - w_prev)
+        scale = (np.abs(e_t) + eta32 * np.abs(g64) + beta32 * dl + np.abs(r.e_half) + np.abs(e_n)).sum(0)
+        budget = 8 * U * (np.abs(w_n) + np.abs(w_t) + (K + 3) / K * scale + beta32 * dl)
+        np.testing.assert_array_less(np.abs(lhs - rhs), budget + 1e-30)
+        w_prev = w_t
+
+
+@pytest.mark.parametrize("variant", [oracle.ALG3, oracle.ALG4])
+def test_variants_reduce_to_gmc(variant):
+    """Bitwise: with beta = 0 Alg. 3 is GMC; with beta = 0 and eta = 1 Alg. 4
+    is GMC (the learning-rate factor and the 1/K scale coincide)."""
+    rng = np.random.default_rng(24)
+    d, K, T = 500, 3, 10
+    eta = 1.0 if variant == oracle.ALG4 else 0.1
+    a = GMC(d, K, beta=0.0, eta=eta, compressor=TOPK, ratio=0.05)
+    b = GMC(d, K, beta=0.0, eta=eta, compressor=TOPK, ratio=0.05, variant=variant)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    a.set_params(w0)
+    b.set_params(w0)
+    for g in _grads(rng, T, K, d):
+        ra, rb = a.step(g), b.step(g)
+        for k in range(K):
+            np.testing.assert_array_equal(ra.supports[k], rb.supports[k])
+        assert np.array_equal(a.w.view(np.uint32), b.w.view(np.uint32))
+        assert np.array_equal(a.e.view(np.uint32), b.e.view(np.uint32))
+
+
+def test_alg4_is_gmc_scaled_under_constant_eta():
+    """The appendix: with a constant learning rate Alg. 4 is Alg. 1, its
+    residual being eta times GMC's. Same supports, e4 = eta e1 and w4 = w1 up
+    to fp32 rounding."""
+    rng = np.random.default_rng(25)
+    d, K, T, eta = 800, 4, 12, 0.25
+    a = GMC(d, K, beta=0.9, eta=eta, compressor=TOPK, ratio=0.02)
+    b = GMC(d, K, beta=0.9, eta=eta, compressor=TOPK, ratio=0.02, variant=oracle.ALG4)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    a.set_params(w0)
+    b.set_params(w0)
+    for g in _grads(rng, T, K, d):
+        ra, rb = a.step(g), b.step(g)
+        for k in range(K):
+            np.testing.assert_array_equal(ra.supports[k], rb.supports[k])
+        np.testing.assert_allclose(b.e, float(a.eta) * a.e.astype(np.float64), rtol=1e-4, atol=1e-6)
+        np.testing.assert_allclose(b.w, a.w, rtol=1e-5, atol=1e-6)
+
+
+def test_variants_refuse_gmcplus_and_rbgs():
+    with pytest.raises(ValueError):
+        GMC(10, 2, 0.9, 0.1, compressor=RBGS, block=2, variant=oracle.ALG3)
+    with pytest.raises(ValueError):
+        GMC(10, 2, 0.9, 0.1, lam=0.5, variant=oracle.ALG4)
+
+
+# ---------------------------------------------------------------------------
 # Approximate top-s (Sec. 5.1): sample, threshold, selection
 # ---------------------------------------------------------------------------
 
