@@ -225,7 +225,8 @@ def oracle_sample(wl, budget_s: float = 12.0, max_steps: int = 50, workers: int 
     d_s = min(wl.d, d_sample)
     gen = workloads.NumpyGradients(wl, seed=0, d=d_s, K=K_s)
     o = oracle.GMC(d_s, K_s, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
-                   block=wl.block, lam=wl.lam, seed=0, per_worker=wl.per_worker)
+                   block=wl.block, lam=wl.lam, seed=0, per_worker=wl.per_worker,
+                   variant=wl.variant)
     o.set_params(workloads.init_params(wl.d)[:d_s])
     spent, steps = 0.0, 0
     while steps < max_steps and (spent < budget_s or steps == 0):
@@ -275,11 +276,13 @@ def config_of(wl, args):
     return {"workload": f"{wl.name}: d={wl.d:,}, K={wl.K}, {wl.compressor}"
                         + (f" ratio {wl.ratio:.6g}" if wl.compressor != "rbgs"
                            else f" block {wl.block}, {wl.ratio:.0%} of blocks, lambda {wl.lam}")
-                        + f", beta {wl.beta}, eta {wl.eta}",
+                        + f", beta {wl.beta}, eta {wl.eta}"
+                        + ("" if wl.variant == "gmc" else f", variant {wl.variant}"),
             "d": wl.d, "K": wl.K, "compressor": wl.compressor, "ratio": wl.ratio,
             "block": wl.block if wl.compressor == "rbgs" else None,
             "per_worker_blocks": wl.per_worker if wl.compressor == "rbgs" else None,
-            "lambda": wl.lam, "l2": "inputs larger than L2 (gradient batches rotate)",
+            "lambda": wl.lam, "variant": wl.variant,
+            "l2": "inputs larger than L2 (gradient batches rotate)",
             "parallelism": f"replicas x{args.gpus}"}
 
 
@@ -294,7 +297,7 @@ def run_gmc(args, wl, world, rank, local):
     torch.cuda.set_device(dev)
     gpu = GMC(wl.d, wl.K, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
               block=wl.block, lam=wl.lam if wl.compressor == "rbgs" else None, seed=0,
-              per_worker=wl.per_worker, device=dev)
+              per_worker=wl.per_worker, variant=wl.variant, device=dev)
     w0 = torch.from_numpy(workloads.init_params(wl.d)).to(dev)
     gen = workloads.TorchGradients(wl, dev, seed=rank)
     n_batches = 2 if 4.0 * wl.K * wl.d > 2 * L2_BYTES else max(2, math.ceil(4 * L2_BYTES / (4.0 * wl.K * wl.d)))

@@ -72,6 +72,16 @@ typedef struct gmc_ctx* gmc_t;
                              than min(d, 4 s + 4096) do (s = max(1, floor(ratio*d))):
                              then the exact top of that many */
 
+/* Variants of the step (gmc_set_variant): the method, and the appendix's other
+ * ways to combine momentum with error feedback, for comparison. */
+#define GMC_VARIANT_GMC              0 /* Alg. 1 (default) */
+#define GMC_VARIANT_SERVER_MOMENTUM  1 /* Alg. 3: e_{t+1/2,k} = e_{t,k} + g_{t,k};
+                                          w_{t+1} = (w_t - (eta/K) sum_k C_k)
+                                                    + beta (w_t - w_{t-1}), a dense update */
+#define GMC_VARIANT_LR_IN_RESIDUAL   2 /* Alg. 4: e_{t+1/2,k} = (e_{t,k} + eta g_{t,k})
+                                                             - beta (w_t - w_{t-1});
+                                          w_{t+1} = w_t - fl(1/K) sum_k C_k */
+
 /* Top-k selection engines; both give identical results. */
 #define GMC_SELECT_SAMPLED 0 /* default: a sampled threshold filters candidates in the one
                                 dense pass; exact radix select among them; falls back to
@@ -121,7 +131,8 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta,
 /* gmc_destroy -- synchronise the device and free everything the handle owns. */
 void gmc_destroy(gmc_t h);
 
-/* gmc_set_lambda -- GMC+ detach coefficient lambda in [0,1] (Alg. 2); 0 is GMC. */
+/* gmc_set_lambda -- GMC+ detach coefficient lambda in [0,1] (Alg. 2); 0 is GMC.
+ * GMC_EINVAL for lambda != 0 under an appendix variant (GMC+ detaches Alg. 1). */
 int gmc_set_lambda(gmc_t h, float lambda);
 
 /* gmc_set_rbgs_mode -- 0: one block choice per step shared by all workers, as in
@@ -136,6 +147,16 @@ int gmc_set_seed(gmc_t h, uint64_t seed);
 /* gmc_set_eta -- change eta between steps (e.g. the cosine schedule of Sec. 5.1);
  * takes effect at the next gmc_step. */
 int gmc_set_eta(gmc_t h, float eta);
+
+/* gmc_set_variant -- the step's form (GMC_VARIANT_*; default Alg. 1). Only for the
+ * top-k compressors (exact and approximate) with lambda = 0, and only before the
+ * first step after gmc_create or gmc_set_params (GMC_ESTATE otherwise), since the
+ * residuals mean another thing under each form. GMC_VARIANT_SERVER_MOMENTUM
+ * allocates d floats of w_t - w_{t-1} (GMC_ENOMEM if that fails) and turns off
+ * the deferred aggregation: every step ends with a dense pass over w. Synchronising
+ * when it allocates. Arithmetic: each operation rounded once, in the order written
+ * beside the GMC_VARIANT_* constants. */
+int gmc_set_variant(gmc_t h, int32_t variant);
 
 /* gmc_set_select_mode -- GMC_SELECT_SAMPLED (default) or GMC_SELECT_DENSE (exact
  * top-k only: GMC_EINVAL for GMC_TOPK_APPROX, which its sample defines). */

@@ -36,6 +36,8 @@ struct gmc_ctx {
   uint64_t seed = 0;
   int per_worker = 0;
   int select_mode = GMC_SELECT_SAMPLED;
+  int variant = GMC_VARIANT_GMC;  // Alg. 1, or the appendix's Alg. 3 / Alg. 4
+  float* mom = nullptr;           // Alg. 3: w_t - w_{t-1} (allocated by gmc_set_variant)
   float* detach_out = nullptr;
   int64_t detach_ld = 0;
   // geometry
@@ -193,6 +195,17 @@ void drain_profile(gmc_ctx* h) {
 void set_constants(gmc_ctx* h, TopkArgs* A) {
   A->c = h->beta / h->eta;
   A->a = h->eta / (float)h->K;
+  A->beta = h->beta;
+  A->mom = h->mom;
+  if (h->variant == GMC_VARIANT_SERVER_MOMENTUM) {  // Alg. 3: e + g; the momentum is the server's
+    A->c = 0.f;
+    A->server_mom = 1;
+  } else if (h->variant == GMC_VARIANT_LR_IN_RESIDUAL) {  // Alg. 4: e + eta*g - beta*dw, w -= (1/K) sum
+    A->c = h->beta;
+    A->a = 1.f / (float)h->K;
+    A->gscale = 1;
+    A->gs = h->eta;
+  }
 }
 
 // Arguments of step t's top-k kernels; chunk buffers alternate with the parity of t.
@@ -319,7 +332,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
     A.g_direct = direct ? 1 : 0;
     A.pending = h->agg_pending ? 1 : 0;
     A.a_prev = h->a_pending;
-    const bool defer = h->tile == kBulkTile && !eager && !h->detach_out;
+    const bool defer = h->tile == kBulkTile && !eager && !h->detach_out && !A.server_mom;
     const double kk = (double)h->K * (double)h->ksel;
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
@@ -337,9 +350,11 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
       TopkArgs B = A;
       B.a_prev = A.a;
       B.total_ctr = nullptr;  // k_finalize adds the step's counts to the totals
-      GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk, s, [&] {
+      GMC_TRY(timed(h, GMC_KERNEL_AGGREGATE, 24.0 * kk + (B.server_mom ? 20.0 * h->d : 0.0), s, [&] {
         cudaError_t err = launch_mark(B, h->grid_agg, s);
-        return err != cudaSuccess ? err : launch_owner_sum(B, h->grid_agg, s);
+        if (err == cudaSuccess) err = launch_owner_sum(B, h->grid_agg, s);
+        if (err == cudaSuccess && B.server_mom) err = launch_server_update(B, s);  // Alg. 3
+        return err;
       }));
     }
     pairs_add = approx ? 0ull : (unsigned long long)h->K * h->ksel;  // approximate: counted on the device
@@ -596,6 +611,7 @@ void gmc_destroy(gmc_t h) {
 
 int gmc_set_lambda(gmc_t h, float lambda) {
   if (!h || !finite_f(lambda) || lambda < 0.f || lambda > 1.f) return GMC_EINVAL;
+  if (lambda != 0.f && h->variant != GMC_VARIANT_GMC) return GMC_EINVAL;  // GMC+ detaches Alg. 1
   h->lambda = lambda;
   return GMC_OK;
 }
@@ -615,6 +631,23 @@ int gmc_set_seed(gmc_t h, uint64_t seed) {
 int gmc_set_eta(gmc_t h, float eta) {
   if (!h || !finite_f(eta) || !(eta > 0.f)) return GMC_EINVAL;
   h->eta = eta;
+  return GMC_OK;
+}
+
+int gmc_set_variant(gmc_t h, int32_t variant) {
+  if (!h) return GMC_EINVAL;
+  if (variant != GMC_VARIANT_GMC && variant != GMC_VARIANT_SERVER_MOMENTUM &&
+      variant != GMC_VARIANT_LR_IN_RESIDUAL)
+    return GMC_EINVAL;
+  if (variant != GMC_VARIANT_GMC && (h->compressor == GMC_RBGS || h->lambda != 0.f)) return GMC_EINVAL;
+  if (h->initialized && h->t > 0) return GMC_ESTATE;  // the residuals mean another thing
+  if (variant == GMC_VARIANT_SERVER_MOMENTUM && !h->mom) {
+    DeviceGuard g(h->device);
+    cudaError_t err = dalloc(h, &h->mom, (size_t)h->ld);
+    if (err == cudaSuccess) err = cudaMemset(h->mom, 0, (size_t)h->ld * sizeof(float));
+    if (err != cudaSuccess) return status_of(err);
+  }
+  h->variant = variant;
   return GMC_OK;
 }
 
@@ -643,6 +676,7 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
   GMC_TRY(cudaMemcpyAsync(h->w, w0_dev, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice, s));
   GMC_TRY(cudaMemsetAsync(h->e, 0, (size_t)h->K * h->ld * sizeof(float), s));
   GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
+  if (h->mom) GMC_TRY(cudaMemsetAsync(h->mom, 0, (size_t)h->ld * sizeof(float), s));
   if (h->compressor != GMC_RBGS) {
     for (int p = 0; p < 2; ++p)
       GMC_TRY(cudaMemsetAsync(h->chunk[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint2), s));

@@ -28,7 +28,16 @@ struct TopkArgs {
   int64_t d;
   float* dlt;                // w_t - w_{t-1}, dense, zero outside the last union
   float* w;                  // parameters (ld floats)
-  float c, a;                // fl(beta/eta), fl(eta/K)
+  float c, a;                // fl(beta/eta), fl(eta/K) (Alg. 4: beta and fl(1/K); Alg. 3: c = 0)
+  // The appendix variants: Alg. 4 scales the gradient by eta in the
+  // accumulator (gscale, gs = eta); Alg. 3 adds beta (w_t - w_{t-1}) on the
+  // server, densely (server_mom: the aggregate leaves the sum in dlt, and
+  // k_server_update applies w_{t+1} = (w_t - a*s) + beta*mom, mom = w_t - w_{t-1}).
+  int gscale;
+  float gs;
+  int server_mom;
+  float beta;
+  float* mom;                // Alg. 3: w_t - w_{t-1} over [0, d)
   int K;
   int64_t n_tiles;
   int tile;                  // elements per tile
@@ -136,6 +145,8 @@ cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s);
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s);
 // Approximate top-s: T = theta, every tie kept, the count; or the dense path.
 cudaError_t launch_select_approx(const TopkArgs& A, cudaStream_t s);
+// Alg. 3's server step over [0, d): w_{t+1} = (w_t - a*s) + beta*(w_t - w_{t-1}).
+cudaError_t launch_server_update(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s);
 constexpr int kBulkTile = 4096;  // tile of the bulk-copy accumulate pass (k_accumulate_bulk)
 constexpr int kBulkMaxK = 16;    // workers the bulk-copy pass takes (its shared memory grows with K)

@@ -18,6 +18,8 @@
 //
 // Keys are the fp32 bit patterns with the sign cleared (monotone in |v|); the
 // selected set is the first k elements under (key descending, index ascending).
+#include <algorithm>
+
 #include "gmc_internal.h"
 
 namespace gmc {
@@ -41,6 +43,17 @@ __device__ __forceinline__ float4 load_g4(const float* __restrict__ g, int64_t j
   if (j + 1 < d) r.y = g[j + 1];
   if (j + 2 < d) r.z = g[j + 2];
   return r;
+}
+
+// Alg. 4 feeds eta * g into the accumulator: one more rounded product.
+__device__ __forceinline__ float4 scale_g(const TopkArgs& A, float4 g) {
+  if (A.gscale) {
+    g.x = __fmul_rn(A.gs, g.x);
+    g.y = __fmul_rn(A.gs, g.y);
+    g.z = __fmul_rn(A.gs, g.z);
+    g.w = __fmul_rn(A.gs, g.w);
+  }
+  return g;
 }
 
 __device__ __forceinline__ int g_mode(const float* p) {
@@ -179,12 +192,12 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
         const int64_t j = A.sample_pend[2 * A.sample_stride + i];
         const uint32_t m = A.sample_pend[i];
         ev[q] = ((m >> k) & 1u) ? 0.f : ek[j];
-        gv[q] = gk[j];
+        gv[q] = A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j];
         dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
       } else if (i < i_hi) {
         const int64_t j = sample_coord(A, skey, i);
         ev[q] = ek[j];
-        gv[q] = gk[j];
+        gv[q] = A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j];
         dv[q] = A.dlt[j];
         if (A.pending) {  // as if the previous step's aggregation were applied at j
           const uint32_t m = A.sample_pend[i];
@@ -628,7 +641,7 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
       for (int u = 0; u < U; ++u) {
         const int l = u * 128 + lane * 4;
         ev[u] = __ldcs(reinterpret_cast<const float4*>(ekt + l));
-        gv[u] = load_g4(gk, (int64_t)s0 + l, A.d, gm);
+        gv[u] = scale_g(A, load_g4(gk, (int64_t)s0 + l, A.d, gm));
       }
       float v[U][4];
       uint32_t bits[U];
@@ -999,6 +1012,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
           if (l + 2 >= lim) g4.z = 0.f;
           if (l + 3 >= lim) g4.w = 0.f;
         }
+        g4 = scale_g(A, g4);
         if (many) {  // more union coordinates than lanes: per-element sender masks
           const uint4 m4 = *reinterpret_cast<const uint4*>(mkw + l);
           if ((m4.x >> k) & 1u) e4.x = 0.f;
@@ -1575,13 +1589,17 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
           A.e[(int64_t)b * A.ld + j] = 0.f;  // e_{t+1,b} = e_{t+1/2,b} - C(.) = +0 where sent
         }
       }
+      A.mask[j] = 0u;
+      ++uni;
+      if (A.server_mom) {  // Alg. 3: k_server_update applies the sum with the momentum term
+        A.dlt[j] = sum;
+        continue;
+      }
       const float wn = __fsub_rn(wo, __fmul_rn(A.a_prev, sum));
       A.w[j] = wn;
       const float dd = __fsub_rn(wn, wo);
       A.dlt[j] = dd;
-      A.mask[j] = 0u;
       changed += (dd != 0.f);
-      ++uni;
     }
   }
   uni = warp_sum(uni);
@@ -1593,6 +1611,46 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
       if (changed) atomicAdd(&c->v[kChanged], changed);
     }
   }
+}
+
+// Alg. 3, the server with the momentum term, over every coordinate:
+// w_{t+1} = (w_t - a*s) + beta*(w_t - w_{t-1}), s the workers' sum (left in
+// dlt by the aggregate on the union, +0 elsewhere); then mom = w_{t+1} - w_t
+// (what fl(w_{t+1} - w_t) gives the next step) and dlt back to zero.
+__global__ void __launch_bounds__(kThreads) k_server_update(TopkArgs A) {
+  unsigned long long changed = 0;
+  const int64_t n4 = A.d >> 2;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < n4; q += stride) {
+    const float4 s4 = __ldcs(reinterpret_cast<const float4*>(A.dlt) + q);
+    const float4 w4 = __ldcs(reinterpret_cast<const float4*>(A.w) + q);
+    const float4 m4 = __ldcs(reinterpret_cast<const float4*>(A.mom) + q);
+    const float s[4] = {s4.x, s4.y, s4.z, s4.w}, wo[4] = {w4.x, w4.y, w4.z, w4.w};
+    const float mo[4] = {m4.x, m4.y, m4.z, m4.w};
+    float wn[4], mn[4];
+    bool nz = false;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      wn[i] = __fadd_rn(__fsub_rn(wo[i], __fmul_rn(A.a, s[i])), __fmul_rn(A.beta, mo[i]));
+      mn[i] = __fsub_rn(wn[i], wo[i]);
+      changed += mn[i] != 0.f;
+      nz |= __float_as_uint(s[i]) != 0u;
+    }
+    __stcs(reinterpret_cast<float4*>(A.w) + q, make_float4(wn[0], wn[1], wn[2], wn[3]));
+    __stcs(reinterpret_cast<float4*>(A.mom) + q, make_float4(mn[0], mn[1], mn[2], mn[3]));
+    if (nz) reinterpret_cast<float4*>(A.dlt)[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  for (int64_t j = (n4 << 2) + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < A.d; j += stride) {
+    const float s = A.dlt[j], wo = A.w[j];
+    const float wn = __fadd_rn(__fsub_rn(wo, __fmul_rn(A.a, s)), __fmul_rn(A.beta, A.mom[j]));
+    const float mn = __fsub_rn(wn, wo);
+    A.w[j] = wn;
+    A.mom[j] = mn;
+    changed += mn != 0.f;
+    if (__float_as_uint(s) != 0u) A.dlt[j] = 0.f;
+  }
+  changed = warp_sum(changed);
+  if ((threadIdx.x & 31) == 0 && changed) atomicAdd(&A.step_ctr->v[kChanged], changed);
 }
 
 // (index, value) pairs of worker k's last C(.) in ascending index order: its
@@ -1735,6 +1793,18 @@ cudaError_t launch_mark(const TopkArgs& A, int grid, cudaStream_t s) {
 
 cudaError_t launch_owner_sum(const TopkArgs& A, int grid, cudaStream_t s) {
   k_owner_sum<<<dim3(grid, A.K), kThreads, 0, s>>>(A);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_server_update(const TopkArgs& A, cudaStream_t s) {
+  int n = 0;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_server_update, kThreads, 0);
+  int dev = 0, sms = 1;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (A.d / 4 + kThreads - 1) / kThreads;
+  const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sms * std::max(n, 1)));
+  k_server_update<<<grid, kThreads, 0, s>>>(A);
   return cudaGetLastError();
 }
 

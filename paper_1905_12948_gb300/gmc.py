@@ -16,6 +16,7 @@ LIB_PATH = os.path.join(_PKG, "libgmc.so")
 
 GMC_OK, GMC_EINVAL, GMC_ENOMEM, GMC_ECUDA, GMC_ENONFINITE, GMC_ESTATE, GMC_EINTERNAL, GMC_ETOOBIG = range(8)
 GMC_TOPK, GMC_RBGS, GMC_TOPK_APPROX = 0, 1, 2
+VARIANTS = {"gmc": 0, "server_momentum": 1, "lr_in_residual": 2}  # Alg. 1, Alg. 3, Alg. 4
 GMC_SELECT_SAMPLED, GMC_SELECT_DENSE = 0, 1
 STAT_NAMES = ["steps", "pairs", "nnz", "union", "changed", "fallbacks", "nonfinite", "reserved"]
 GMC_STAT_COUNT = 8
@@ -38,6 +39,7 @@ _SIGNATURES = {
     "gmc_set_seed": (ctypes.c_int, [_c_p, _u64]),
     "gmc_set_eta": (ctypes.c_int, [_c_p, _f32]),
     "gmc_set_select_mode": (ctypes.c_int, [_c_p, _i32]),
+    "gmc_set_variant": (ctypes.c_int, [_c_p, _i32]),
     "gmc_set_detach_output": (ctypes.c_int, [_c_p, _c_p, _i64]),
     "gmc_set_params": (ctypes.c_int, [_c_p, _c_p, _c_p]),
     "gmc_step": (ctypes.c_int, [_c_p, _c_p, _c_p]),
@@ -113,7 +115,7 @@ class GMC:
     def __init__(self, d: int, K: int, beta: float, eta: float, compressor: str = "topk",
                  ratio: float = 0.01, block: int = 4096, lam: Optional[float] = None,
                  seed: int = 0, per_worker: bool = False, select_mode: str = "sampled",
-                 device=None):
+                 variant: str = "gmc", device=None):
         import torch
         self.torch = torch
         self.lib = load()
@@ -132,6 +134,9 @@ class GMC:
         _check(self.lib.gmc_set_rbgs_mode(h, int(bool(per_worker))), "gmc_set_rbgs_mode")
         mode = {"sampled": GMC_SELECT_SAMPLED, "dense": GMC_SELECT_DENSE}[select_mode]
         _check(self.lib.gmc_set_select_mode(h, mode), "gmc_set_select_mode")
+        if variant != "gmc":
+            with torch.cuda.device(self.device):
+                _check(self.lib.gmc_set_variant(h, VARIANTS[variant]), "gmc_set_variant")
         self._detach = None
 
     def close(self) -> None:

@@ -24,7 +24,8 @@ class Pair:
     """A CUDA handle and an oracle instance fed identical inputs."""
 
     def __init__(self, d, K, beta, eta, compressor="topk", ratio=0.01, block=4096, lam=None,
-                 seed=0, per_worker=False, select_mode="sampled", w0=None, device="cuda"):
+                 seed=0, per_worker=False, select_mode="sampled", w0=None, device="cuda",
+                 variant="gmc"):
         import torch
         from paper_1905_12948_gb300 import GMC
         self.torch = torch
@@ -32,9 +33,10 @@ class Pair:
         self.dev = torch.device(device)
         lam_or = (0.5 if compressor == "rbgs" else 0.0) if lam is None else lam
         self.gpu = GMC(d, K, beta, eta, compressor=compressor, ratio=ratio, block=block, lam=lam,
-                       seed=seed, per_worker=per_worker, select_mode=select_mode, device=self.dev)
+                       seed=seed, per_worker=per_worker, select_mode=select_mode, device=self.dev,
+                       variant=variant)
         self.ref = oracle.GMC(d, K, beta, eta, compressor=compressor, ratio=ratio, block=block,
-                              lam=lam_or, seed=seed, per_worker=per_worker)
+                              lam=lam_or, seed=seed, per_worker=per_worker, variant=variant)
         if w0 is None:
             w0 = (np.random.default_rng(seed + 17).standard_normal(d) * 0.01).astype(np.float32)
         self.gpu.set_params(torch.from_numpy(w0).to(self.dev))

@@ -53,6 +53,7 @@ class Workload:
     noniid: float = 0.0         # per-worker mean offset std as a multiple of the segment std
     iid_unit: bool = False      # gradients N(0,1) i.i.d., no segments
     w0_std: float = 0.01
+    variant: str = "gmc"        # Alg. 1, or the appendix's "server_momentum" (Alg. 3) / "lr_in_residual" (Alg. 4)
 
     @property
     def k(self) -> int:
@@ -75,6 +76,13 @@ WORKLOADS = [
     Workload("vgg16_approx", d=138_357_544, K=8, compressor="topk_approx", ratio=1 / 1024,
              beta=0.9, eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
              scale_lo=1e-4, scale_hi=1e-1, noniid=0.02),
+    # the vgg16 configuration under the appendix's Alg. 3 and Alg. 4
+    Workload("vgg16_alg3", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
+             eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
+             scale_lo=1e-4, scale_hi=1e-1, noniid=0.02, variant="server_momentum"),
+    Workload("vgg16_alg4", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
+             eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
+             scale_lo=1e-4, scale_hi=1e-1, noniid=0.02, variant="lr_in_residual"),
 ]
 
 
