@@ -22,6 +22,8 @@ pytestmark = pytest.mark.gpu
     ("resnet50", 2, True, False),   # same, per-worker blocks
     ("vgg16", 3, False, True),      # d = 138,357,544, K = 8, top-k 0.1%
     ("vgg16_approx", 3, False, True),  # the same under the approximate top-s of Sec. 5.1
+    ("vgg16_alg3", 2, False, False),   # the same under the appendix's Alg. 3 (eager, dense server step)
+    ("vgg16_alg4", 2, False, True),    # and Alg. 4
 ])
 def test_fullsize_parity(name, steps, per_worker, deferred):
     import torch
@@ -31,7 +33,7 @@ def test_fullsize_parity(name, steps, per_worker, deferred):
     rbgs = wl.compressor == "rbgs"
     p = Pair(wl.d, wl.K, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
              block=wl.block, lam=wl.lam if rbgs else None, seed=0, per_worker=per_worker,
-             w0=workloads.init_params(wl.d), device=dev)
+             w0=workloads.init_params(wl.d), device=dev, variant=wl.variant)
     for t in range(steps):
         g_dev = gen(t)
         assert bool(torch.isfinite(g_dev).all()), "synthetic gradients must be finite"
