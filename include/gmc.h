@@ -234,6 +234,31 @@ int gmc_get_worker_params(gmc_t h, int32_t k, float* out_dev, void* stream);
  * sum_t sum_k ||C_k||_0) / (d K T), halved for RBGS (no indices, Sec. 5.2). */
 int gmc_get_stats(gmc_t h, uint64_t* counters_host, int32_t n, double* rcc_host);
 
+/* Checkpoint / resume. A saved state is the handle's state between steps as
+ * Alg. 1 defines it (any pending aggregation applied first): w_t,
+ * w_t - w_{t-1}, every residual e_{t,k}, Alg. 3's server momentum, the step t,
+ * eta, seed, lambda, the RBGS mode, the selection engine and the cumulative
+ * counters, behind a fixed header (magic "GMCSTATE", version 1) holding d, K,
+ * the compressor, ratio, block and variant. Host memory, little-endian fp32.
+ *
+ * gmc_state_bytes -- bytes gmc_save_state writes for this handle (-1: invalid
+ * handle). */
+int64_t gmc_state_bytes(gmc_t h);
+
+/* gmc_save_state -- synchronising. Writes gmc_state_bytes(h) bytes to host_out
+ * (any host memory, capacity bytes). GMC_EINVAL if capacity is too small,
+ * GMC_ESTATE before gmc_set_params. */
+int gmc_save_state(gmc_t h, void* host_out, int64_t capacity);
+
+/* gmc_load_state -- synchronising. Replaces the handle's state with a saved one
+ * (bytes long). The handle must have been created with the same d, K,
+ * compressor, ratio (and block for RBGS) and set to the same variant: else, or
+ * for a malformed buffer, GMC_EINVAL and the state is left as it was. The next
+ * gmc_step continues the saved trajectory exactly (it reads w_t - w_{t-1}
+ * densely once, as no pair lists of the step before were saved);
+ * gmc_get_selected returns GMC_ESTATE until that step. */
+int gmc_load_state(gmc_t h, const void* host_in, int64_t bytes);
+
 /* gmc_check -- synchronising. GMC_OK, or the first data-dependent error recorded
  * since gmc_set_params (GMC_ENONFINITE, GMC_EINTERNAL), or GMC_ECUDA. */
 int gmc_check(gmc_t h);

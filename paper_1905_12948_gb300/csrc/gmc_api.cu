@@ -52,6 +52,7 @@ struct gmc_ctx {
   // state
   int64_t t = 0;
   bool initialized = false;
+  bool restored = false;  // gmc_load_state: the next step reads w_t - w_{t-1} densely
   float* e = nullptr;
   float* w = nullptr;
   float* dlt = nullptr;
@@ -228,7 +229,8 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.sample_rank = h->sample_rank;
   A.sample_chunks = h->sample_chunks;
   A.sample_blocks = h->sample_blocks;
-  A.has_prev = t > 0;
+  A.dense_prev = h->restored && t == h->t ? 1 : 0;
+  A.has_prev = t > 0 && !A.dense_prev;
   A.dense_mode = h->select_mode == GMC_SELECT_DENSE;
   A.sel = h->sel;
   A.ghist = h->ghist;
@@ -361,6 +363,9 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
   } else {
     RbgsArgs A = rbgs_args(h, grads);
     A.g_direct = direct ? 1 : 0;
+    // restored state: w_t - w_{t-1} may be non-zero in any block (zero outside
+    // the last union, where dlt holds it): flag every block as the last union's
+    if (h->restored && h->t > 0) GMC_TRY(cudaMemsetAsync(A.uflag_prev, 1, (size_t)h->nb, s));
     GMC_TRY(cudaMemsetAsync(A.uflag_cur, 0, (size_t)h->nb, s));
     GMC_TRY(timed(h, GMC_KERNEL_RBGS_PICK, 0.0, s, [&] { return launch_rbgs_pick(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_RBGS_STEP, 12.0 * Kd, s,
@@ -374,6 +379,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
                 [&] { return launch_finalize(h->step_ctr, h->total_ctr, pairs_add, s); }));
   if (h->ev_step) GMC_TRY(cudaEventRecord(h->ev_step, s));
   h->t += 1;
+  h->restored = false;
   return GMC_OK;
 }
 
@@ -667,13 +673,14 @@ int gmc_set_detach_output(gmc_t h, float* out_dev, int64_t ld) {
   return GMC_OK;
 }
 
-int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
-  if (!h || !w0_dev) return GMC_EINVAL;
-  DeviceGuard g(h->device);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
+}  // extern "C"
+
+namespace {
+// Everything but w back to the start of Alg. 1 (e = 0, w_{-1} = w_0, t = 0,
+// counters cleared), on stream s.
+int reset_state(gmc_ctx* h, cudaStream_t s) {
   GMC_TRY(order_after_flush(h, s, true));
   h->agg_pending = false;  // a pending aggregation of the old state is dropped
-  GMC_TRY(cudaMemcpyAsync(h->w, w0_dev, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice, s));
   GMC_TRY(cudaMemsetAsync(h->e, 0, (size_t)h->K * h->ld * sizeof(float), s));
   GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
   if (h->mom) GMC_TRY(cudaMemsetAsync(h->mom, 0, (size_t)h->ld * sizeof(float), s));
@@ -689,7 +696,20 @@ int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
   GMC_TRY(cudaMemsetAsync(h->total_ctr, 0, sizeof(Counters), s));
   GMC_TRY(cudaMemsetAsync(h->status, 0, sizeof(unsigned), s));
   h->t = 0;
+  h->restored = false;
   h->initialized = true;
+  return GMC_OK;
+}
+}  // namespace
+
+extern "C" {
+
+int gmc_set_params(gmc_t h, const float* w0_dev, void* stream) {
+  if (!h || !w0_dev) return GMC_EINVAL;
+  DeviceGuard g(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  GMC_TRY_ST(reset_state(h, s));
+  GMC_TRY(cudaMemcpyAsync(h->w, w0_dev, (size_t)h->d * sizeof(float), cudaMemcpyDeviceToDevice, s));
   return GMC_OK;
 }
 
@@ -759,7 +779,7 @@ int64_t gmc_selected_capacity(gmc_t h) {
 int gmc_get_selected(gmc_t h, int32_t k, uint32_t* idx_dev, float* val_dev, int64_t capacity,
                      int64_t* count_host, void* stream) {
   if (!h || !idx_dev || !val_dev || !count_host || k < 0 || k >= h->K) return GMC_EINVAL;
-  if (!h->initialized || h->t == 0) return GMC_ESTATE;
+  if (!h->initialized || h->t == 0 || h->restored) return GMC_ESTATE;
   DeviceGuard g(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (h->compressor != GMC_RBGS) {
@@ -820,6 +840,136 @@ int gmc_get_stats(gmc_t h, uint64_t* counters_host, int32_t n, double* rcc_host)
     }
     *rcc_host = r;
   }
+  return GMC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// checkpoint / resume
+// ---------------------------------------------------------------------------
+namespace {
+// Fixed-layout header of a saved state, followed by w (d floats), w_t - w_{t-1}
+// (d floats), the K residual rows (d floats each) and, for Alg. 3, the server's
+// w_t - w_{t-1} (d floats); all little-endian fp32 as the GPU holds them.
+struct StateHeader {
+  char magic[8];
+  uint32_t version, header_bytes;
+  int64_t d;
+  int32_t K, compressor;
+  double ratio;
+  int64_t block;
+  int32_t variant, per_worker;
+  uint64_t seed;
+  int64_t t;
+  float beta, eta, lambda;
+  int32_t select_mode;
+  uint64_t totals[8];
+  uint32_t status, has_mom;
+};
+constexpr char kMagic[8] = {'G', 'M', 'C', 'S', 'T', 'A', 'T', 'E'};
+constexpr uint32_t kStateVersion = 1;
+
+int64_t state_bytes(const gmc_ctx* h) {
+  const int64_t rows = (int64_t)(2 + h->K) + (h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1 : 0);
+  return (int64_t)sizeof(StateHeader) + rows * h->d * (int64_t)sizeof(float);
+}
+}  // namespace
+
+int64_t gmc_state_bytes(gmc_t h) {
+  if (!h) return -1;
+  return state_bytes(h);
+}
+
+int gmc_save_state(gmc_t h, void* host_out, int64_t capacity) {
+  if (!h || !host_out) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  if (capacity < state_bytes(h)) return GMC_EINVAL;
+  DeviceGuard g(h->device);
+  GMC_TRY_ST(flush(h, h->aux));  // the state Alg. 1 defines: no aggregation left pending
+  GMC_TRY(cudaDeviceSynchronize());
+  StateHeader H;
+  std::memset(&H, 0, sizeof(H));
+  std::memcpy(H.magic, kMagic, sizeof(kMagic));
+  H.version = kStateVersion;
+  H.header_bytes = (uint32_t)sizeof(StateHeader);
+  H.d = h->d;
+  H.K = h->K;
+  H.compressor = h->compressor;
+  H.ratio = h->ratio;
+  H.block = h->block;
+  H.variant = h->variant;
+  H.per_worker = h->per_worker;
+  H.seed = h->seed;
+  H.t = h->t;
+  H.beta = h->beta;
+  H.eta = h->eta;
+  H.lambda = h->lambda;
+  H.select_mode = h->select_mode;
+  Counters c;
+  GMC_TRY(cudaMemcpy(&c, h->total_ctr, sizeof(Counters), cudaMemcpyDeviceToHost));
+  for (int i = 0; i < 8; ++i) H.totals[i] = c.v[i];
+  GMC_TRY(cudaMemcpy(&H.status, h->status, sizeof(unsigned), cudaMemcpyDeviceToHost));
+  H.has_mom = h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1u : 0u;
+  char* out = static_cast<char*>(host_out);
+  std::memcpy(out, &H, sizeof(H));
+  const size_t row = (size_t)h->d * sizeof(float);
+  char* p = out + sizeof(H);
+  GMC_TRY(cudaMemcpy(p, h->w, row, cudaMemcpyDeviceToHost));
+  p += row;
+  // w_t - w_{t-1}: where the step left it (dlt, zero outside the last union),
+  // or, for Alg. 3, the server's dense copy (dlt is zero between its steps)
+  GMC_TRY(cudaMemcpy(p, h->dlt, row, cudaMemcpyDeviceToHost));
+  p += row;
+  GMC_TRY(cudaMemcpy2D(p, row, h->e, (size_t)h->ld * sizeof(float), row, (size_t)h->K,
+                       cudaMemcpyDeviceToHost));
+  p += row * h->K;
+  if (H.has_mom) GMC_TRY(cudaMemcpy(p, h->mom, row, cudaMemcpyDeviceToHost));
+  return GMC_OK;
+}
+
+int gmc_load_state(gmc_t h, const void* host_in, int64_t bytes) {
+  if (!h || !host_in || bytes < (int64_t)sizeof(StateHeader)) return GMC_EINVAL;
+  StateHeader H;
+  std::memcpy(&H, host_in, sizeof(H));
+  if (std::memcmp(H.magic, kMagic, sizeof(kMagic)) != 0 || H.version != kStateVersion ||
+      H.header_bytes != sizeof(StateHeader))
+    return GMC_EINVAL;
+  // the handle must have been created for the same problem and form
+  if (H.d != h->d || H.K != h->K || H.compressor != h->compressor || H.ratio != h->ratio ||
+      (h->compressor == GMC_RBGS && H.block != h->block) || H.variant != h->variant ||
+      H.t < 0 || H.has_mom != (h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1u : 0u))
+    return GMC_EINVAL;
+  if (bytes < state_bytes(h)) return GMC_EINVAL;
+  if (!finite_f(H.eta) || !(H.eta > 0.f) || !finite_f(H.lambda) || H.lambda < 0.f || H.lambda > 1.f ||
+      (H.per_worker != 0 && H.per_worker != 1) ||
+      (H.select_mode != GMC_SELECT_SAMPLED && H.select_mode != GMC_SELECT_DENSE))
+    return GMC_EINVAL;
+  DeviceGuard g(h->device);
+  GMC_TRY(cudaDeviceSynchronize());
+  const char* p = static_cast<const char*>(host_in) + sizeof(H);
+  GMC_TRY_ST(reset_state(h, h->aux));  // as gmc_set_params: e, dlt, mom, tables, counters cleared
+  GMC_TRY(cudaStreamSynchronize(h->aux));
+  const size_t row = (size_t)h->d * sizeof(float);
+  GMC_TRY(cudaMemcpy(h->w, p, row, cudaMemcpyHostToDevice));
+  p += row;
+  GMC_TRY(cudaMemcpy(h->dlt, p, row, cudaMemcpyHostToDevice));
+  p += row;
+  GMC_TRY(cudaMemcpy2D(h->e, (size_t)h->ld * sizeof(float), p, row, row, (size_t)h->K,
+                       cudaMemcpyHostToDevice));
+  p += row * h->K;
+  if (H.has_mom) GMC_TRY(cudaMemcpy(h->mom, p, row, cudaMemcpyHostToDevice));
+  Counters c;
+  for (int i = 0; i < 8; ++i) c.v[i] = H.totals[i];
+  GMC_TRY(cudaMemcpy(h->total_ctr, &c, sizeof(Counters), cudaMemcpyHostToDevice));
+  unsigned st = H.status;
+  GMC_TRY(cudaMemcpy(h->status, &st, sizeof(unsigned), cudaMemcpyHostToDevice));
+  h->seed = H.seed;
+  h->per_worker = H.per_worker;
+  h->eta = H.eta;
+  h->lambda = H.lambda;
+  h->select_mode = H.select_mode;
+  h->t = H.t;
+  h->restored = H.t > 0;
+  GMC_TRY(cudaDeviceSynchronize());
   return GMC_OK;
 }
 

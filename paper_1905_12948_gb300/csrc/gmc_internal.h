@@ -61,7 +61,8 @@ struct TopkArgs {
   int64_t t;
   uint32_t limit;
   int theta_blocks;          // blocks per worker of k_sample_theta
-  int has_prev;              // a previous step exists (t > 0)
+  int has_prev;              // a previous step's pair lists exist (t > 0, not just restored)
+  int dense_prev;            // restored state: w_t - w_{t-1} is in dlt over [0, d), no pair lists
   int dense_mode;            // GMC_SELECT_DENSE
   WorkerSel* sel;            // K entries
   uint32_t* ghist;           // K x kHistBins: the sample's histogram (zero between uses)

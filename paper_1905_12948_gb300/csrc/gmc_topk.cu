@@ -424,10 +424,30 @@ __global__ void __launch_bounds__(kThreads) k_sample_theta(TopkArgs A) {
 // tile; for each worker it writes v over e and appends its candidates as one
 // index-sorted sub-chunk, reserved at once -- warps never wait for each other.
 // ---------------------------------------------------------------------------
+// A restored state (gmc_load_state): w_t - w_{t-1} is in dlt over the whole
+// range, with no pair lists of the step before. Read it densely for one warp's
+// sub-tile [sub0, sub0 + n) (n a multiple of 4, sub0 16-byte aligned, inside
+// ld) and clear it, as the listed path does.
+__device__ __forceinline__ void stage_delta_dense(const TopkArgs& A, uint32_t sub0, int n, float* dlw,
+                                                  int lane) {
+  for (int i = lane; i < n / 4; i += 32) {
+    float4* p = reinterpret_cast<float4*>(A.dlt + sub0) + i;
+    const float4 x = *p;
+    reinterpret_cast<float4*>(dlw)[i] = x;
+    if ((__float_as_uint(x.x) | __float_as_uint(x.y) | __float_as_uint(x.z) | __float_as_uint(x.w)) != 0u)
+      *p = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncwarp();
+}
+
 // w_t - w_{t-1} on one warp's sub-tile [sub0, sub0 + n) into dlw: non-zero only
 // where the previous step sent pairs, listed by its sub-chunks (k', tile, w).
 __device__ __forceinline__ void stage_delta_warp(const TopkArgs& A, int64_t tile, int w,
                                                  uint32_t sub0, int n, float* dlw, int lane) {
+  if (A.dense_prev) {
+    stage_delta_dense(A, sub0, n, dlw, lane);
+    return;
+  }
   for (int i = lane; i < n / 4; i += 32)
     reinterpret_cast<float4*>(dlw)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
   __syncwarp();
@@ -933,7 +953,9 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     if (lead) {
       uint32_t up = ~0u;
       bool many = false;
-      if (p0.total <= 32u) {
+      if (A.dense_prev) {  // restored state: no pairs, w_t - w_{t-1} read densely
+        stage_delta_dense(A, s0, kSub, dlw, lane);
+      } else if (p0.total <= 32u) {
         up = apply_pairs(A, s0, p0, sm.Tp, sm.tip, w0, dlw, mkw, lane, lt, uni, chg);
       } else if (A.pending) {
         stage_pending_warp(A, tile, sw, s0, kSub, dlw, mkw, lane, uni, chg);

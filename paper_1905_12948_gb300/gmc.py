@@ -40,6 +40,9 @@ _SIGNATURES = {
     "gmc_set_eta": (ctypes.c_int, [_c_p, _f32]),
     "gmc_set_select_mode": (ctypes.c_int, [_c_p, _i32]),
     "gmc_set_variant": (ctypes.c_int, [_c_p, _i32]),
+    "gmc_state_bytes": (_i64, [_c_p]),
+    "gmc_save_state": (ctypes.c_int, [_c_p, _c_p, _i64]),
+    "gmc_load_state": (ctypes.c_int, [_c_p, _c_p, _i64]),
     "gmc_set_detach_output": (ctypes.c_int, [_c_p, _c_p, _i64]),
     "gmc_set_params": (ctypes.c_int, [_c_p, _c_p, _c_p]),
     "gmc_step": (ctypes.c_int, [_c_p, _c_p, _c_p]),
@@ -221,6 +224,20 @@ class GMC:
         out = {name: int(arr[i]) for i, name in enumerate(STAT_NAMES[:7])}
         out["rcc"] = rcc.value
         return out
+
+    def save_state(self):
+        """The handle's state between steps (gmc_save_state) as a numpy uint8 array."""
+        import numpy as np
+        n = int(self.lib.gmc_state_bytes(self.h))
+        buf = np.empty(n, np.uint8)
+        _check(self.lib.gmc_save_state(self.h, buf.ctypes.data, n), "gmc_save_state")
+        return buf
+
+    def load_state(self, buf) -> None:
+        """Continue from a state saved by save_state (gmc_load_state)."""
+        import numpy as np
+        buf = np.ascontiguousarray(buf, np.uint8)
+        _check(self.lib.gmc_load_state(self.h, buf.ctypes.data, buf.size), "gmc_load_state")
 
     def check(self) -> int:
         return int(self.lib.gmc_check(self.h))
