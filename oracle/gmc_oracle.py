@@ -28,6 +28,14 @@ Communication in Distributed Learning", arXiv 1905.12948):
       Alg. 4 (learning rate inside the residual):
         e_{t+1/2,k} = e_{t,k} + eta g_{t,k} - beta (w_t - w_{t-1});
         w_{t+1} = w_t - (1/K) sum_k C(e_{t+1/2,k}).
+  * The local-momentum baseline the paper compares against (Sec. 2.3, eq. (3),
+    with error feedback: DGC without momentum factor masking, Sec. 3.1):
+        m_{t+1,k} = beta m_{t,k} + eta g_{t,k},  m_{0,k} = 0
+        e_{t+1/2,k} = e_{t,k} + m_{t+1,k}; C and the residual as in Alg. 1;
+        w_{t+1} = w_t - (1/K) sum_k C(e_{t+1/2,k});
+    with masking (DGC w/ mfm), m_{t+1,k} is also set to 0 where worker k sent;
+    the detached point of the DEF-A-like form is w_{t,k} = w_t - lambda e_{t,k}
+    (the residual already carries eta).
 
 Precision. The paper fixes none. Top-s turns floating-point magnitudes into an
 integer decision (which indices are sent), so that decision is taken in the
@@ -78,6 +86,8 @@ TOPK_APPROX = "topk_approx"
 ALG1 = "gmc"               # Algorithm 1 (the method)
 ALG3 = "server_momentum"   # Algorithm 3: momentum term on the server
 ALG4 = "lr_in_residual"    # Algorithm 4: learning rate inside the residual
+LOCAL = "local_momentum"   # local momentum with error feedback (DGC w/o mfm)
+LOCAL_MFM = "local_momentum_mfm"  # the same with momentum factor masking (DGC w/ mfm)
 
 APPROX_SAMPLE_DIV = 100  # |S| = d/100 (Sec. 5.1)
 
@@ -269,10 +279,12 @@ class GMC:
             raise ValueError("ratio must be in (0, 1]")
         if compressor not in (TOPK, RBGS, TOPK_APPROX):
             raise ValueError("unknown compressor")
-        if variant not in (ALG1, ALG3, ALG4):
+        if variant not in (ALG1, ALG3, ALG4, LOCAL, LOCAL_MFM):
             raise ValueError("unknown variant")
-        if variant != ALG1 and (compressor == RBGS or lam != 0.0):
-            raise ValueError("the appendix variants are GMC with a top-s compressor")
+        if variant != ALG1 and compressor == RBGS:
+            raise ValueError("the variants take a top-s compressor")
+        if variant in (ALG3, ALG4) and lam != 0.0:
+            raise ValueError("GMC+ detaches Alg. 1 only")
         self.variant = variant
         self.d, self.K = d, K
         self.beta = F32(beta)
@@ -303,9 +315,11 @@ class GMC:
         self.eta = F32(eta)
         self.c = F32(self.beta / self.eta)          # beta / eta
         self.a = F32(self.eta / F32(self.K))        # eta / K
-        if self.variant == ALG4:
+        if self.variant in (ALG4, LOCAL, LOCAL_MFM):
             self.a = F32(F32(1.0) / F32(self.K))    # 1 / K
         self.b = F32(self.lam * self.eta)           # lambda * eta
+        if self.variant in (LOCAL, LOCAL_MFM):
+            self.b = self.lam                       # lambda (e carries eta)
 
     def set_params(self, w0: np.ndarray) -> None:
         """Initial state: w_{-1} = w_0 and e_{0,k} = 0 (Alg. 1 and Alg. 2)."""
@@ -315,6 +329,7 @@ class GMC:
         self.w = w0.copy()
         self.w_prev = w0.copy()
         self.e = np.zeros((self.K, self.d), F32)
+        self.u = np.zeros((self.K, self.d), F32)    # local momentum m_{t,k} (local variants)
         self.t = 0
         self.totals = dict(steps=0, pairs=0, nnz=0, union=0, changed=0)
 
@@ -338,8 +353,11 @@ class GMC:
             e_half = (self.e + g) - self.c * (self.w - self.w_prev)
         elif self.variant == ALG3:   # e_{t,k} + g_{t,k}
             e_half = self.e + g
-        else:                        # e_{t,k} + eta g_{t,k} - beta (w_t - w_{t-1})
+        elif self.variant == ALG4:   # e_{t,k} + eta g_{t,k} - beta (w_t - w_{t-1})
             e_half = (self.e + self.eta * g) - self.beta * (self.w - self.w_prev)
+        else:                        # m = beta m + eta g; e_{t,k} + m_{t+1,k}
+            m_next = self.beta * self.u + self.eta * g
+            e_half = self.e + m_next
 
         # workers: C(e_{t+1/2,k}) -- its support and values
         blocks = sample = thresholds = None
@@ -361,6 +379,11 @@ class GMC:
         e_next = e_half.copy()
         for k in range(K):
             e_next[k, supports[k]] = F32(0.0)
+        if self.variant in (LOCAL, LOCAL_MFM):
+            if self.variant == LOCAL_MFM:  # momentum factor masking
+                for k in range(K):
+                    m_next[k, supports[k]] = F32(0.0)
+            self.u = m_next
 
         # server: w_{t+1} = w_t - (eta/K) sum_k C(e_{t+1/2,k}), workers summed in order
         # (Alg. 4: 1/K in a; Alg. 3 adds beta (w_t - w_{t-1}))

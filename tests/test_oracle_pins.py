@@ -530,6 +530,100 @@ def test_alg4_is_gmc_scaled_under_constant_eta():
         np.testing.assert_allclose(b.w, a.w, rtol=1e-5, atol=1e-6)
 
 
+# ---------------------------------------------------------------------------
+# The local-momentum baseline (Sec. 2.3 eq. (3) with error feedback: DGC w/o
+# and w/ momentum factor masking)
+# ---------------------------------------------------------------------------
+
+def test_local_momentum_without_compression_is_serial_msgd():
+    """Sec. 2.3: local momentum without sparsification is serial MSGD (the
+    heavy-ball recursion), with e = 0 exactly."""
+    rng = np.random.default_rng(41)
+    d, K, T, eta, beta = 129, 4, 40, 0.05, 0.9
+    o = GMC(d, K, beta=beta, eta=eta, compressor=TOPK, ratio=1.0, variant=oracle.LOCAL)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    o.set_params(w0)
+    grads = _grads(rng, T, K, d)
+    eta32, beta32 = float(np.float32(eta)), float(np.float32(beta))
+    ref = _heavy_ball(w0.astype(np.float64), [g.astype(np.float64) for g in grads], eta32, beta32)
+    m_abs = np.zeros((K, d))
+    budget = np.zeros(d)
+    for t, g in enumerate(grads):
+        w_t = o.w.astype(np.float64)
+        o.step(g)
+        assert not np.any(o.e)
+        m_abs = beta32 * m_abs + eta32 * np.abs(g.astype(np.float64))
+        budget += 6 * U * (np.abs(o.w.astype(np.float64)) + np.abs(w_t) + (K + 3) / K * m_abs.sum(0))
+        np.testing.assert_array_less(np.abs(o.w - ref[t + 1]), 2 * budget / (1 - beta32) + 1e-30)
+
+
+def test_momentum_factor_masking_without_compression_is_sgd():
+    """Sec. 3.1's remark: with momentum factor masking and no sparsification,
+    every coordinate is sent each step, the momentum is reset, and the method
+    is plain distributed SGD: w_{t+1} = w_t - eta * mean_k g_{t,k}."""
+    rng = np.random.default_rng(42)
+    d, K, T, eta = 257, 3, 20, 0.1
+    o = GMC(d, K, beta=0.9, eta=eta, compressor=TOPK, ratio=1.0, variant=oracle.LOCAL_MFM)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    o.set_params(w0)
+    w_ref = w0.astype(np.float64)
+    tol = np.zeros(d)
+    eta32 = float(np.float32(eta))
+    for g in _grads(rng, T, K, d):
+        o.step(g)
+        assert not np.any(o.e) and not np.any(o.u)
+        g64 = g.astype(np.float64)
+        w_ref = w_ref - eta32 / K * g64.sum(0)
+        tol += (K + 3) * U * eta32 / K * np.abs(g64).sum(0) + 2 * U * np.abs(o.w)
+        np.testing.assert_array_less(np.abs(o.w - w_ref), 2 * tol + 1e-30)
+
+
+@pytest.mark.parametrize("variant", [oracle.LOCAL, oracle.LOCAL_MFM])
+def test_local_momentum_update_rule(variant):
+    """With C eliminated: w_{t+1} - w_t = -ebar_t - mbar_{t+1} + ebar_{t+1},
+    and the momentum follows m_{t+1} = beta m_t + eta g off the sent
+    coordinates (and is 0 on them with masking)."""
+    rng = np.random.default_rng(43)
+    d, K, T, eta, beta = 500, 4, 25, 0.1, 0.9
+    o = GMC(d, K, beta=beta, eta=eta, compressor=TOPK, ratio=0.03, variant=variant)
+    o.set_params(rng.standard_normal(d).astype(np.float32))
+    eta32, beta32 = float(np.float32(eta)), float(np.float32(beta))
+    for g in _grads(rng, T, K, d):
+        w_t, e_t, m_t = (x.astype(np.float64) for x in (o.w, o.e, o.u))
+        r = o.step(g)
+        w_n, e_n, m_n = (x.astype(np.float64) for x in (o.w, o.e, o.u))
+        m_new = beta32 * m_t + eta32 * g.astype(np.float64)
+        sent = np.zeros((K, d), bool)
+        for k in range(K):
+            sent[k, r.supports[k]] = True
+        mb = 4 * U * (beta32 * np.abs(m_t) + eta32 * np.abs(g))
+        want = np.where(sent, 0.0, m_new) if variant == oracle.LOCAL_MFM else m_new
+        np.testing.assert_array_less(np.abs(m_n - want), mb + 1e-30)
+        lhs = w_n - w_t
+        rhs = -e_t.mean(0) - m_new.mean(0) + e_n.mean(0)
+        scale = (np.abs(e_t) + np.abs(m_new) + np.abs(r.e_half) + np.abs(e_n)).sum(0)
+        budget = 8 * U * (np.abs(w_n) + np.abs(w_t) + (K + 3) / K * scale)
+        np.testing.assert_array_less(np.abs(lhs - rhs), budget + 1e-30)
+
+
+def test_local_momentum_at_beta_zero_is_alg4():
+    """Bitwise: with beta = 0 the local momentum is eta g and the step is
+    Alg. 4's (which then has no momentum term either)."""
+    rng = np.random.default_rng(44)
+    d, K = 400, 3
+    a = GMC(d, K, beta=0.0, eta=0.3, compressor=TOPK, ratio=0.05, variant=oracle.ALG4)
+    b = GMC(d, K, beta=0.0, eta=0.3, compressor=TOPK, ratio=0.05, variant=oracle.LOCAL)
+    w0 = rng.standard_normal(d).astype(np.float32)
+    a.set_params(w0)
+    b.set_params(w0)
+    for g in _grads(rng, 8, K, d):
+        ra, rb = a.step(g), b.step(g)
+        for k in range(K):
+            np.testing.assert_array_equal(ra.supports[k], rb.supports[k])
+        assert np.array_equal(a.w.view(np.uint32), b.w.view(np.uint32))
+        assert np.array_equal(a.e.view(np.uint32), b.e.view(np.uint32))
+
+
 def test_variants_refuse_gmcplus_and_rbgs():
     with pytest.raises(ValueError):
         GMC(10, 2, 0.9, 0.1, compressor=RBGS, block=2, variant=oracle.ALG3)
