@@ -81,6 +81,13 @@ typedef struct gmc_ctx* gmc_t;
 #define GMC_VARIANT_LR_IN_RESIDUAL   2 /* Alg. 4: e_{t+1/2,k} = (e_{t,k} + eta g_{t,k})
                                                              - beta (w_t - w_{t-1});
                                           w_{t+1} = w_t - fl(1/K) sum_k C_k */
+/* The local-momentum baseline the paper compares against (Sec. 2.3 eq. (3) with
+ * error feedback; DGC without / with momentum factor masking, Sec. 3.1):
+ *   m_{t+1,k} = beta m_{t,k} + eta g_{t,k} (m_{0,k} = 0), e_{t+1/2,k} = e_{t,k} + m_{t+1,k},
+ *   w_{t+1} = w_t - fl(1/K) sum_k C_k; with masking, m_{t+1,k} = 0 where worker k sent.
+ *   Its detached point (DEF-A-like, lambda > 0) is w_{t,k} = w_t - lambda e_{t,k}. */
+#define GMC_VARIANT_LOCAL_MOMENTUM      3
+#define GMC_VARIANT_LOCAL_MOMENTUM_MFM  4
 
 /* Top-k selection engines; both give identical results. */
 #define GMC_SELECT_SAMPLED 0 /* default: a sampled threshold filters candidates in the one
@@ -132,7 +139,8 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta,
 void gmc_destroy(gmc_t h);
 
 /* gmc_set_lambda -- GMC+ detach coefficient lambda in [0,1] (Alg. 2); 0 is GMC.
- * GMC_EINVAL for lambda != 0 under an appendix variant (GMC+ detaches Alg. 1). */
+ * GMC_EINVAL for lambda != 0 under Alg. 3 / Alg. 4 (GMC+ detaches Alg. 1); the
+ * local-momentum baseline detaches as w_t - lambda e_{t,k}. */
 int gmc_set_lambda(gmc_t h, float lambda);
 
 /* gmc_set_rbgs_mode -- 0: one block choice per step shared by all workers, as in
@@ -149,13 +157,16 @@ int gmc_set_seed(gmc_t h, uint64_t seed);
 int gmc_set_eta(gmc_t h, float eta);
 
 /* gmc_set_variant -- the step's form (GMC_VARIANT_*; default Alg. 1). Only for the
- * top-k compressors (exact and approximate) with lambda = 0, and only before the
- * first step after gmc_create or gmc_set_params (GMC_ESTATE otherwise), since the
- * residuals mean another thing under each form. GMC_VARIANT_SERVER_MOMENTUM
- * allocates d floats of w_t - w_{t-1} (GMC_ENOMEM if that fails) and turns off
- * the deferred aggregation: every step ends with a dense pass over w. Synchronising
- * when it allocates. Arithmetic: each operation rounded once, in the order written
- * beside the GMC_VARIANT_* constants. */
+ * top-k compressors (exact and approximate), with lambda = 0 for Alg. 3 / Alg. 4,
+ * and only before the first step after gmc_create or gmc_set_params (GMC_ESTATE
+ * otherwise), since the residuals mean another thing under each form.
+ * GMC_VARIANT_SERVER_MOMENTUM allocates d floats of w_t - w_{t-1} and turns off
+ * the deferred aggregation: every step ends with a dense pass over w. The
+ * local-momentum variants allocate K x d floats of momentum (read and written
+ * by every step's dense pass); masking turns off the deferred aggregation.
+ * GMC_ENOMEM if an allocation fails; synchronising when it allocates.
+ * Arithmetic: each operation rounded once, in the order written beside the
+ * GMC_VARIANT_* constants. */
 int gmc_set_variant(gmc_t h, int32_t variant);
 
 /* gmc_set_select_mode -- GMC_SELECT_SAMPLED (default) or GMC_SELECT_DENSE (exact

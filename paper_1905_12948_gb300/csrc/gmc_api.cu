@@ -38,6 +38,7 @@ struct gmc_ctx {
   int select_mode = GMC_SELECT_SAMPLED;
   int variant = GMC_VARIANT_GMC;  // Alg. 1, or the appendix's Alg. 3 / Alg. 4
   float* mom = nullptr;           // Alg. 3: w_t - w_{t-1} (allocated by gmc_set_variant)
+  float* lm = nullptr;            // local momentum: K rows of ld (allocated by gmc_set_variant)
   float* detach_out = nullptr;
   int64_t detach_ld = 0;
   // geometry
@@ -193,6 +194,13 @@ void drain_profile(gmc_ctx* h) {
   h->pending.clear();
 }
 
+bool local_variant(const gmc_ctx* h) {
+  return h->variant == GMC_VARIANT_LOCAL_MOMENTUM || h->variant == GMC_VARIANT_LOCAL_MOMENTUM_MFM;
+}
+// Detach coefficient: fl(lambda*eta) (Alg. 2); lambda for the local-momentum
+// baseline, whose residual already carries eta.
+float detach_b(const gmc_ctx* h) { return local_variant(h) ? h->lambda : h->lambda * h->eta; }
+
 void set_constants(gmc_ctx* h, TopkArgs* A) {
   A->c = h->beta / h->eta;
   A->a = h->eta / (float)h->K;
@@ -206,6 +214,13 @@ void set_constants(gmc_ctx* h, TopkArgs* A) {
     A->a = 1.f / (float)h->K;
     A->gscale = 1;
     A->gs = h->eta;
+  } else if (h->variant == GMC_VARIANT_LOCAL_MOMENTUM || h->variant == GMC_VARIANT_LOCAL_MOMENTUM_MFM) {
+    A->c = 0.f;  // e + m, m = beta*m + eta*g; w -= (1/K) sum
+    A->a = 1.f / (float)h->K;
+    A->gs = h->eta;
+    A->local_mom = 1;
+    A->mfm = h->variant == GMC_VARIANT_LOCAL_MOMENTUM_MFM ? 1 : 0;
+    A->lm = h->lm;
   }
 }
 
@@ -334,7 +349,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
     A.g_direct = direct ? 1 : 0;
     A.pending = h->agg_pending ? 1 : 0;
     A.a_prev = h->a_pending;
-    const bool defer = h->tile == kBulkTile && !eager && !h->detach_out && !A.server_mom;
+    const bool defer = h->tile == kBulkTile && !eager && !h->detach_out && !A.server_mom && !A.mfm;
     const double kk = (double)h->K * (double)h->ksel;
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
     GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
@@ -372,7 +387,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
                   [&] { return launch_rbgs_step(A, h->grid_rbgs, s); }));
   }
   if (h->detach_out) {
-    DetachArgs D{h->w, h->e, h->ld, h->d, h->lambda * h->eta, h->detach_out, h->detach_ld, 0, h->K};
+    DetachArgs D{h->w, h->e, h->ld, h->d, detach_b(h), h->detach_out, h->detach_ld, 0, h->K};
     GMC_TRY(timed(h, GMC_KERNEL_DETACH, 8.0 * Kd + 4.0 * h->d, s, [&] { return launch_detach(D, s); }));
   }
   GMC_TRY(timed(h, GMC_KERNEL_OTHER, 0.0, s,
@@ -617,7 +632,9 @@ void gmc_destroy(gmc_t h) {
 
 int gmc_set_lambda(gmc_t h, float lambda) {
   if (!h || !finite_f(lambda) || lambda < 0.f || lambda > 1.f) return GMC_EINVAL;
-  if (lambda != 0.f && h->variant != GMC_VARIANT_GMC) return GMC_EINVAL;  // GMC+ detaches Alg. 1
+  // GMC+ detaches Alg. 1; the local-momentum baseline detaches as DEF-A does
+  if (lambda != 0.f && (h->variant == GMC_VARIANT_SERVER_MOMENTUM || h->variant == GMC_VARIANT_LR_IN_RESIDUAL))
+    return GMC_EINVAL;
   h->lambda = lambda;
   return GMC_OK;
 }
@@ -642,15 +659,20 @@ int gmc_set_eta(gmc_t h, float eta) {
 
 int gmc_set_variant(gmc_t h, int32_t variant) {
   if (!h) return GMC_EINVAL;
-  if (variant != GMC_VARIANT_GMC && variant != GMC_VARIANT_SERVER_MOMENTUM &&
-      variant != GMC_VARIANT_LR_IN_RESIDUAL)
+  if (variant < GMC_VARIANT_GMC || variant > GMC_VARIANT_LOCAL_MOMENTUM_MFM) return GMC_EINVAL;
+  if (variant != GMC_VARIANT_GMC && h->compressor == GMC_RBGS) return GMC_EINVAL;
+  if ((variant == GMC_VARIANT_SERVER_MOMENTUM || variant == GMC_VARIANT_LR_IN_RESIDUAL) && h->lambda != 0.f)
     return GMC_EINVAL;
-  if (variant != GMC_VARIANT_GMC && (h->compressor == GMC_RBGS || h->lambda != 0.f)) return GMC_EINVAL;
   if (h->initialized && h->t > 0) return GMC_ESTATE;  // the residuals mean another thing
   if (variant == GMC_VARIANT_SERVER_MOMENTUM && !h->mom) {
     DeviceGuard g(h->device);
     cudaError_t err = dalloc(h, &h->mom, (size_t)h->ld);
     if (err == cudaSuccess) err = cudaMemset(h->mom, 0, (size_t)h->ld * sizeof(float));
+    if (err != cudaSuccess) return status_of(err);
+  }
+  if ((variant == GMC_VARIANT_LOCAL_MOMENTUM || variant == GMC_VARIANT_LOCAL_MOMENTUM_MFM) && !h->lm) {
+    DeviceGuard g(h->device);
+    cudaError_t err = dalloc(h, &h->lm, (size_t)h->K * h->ld);
     if (err != cudaSuccess) return status_of(err);
   }
   h->variant = variant;
@@ -684,6 +706,7 @@ int reset_state(gmc_ctx* h, cudaStream_t s) {
   GMC_TRY(cudaMemsetAsync(h->e, 0, (size_t)h->K * h->ld * sizeof(float), s));
   GMC_TRY(cudaMemsetAsync(h->dlt, 0, (size_t)h->ld * sizeof(float), s));
   if (h->mom) GMC_TRY(cudaMemsetAsync(h->mom, 0, (size_t)h->ld * sizeof(float), s));
+  if (h->lm) GMC_TRY(cudaMemsetAsync(h->lm, 0, (size_t)h->K * h->ld * sizeof(float), s));
   if (h->compressor != GMC_RBGS) {
     for (int p = 0; p < 2; ++p)
       GMC_TRY(cudaMemsetAsync(h->chunk[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint2), s));
@@ -816,7 +839,7 @@ int gmc_get_worker_params(gmc_t h, int32_t k, float* out_dev, void* stream) {
   DeviceGuard g(h->device);
   GMC_TRY_ST(flush(h, static_cast<cudaStream_t>(stream)));
   GMC_TRY(order_after_flush(h, static_cast<cudaStream_t>(stream), false));
-  DetachArgs D{h->w, h->e, h->ld, h->d, h->lambda * h->eta, out_dev, h->d, k, k + 1};
+  DetachArgs D{h->w, h->e, h->ld, h->d, detach_b(h), out_dev, h->d, k, k + 1};
   GMC_TRY(launch_detach(D, static_cast<cudaStream_t>(stream)));
   return GMC_OK;
 }
@@ -863,13 +886,14 @@ struct StateHeader {
   float beta, eta, lambda;
   int32_t select_mode;
   uint64_t totals[8];
-  uint32_t status, has_mom;
+  uint32_t status, has_mom, lm_rows, pad;
 };
 constexpr char kMagic[8] = {'G', 'M', 'C', 'S', 'T', 'A', 'T', 'E'};
 constexpr uint32_t kStateVersion = 1;
 
 int64_t state_bytes(const gmc_ctx* h) {
-  const int64_t rows = (int64_t)(2 + h->K) + (h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1 : 0);
+  const int64_t rows = (int64_t)(2 + h->K) + (h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1 : 0) +
+                       (local_variant(h) ? h->K : 0);
   return (int64_t)sizeof(StateHeader) + rows * h->d * (int64_t)sizeof(float);
 }
 }  // namespace
@@ -909,6 +933,7 @@ int gmc_save_state(gmc_t h, void* host_out, int64_t capacity) {
   for (int i = 0; i < 8; ++i) H.totals[i] = c.v[i];
   GMC_TRY(cudaMemcpy(&H.status, h->status, sizeof(unsigned), cudaMemcpyDeviceToHost));
   H.has_mom = h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1u : 0u;
+  H.lm_rows = local_variant(h) ? (uint32_t)h->K : 0u;
   char* out = static_cast<char*>(host_out);
   std::memcpy(out, &H, sizeof(H));
   const size_t row = (size_t)h->d * sizeof(float);
@@ -922,7 +947,13 @@ int gmc_save_state(gmc_t h, void* host_out, int64_t capacity) {
   GMC_TRY(cudaMemcpy2D(p, row, h->e, (size_t)h->ld * sizeof(float), row, (size_t)h->K,
                        cudaMemcpyDeviceToHost));
   p += row * h->K;
-  if (H.has_mom) GMC_TRY(cudaMemcpy(p, h->mom, row, cudaMemcpyDeviceToHost));
+  if (H.has_mom) {
+    GMC_TRY(cudaMemcpy(p, h->mom, row, cudaMemcpyDeviceToHost));
+    p += row;
+  }
+  if (H.lm_rows)
+    GMC_TRY(cudaMemcpy2D(p, row, h->lm, (size_t)h->ld * sizeof(float), row, (size_t)h->K,
+                         cudaMemcpyDeviceToHost));
   return GMC_OK;
 }
 
@@ -936,7 +967,8 @@ int gmc_load_state(gmc_t h, const void* host_in, int64_t bytes) {
   // the handle must have been created for the same problem and form
   if (H.d != h->d || H.K != h->K || H.compressor != h->compressor || H.ratio != h->ratio ||
       (h->compressor == GMC_RBGS && H.block != h->block) || H.variant != h->variant ||
-      H.t < 0 || H.has_mom != (h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1u : 0u))
+      H.t < 0 || H.has_mom != (h->variant == GMC_VARIANT_SERVER_MOMENTUM ? 1u : 0u) ||
+      H.lm_rows != (local_variant(h) ? (uint32_t)h->K : 0u))
     return GMC_EINVAL;
   if (bytes < state_bytes(h)) return GMC_EINVAL;
   if (!finite_f(H.eta) || !(H.eta > 0.f) || !finite_f(H.lambda) || H.lambda < 0.f || H.lambda > 1.f ||
@@ -956,7 +988,13 @@ int gmc_load_state(gmc_t h, const void* host_in, int64_t bytes) {
   GMC_TRY(cudaMemcpy2D(h->e, (size_t)h->ld * sizeof(float), p, row, row, (size_t)h->K,
                        cudaMemcpyHostToDevice));
   p += row * h->K;
-  if (H.has_mom) GMC_TRY(cudaMemcpy(h->mom, p, row, cudaMemcpyHostToDevice));
+  if (H.has_mom) {
+    GMC_TRY(cudaMemcpy(h->mom, p, row, cudaMemcpyHostToDevice));
+    p += row;
+  }
+  if (H.lm_rows)
+    GMC_TRY(cudaMemcpy2D(h->lm, (size_t)h->ld * sizeof(float), p, row, row, (size_t)h->K,
+                         cudaMemcpyHostToDevice));
   Counters c;
   for (int i = 0; i < 8; ++i) c.v[i] = H.totals[i];
   GMC_TRY(cudaMemcpy(h->total_ctr, &c, sizeof(Counters), cudaMemcpyHostToDevice));

@@ -38,6 +38,12 @@ struct TopkArgs {
   int server_mom;
   float beta;
   float* mom;                // Alg. 3: w_t - w_{t-1} over [0, d)
+  // The local-momentum baseline (Sec. 2.3 eq. (3) with error feedback): each
+  // worker's m = beta*m + eta*g (lm, K rows of ld) replaces g in the
+  // accumulator (c = 0, a = fl(1/K)); mfm: m = 0 where the worker sent.
+  int local_mom;
+  int mfm;
+  float* lm;
   int K;
   int64_t n_tiles;
   int tile;                  // elements per tile

@@ -45,6 +45,25 @@ __device__ __forceinline__ float4 load_g4(const float* __restrict__ g, int64_t j
   return r;
 }
 
+// The local momentum of worker k at sampled coordinate j, formed from g
+// (m_{t+1} = beta*m_t + eta*g, Sec. 2.3 eq. (3)) without storing it.
+__device__ __forceinline__ float local_m(const TopkArgs& A, int k, int64_t j, float g) {
+  return __fadd_rn(__fmul_rn(A.beta, A.lm[(int64_t)k * A.ld + j]), __fmul_rn(A.gs, g));
+}
+// The local-momentum baseline: m = beta*m + eta*g over 4 coordinates of row k
+// at p (16-byte aligned, inside ld), stored back; returns it for the
+// accumulator in place of g.
+__device__ __forceinline__ float4 local_m4(const TopkArgs& A, float* p, float4 g) {
+  const float4 m = __ldcs(reinterpret_cast<const float4*>(p));
+  float4 r;
+  r.x = __fadd_rn(__fmul_rn(A.beta, m.x), __fmul_rn(A.gs, g.x));
+  r.y = __fadd_rn(__fmul_rn(A.beta, m.y), __fmul_rn(A.gs, g.y));
+  r.z = __fadd_rn(__fmul_rn(A.beta, m.z), __fmul_rn(A.gs, g.z));
+  r.w = __fadd_rn(__fmul_rn(A.beta, m.w), __fmul_rn(A.gs, g.w));
+  __stcs(reinterpret_cast<float4*>(p), r);
+  return r;
+}
+
 // Alg. 4 feeds eta * g into the accumulator: one more rounded product.
 __device__ __forceinline__ float4 scale_g(const TopkArgs& A, float4 g) {
   if (A.gscale) {
@@ -192,12 +211,12 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
         const int64_t j = A.sample_pend[2 * A.sample_stride + i];
         const uint32_t m = A.sample_pend[i];
         ev[q] = ((m >> k) & 1u) ? 0.f : ek[j];
-        gv[q] = A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j];
+        gv[q] = A.local_mom ? local_m(A, k, j, gk[j]) : (A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j]);
         dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
       } else if (i < i_hi) {
         const int64_t j = sample_coord(A, skey, i);
         ev[q] = ek[j];
-        gv[q] = A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j];
+        gv[q] = A.local_mom ? local_m(A, k, j, gk[j]) : (A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j]);
         dv[q] = A.dlt[j];
         if (A.pending) {  // as if the previous step's aggregation were applied at j
           const uint32_t m = A.sample_pend[i];
@@ -662,6 +681,7 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
         const int l = u * 128 + lane * 4;
         ev[u] = __ldcs(reinterpret_cast<const float4*>(ekt + l));
         gv[u] = scale_g(A, load_g4(gk, (int64_t)s0 + l, A.d, gm));
+        if (A.local_mom) gv[u] = local_m4(A, A.lm + (int64_t)k * A.ld + s0 + l, gv[u]);
       }
       float v[U][4];
       uint32_t bits[U];
@@ -1035,6 +1055,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
           if (l + 3 >= lim) g4.w = 0.f;
         }
         g4 = scale_g(A, g4);
+        if (A.local_mom) g4 = local_m4(A, A.lm + (int64_t)k * A.ld + s0 + l, g4);
         if (many) {  // more union coordinates than lanes: per-element sender masks
           const uint4 m4 = *reinterpret_cast<const uint4*>(mkw + l);
           if ((m4.x >> k) & 1u) e4.x = 0.f;
@@ -1609,6 +1630,7 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
         if ((m >> b) & 1u) {
           sum = __fadd_rn(sum, vals[b]);
           A.e[(int64_t)b * A.ld + j] = 0.f;  // e_{t+1,b} = e_{t+1/2,b} - C(.) = +0 where sent
+          if (A.mfm) A.lm[(int64_t)b * A.ld + j] = 0.f;  // momentum factor masking
         }
       }
       A.mask[j] = 0u;

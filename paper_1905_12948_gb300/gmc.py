@@ -16,7 +16,9 @@ LIB_PATH = os.path.join(_PKG, "libgmc.so")
 
 GMC_OK, GMC_EINVAL, GMC_ENOMEM, GMC_ECUDA, GMC_ENONFINITE, GMC_ESTATE, GMC_EINTERNAL, GMC_ETOOBIG = range(8)
 GMC_TOPK, GMC_RBGS, GMC_TOPK_APPROX = 0, 1, 2
-VARIANTS = {"gmc": 0, "server_momentum": 1, "lr_in_residual": 2}  # Alg. 1, Alg. 3, Alg. 4
+# Alg. 1, Alg. 3, Alg. 4, and the local-momentum baseline without / with masking
+VARIANTS = {"gmc": 0, "server_momentum": 1, "lr_in_residual": 2, "local_momentum": 3,
+            "local_momentum_mfm": 4}
 GMC_SELECT_SAMPLED, GMC_SELECT_DENSE = 0, 1
 STAT_NAMES = ["steps", "pairs", "nnz", "union", "changed", "fallbacks", "nonfinite", "reserved"]
 GMC_STAT_COUNT = 8
@@ -131,15 +133,15 @@ class GMC:
             _check(self.lib.gmc_create(ctypes.byref(h), self.d, self.K, beta, eta, comp,
                                        float(ratio), int(block)), "gmc_create")
         self.h = h
+        if variant != "gmc":
+            with torch.cuda.device(self.device):
+                _check(self.lib.gmc_set_variant(h, VARIANTS[variant]), "gmc_set_variant")
         if lam is not None:
             _check(self.lib.gmc_set_lambda(h, lam), "gmc_set_lambda")
         _check(self.lib.gmc_set_seed(h, int(seed) & ((1 << 64) - 1)), "gmc_set_seed")
         _check(self.lib.gmc_set_rbgs_mode(h, int(bool(per_worker))), "gmc_set_rbgs_mode")
         mode = {"sampled": GMC_SELECT_SAMPLED, "dense": GMC_SELECT_DENSE}[select_mode]
         _check(self.lib.gmc_set_select_mode(h, mode), "gmc_set_select_mode")
-        if variant != "gmc":
-            with torch.cuda.device(self.device):
-                _check(self.lib.gmc_set_variant(h, VARIANTS[variant]), "gmc_set_variant")
         self._detach = None
 
     def close(self) -> None:

@@ -1,7 +1,8 @@
 """Checkpoint / resume through the C ABI: a trajectory saved mid-run (with an
 aggregation still pending, for the deferred top-k path) and loaded into a new
 handle continues exactly as the oracle's uninterrupted run, for every
-compressor, both dense passes and the appendix's Alg. 3; malformed or
+compressor, both dense passes and every variant of the step (with their extra
+state: Alg. 3's server momentum, the workers' local momentum); malformed or
 mismatched states are refused."""
 import numpy as np
 import pytest
@@ -28,6 +29,8 @@ CASES = [
     dict(compressor="rbgs", d=70_001, K=3, ratio=0.1, block=1000, lam=0.5, per_worker=True),
     dict(compressor="topk", d=1_300_001, K=3, ratio=0.002, variant="server_momentum"),
     dict(compressor="topk", d=1_300_001, K=3, ratio=0.002, variant="lr_in_residual"),
+    dict(compressor="topk", d=1_300_001, K=3, ratio=0.002, variant="local_momentum"),
+    dict(compressor="topk_approx", d=50_003, K=2, ratio=0.01, variant="local_momentum_mfm"),
 ]
 
 

@@ -24,6 +24,7 @@ pytestmark = pytest.mark.gpu
     ("vgg16_approx", 3, False, True),  # the same under the approximate top-s of Sec. 5.1
     ("vgg16_alg3", 2, False, False),   # the same under the appendix's Alg. 3 (eager, dense server step)
     ("vgg16_alg4", 2, False, True),    # and Alg. 4
+    ("vgg16_local", 2, False, True),   # and the local-momentum baseline
 ])
 def test_fullsize_parity(name, steps, per_worker, deferred):
     import torch

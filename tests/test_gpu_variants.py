@@ -1,7 +1,9 @@
-"""GPU-vs-oracle parity of the appendix variants: Alg. 3 (momentum on the
-server, a dense update of w every step) and Alg. 4 (learning rate inside the
-residual), with both top-k compressors, on the load/store and bulk passes,
-with the learning-rate schedule between steps and host steps."""
+"""GPU-vs-oracle parity of the variants of the step: the appendix's Alg. 3
+(momentum on the server, a dense update of w every step) and Alg. 4
+(learning rate inside the residual), and the local-momentum baseline of
+Sec. 2.3 with error feedback (DGC without / with momentum factor masking),
+with both top-k compressors, on the load/store and bulk passes, with the
+learning-rate schedule between steps and host steps."""
 import numpy as np
 import pytest
 
@@ -9,7 +11,8 @@ from parity_util import Pair
 
 pytestmark = pytest.mark.gpu
 
-VARIANTS = ["server_momentum", "lr_in_residual"]
+VARIANTS = ["server_momentum", "lr_in_residual", "local_momentum", "local_momentum_mfm"]
+EAGER = ("server_momentum", "local_momentum_mfm")  # these aggregate every step at once
 
 
 def _grads(rng, K, d):
@@ -24,8 +27,8 @@ def test_variant_parity(variant, compressor, d, K):
     p = Pair(d, K, 0.9, 0.1, compressor=compressor, ratio=0.002, seed=6, variant=variant)
     for t in range(4):
         r = p.step(_grads(rng, K, d))
-        # Alg. 4 on the bulk pass defers its aggregation: read the state at the end
-        p.compare(r, state=(variant == "server_momentum" or d < 1_000_000 or t == 3))
+        # the others defer their aggregation on the bulk pass: read the state at the end
+        p.compare(r, state=(variant in EAGER or d < 1_000_000 or t == 3))
     s = p.compare_stats()
     assert s["fallbacks"] == 0
     assert p.gpu.check() == 0
@@ -66,6 +69,26 @@ def test_server_momentum_moves_coordinates_off_the_union():
         p.compare(r)
     s = p.compare_stats()
     assert s["changed"] > s["union"]
+
+
+@pytest.mark.parametrize("variant", ["local_momentum", "local_momentum_mfm"])
+def test_local_momentum_detach(variant):
+    """The DEF-A-like detached points of the local-momentum baseline,
+    w_{t,k} = w_t - lambda e_{t,k}, written by the step."""
+    import torch
+    d, K = 1_300_001, 3
+    rng = np.random.default_rng(33)
+    p = Pair(d, K, 0.9, 0.1, ratio=0.002, seed=4, variant=variant, lam=0.3)
+    out = torch.empty((K, d), dtype=torch.float32, device=p.dev)
+    p.gpu.set_detach_output(out)
+    for t in range(3):
+        r = p.step(_grads(rng, K, d))
+        p.compare(r)
+        torch.cuda.synchronize()
+        for k in range(K):
+            np.testing.assert_array_equal(out[k].cpu().numpy().view(np.uint32),
+                                          p.ref.worker_params(k).view(np.uint32))
+    p.compare_stats()
 
 
 def test_variant_refusals():

@@ -53,7 +53,8 @@ class Workload:
     noniid: float = 0.0         # per-worker mean offset std as a multiple of the segment std
     iid_unit: bool = False      # gradients N(0,1) i.i.d., no segments
     w0_std: float = 0.01
-    variant: str = "gmc"        # Alg. 1, or the appendix's "server_momentum" (Alg. 3) / "lr_in_residual" (Alg. 4)
+    variant: str = "gmc"        # Alg. 1, the appendix's "server_momentum" (Alg. 3) / "lr_in_residual"
+                                # (Alg. 4), or the baseline "local_momentum" / "local_momentum_mfm"
 
     @property
     def k(self) -> int:
@@ -83,6 +84,13 @@ WORKLOADS = [
     Workload("vgg16_alg4", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
              eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
              scale_lo=1e-4, scale_hi=1e-1, noniid=0.02, variant="lr_in_residual"),
+    # and under the local-momentum baseline (DGC without / with momentum factor masking)
+    Workload("vgg16_local", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
+             eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
+             scale_lo=1e-4, scale_hi=1e-1, noniid=0.02, variant="local_momentum"),
+    Workload("vgg16_local_mfm", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
+             eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
+             scale_lo=1e-4, scale_hi=1e-1, noniid=0.02, variant="local_momentum_mfm"),
 ]
 
 
