@@ -352,7 +352,8 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
     const bool defer = h->tile == kBulkTile && !eager && !h->detach_out && !A.server_mom && !A.mfm;
     const double kk = (double)h->K * (double)h->ksel;
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
-    GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, 12.0 * Kd, s,
+    // read g, e (and the local momentum), write v over e (and the momentum)
+    GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, (A.local_mom ? 20.0 : 12.0) * Kd, s,
                   [&] { return launch_accumulate(A, h->grid_acc, s); }));
     h->agg_pending = false;
     GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] {

@@ -50,11 +50,10 @@ __device__ __forceinline__ float4 load_g4(const float* __restrict__ g, int64_t j
 __device__ __forceinline__ float local_m(const TopkArgs& A, int k, int64_t j, float g) {
   return __fadd_rn(__fmul_rn(A.beta, A.lm[(int64_t)k * A.ld + j]), __fmul_rn(A.gs, g));
 }
-// The local-momentum baseline: m = beta*m + eta*g over 4 coordinates of row k
-// at p (16-byte aligned, inside ld), stored back; returns it for the
-// accumulator in place of g.
-__device__ __forceinline__ float4 local_m4(const TopkArgs& A, float* p, float4 g) {
-  const float4 m = __ldcs(reinterpret_cast<const float4*>(p));
+// The local-momentum baseline: m = beta*m + eta*g over 4 coordinates (m
+// loaded from p beforehand, p 16-byte aligned inside ld), stored back at p;
+// returns it for the accumulator in place of g.
+__device__ __forceinline__ float4 local_m4(const TopkArgs& A, float* p, float4 m, float4 g) {
   float4 r;
   r.x = __fadd_rn(__fmul_rn(A.beta, m.x), __fmul_rn(A.gs, g.x));
   r.y = __fadd_rn(__fmul_rn(A.beta, m.y), __fmul_rn(A.gs, g.y));
@@ -655,7 +654,9 @@ __device__ __forceinline__ void write_group(const float v[4], uint32_t j, uint32
 }
 
 // load/store version for small tiles; candidates share one region per worker
-template <int U>
+// kLocal: the local-momentum baseline's instantiation (its momentum loads
+// need registers the other forms do without).
+template <int U, bool kLocal>
 __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
   constexpr int SUB = 128 * U;       // elements per warp and worker
   constexpr int T = kWarps * SUB;    // elements per tile
@@ -675,13 +676,18 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
       float* ekt = A.e + (int64_t)k * A.ld + s0;
       const float* gk = A.grads + (int64_t)k * A.d;
       const int gm = g_mode(gk);
-      float4 ev[U], gv[U];
+      float4 ev[U], gv[U], mv[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const int l = u * 128 + lane * 4;
         ev[u] = __ldcs(reinterpret_cast<const float4*>(ekt + l));
         gv[u] = scale_g(A, load_g4(gk, (int64_t)s0 + l, A.d, gm));
-        if (A.local_mom) gv[u] = local_m4(A, A.lm + (int64_t)k * A.ld + s0 + l, gv[u]);
+        if (kLocal) mv[u] = __ldcs(reinterpret_cast<const float4*>(A.lm + (int64_t)k * A.ld + s0 + l));
+      }
+      if (kLocal) {
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+          gv[u] = local_m4(A, A.lm + (int64_t)k * A.ld + s0 + u * 128 + lane * 4, mv[u], gv[u]);
       }
       float v[U][4];
       uint32_t bits[U];
@@ -879,6 +885,7 @@ __device__ __forceinline__ uint32_t apply_pairs(const TopkArgs& A, uint32_t sub0
   return first ? l : ~0u;
 }
 
+template <bool kLocal>
 __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkArgs A) {
   using namespace bulk;
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -1016,6 +1023,12 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     for (int k = gp; ok && k < A.K; k += 2) {
       const uint32_t item = n * (uint32_t)A.K + (uint32_t)k;
       const uint32_t s = item % kStages, r = item / kStages;
+      float4 mv[kSub / 128];  // the local-momentum baseline: m loaded while the stage lands
+      if (kLocal) {
+#pragma unroll
+        for (int u = 0; u < kSub / 128; ++u)
+          mv[u] = __ldcs(reinterpret_cast<const float4*>(A.lm + (int64_t)k * A.ld + s0 + u * 128 + lane * 4));
+      }
       if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
         ok = false;
         break;
@@ -1055,7 +1068,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
           if (l + 3 >= lim) g4.w = 0.f;
         }
         g4 = scale_g(A, g4);
-        if (A.local_mom) g4 = local_m4(A, A.lm + (int64_t)k * A.ld + s0 + l, g4);
+        if (kLocal) g4 = local_m4(A, A.lm + (int64_t)k * A.ld + s0 + l, mv[u], g4);
         if (many) {  // more union coordinates than lanes: per-element sender masks
           const uint4 m4 = *reinterpret_cast<const uint4*>(mkw + l);
           if ((m4.x >> k) & 1u) e4.x = 0.f;
@@ -1755,11 +1768,14 @@ cudaError_t configure_topk_kernels() {
     const cudaError_t e2 = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (err == cudaSuccess) err = e2;
   };
-  set((const void*)k_accumulate<1>, 1024 * 12);
-  set((const void*)k_accumulate<2>, 2048 * 12);
-  set((const void*)k_accumulate<4>, 4096 * 12);
-  set((const void*)k_accumulate<8>, 8192 * 12);
-  set((const void*)k_accumulate_bulk, bulk::smem_bytes(kBulkMaxK));
+  set((const void*)k_accumulate<1, false>, 1024 * 12);
+  set((const void*)k_accumulate<2, false>, 2048 * 12);
+  set((const void*)k_accumulate<4, false>, 4096 * 12);
+  set((const void*)k_accumulate<1, true>, 1024 * 12);
+  set((const void*)k_accumulate<2, true>, 2048 * 12);
+  set((const void*)k_accumulate<4, true>, 4096 * 12);
+  set((const void*)k_accumulate_bulk<false>, bulk::smem_bytes(kBulkMaxK));
+  set((const void*)k_accumulate_bulk<true>, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_select_finish, 2 * kBucketCap * 4);
   set((const void*)k_sample_theta, kBucketCap * 4);
   return err;
@@ -1770,10 +1786,9 @@ int accumulate_blocks_per_sm(int tile) {
   int n = 0;
   const int smem = accumulate_smem_bytes(tile, kMaxK);
   switch (tile_u(tile)) {
-    case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<1>, kThreads, smem); break;
-    case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<2>, kThreads, smem); break;
-    case 4: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<4>, kThreads, smem); break;
-    default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<8>, kThreads, smem); break;
+    case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<1, false>, kThreads, smem); break;
+    case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<2, false>, kThreads, smem); break;
+    default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<4, false>, kThreads, smem); break;
   }
   return n > 0 ? n : 1;
 }
@@ -1797,14 +1812,19 @@ cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
   const int smem = accumulate_smem_bytes(A.tile, A.K);
   if (use_bulk(A.tile)) {
-    k_accumulate_bulk<<<grid, bulk::kThreadsAll, smem, s>>>(A);
+    if (A.local_mom)
+      k_accumulate_bulk<true><<<grid, bulk::kThreadsAll, smem, s>>>(A);
+    else
+      k_accumulate_bulk<false><<<grid, bulk::kThreadsAll, smem, s>>>(A);
     return cudaGetLastError();
   }
   switch (tile_u(A.tile)) {
-    case 1: k_accumulate<1><<<grid, kThreads, smem, s>>>(A); break;
-    case 2: k_accumulate<2><<<grid, kThreads, smem, s>>>(A); break;
-    case 4: k_accumulate<4><<<grid, kThreads, smem, s>>>(A); break;
-    default: k_accumulate<8><<<grid, kThreads, smem, s>>>(A); break;
+    case 1: A.local_mom ? k_accumulate<1, true><<<grid, kThreads, smem, s>>>(A)
+                        : k_accumulate<1, false><<<grid, kThreads, smem, s>>>(A); break;
+    case 2: A.local_mom ? k_accumulate<2, true><<<grid, kThreads, smem, s>>>(A)
+                        : k_accumulate<2, false><<<grid, kThreads, smem, s>>>(A); break;
+    default: A.local_mom ? k_accumulate<4, true><<<grid, kThreads, smem, s>>>(A)
+                         : k_accumulate<4, false><<<grid, kThreads, smem, s>>>(A); break;
   }
   return cudaGetLastError();
 }
