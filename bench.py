@@ -272,16 +272,29 @@ def run_reference(args, wl, world, rank):
     return line
 
 
+def step_bytes(wl) -> float:
+    """Algorithmic bytes of one step's dense work: read g and e, write e
+    (12 B per worker-parameter, 10 with bf16 gradients); the local momentum
+    adds its read and write (8 B), Alg. 3's dense server pass 20 B per parameter."""
+    b = (8.0 + (2.0 if wl.grad_dtype == "bf16" else 4.0)) * wl.K * wl.d
+    if wl.variant in ("local_momentum", "local_momentum_mfm"):
+        b += 8.0 * wl.K * wl.d
+    if wl.variant == "server_momentum":
+        b += 20.0 * wl.d
+    return b
+
+
 def config_of(wl, args):
     return {"workload": f"{wl.name}: d={wl.d:,}, K={wl.K}, {wl.compressor}"
                         + (f" ratio {wl.ratio:.6g}" if wl.compressor != "rbgs"
                            else f" block {wl.block}, {wl.ratio:.0%} of blocks, lambda {wl.lam}")
                         + f", beta {wl.beta}, eta {wl.eta}"
-                        + ("" if wl.variant == "gmc" else f", variant {wl.variant}"),
+                        + ("" if wl.variant == "gmc" else f", variant {wl.variant}")
+                        + ("" if wl.grad_dtype == "f32" else f", {wl.grad_dtype} gradients"),
             "d": wl.d, "K": wl.K, "compressor": wl.compressor, "ratio": wl.ratio,
             "block": wl.block if wl.compressor == "rbgs" else None,
             "per_worker_blocks": wl.per_worker if wl.compressor == "rbgs" else None,
-            "lambda": wl.lam, "variant": wl.variant,
+            "lambda": wl.lam, "variant": wl.variant, "grad_dtype": wl.grad_dtype,
             "l2": "inputs larger than L2 (gradient batches rotate)",
             "parallelism": f"replicas x{args.gpus}"}
 
@@ -300,8 +313,10 @@ def run_gmc(args, wl, world, rank, local):
               per_worker=wl.per_worker, variant=wl.variant, device=dev)
     w0 = torch.from_numpy(workloads.init_params(wl.d)).to(dev)
     gen = workloads.TorchGradients(wl, dev, seed=rank)
-    n_batches = 2 if 4.0 * wl.K * wl.d > 2 * L2_BYTES else max(2, math.ceil(4 * L2_BYTES / (4.0 * wl.K * wl.d)))
-    batches = [gen(t) for t in range(n_batches)]
+    bf16 = wl.grad_dtype == "bf16"
+    gb = (2.0 if bf16 else 4.0) * wl.K * wl.d  # gradient bytes per step
+    n_batches = 2 if gb > 2 * L2_BYTES else max(2, math.ceil(4 * L2_BYTES / gb))
+    batches = [gen(t).to(torch.bfloat16) if bf16 else gen(t) for t in range(n_batches)]
     del gen
     torch.cuda.synchronize()
     stream = torch.cuda.current_stream()
@@ -347,7 +362,7 @@ def run_gmc(args, wl, world, rank, local):
 
     e2e = None
     if not args.no_e2e:
-        host = torch.empty((wl.K, wl.d), dtype=torch.float32).pin_memory()
+        host = torch.empty((wl.K, wl.d), dtype=torch.bfloat16 if bf16 else torch.float32).pin_memory()
         host.copy_(torch.from_numpy(workloads.NumpyGradients(wl, seed=rank, K=wl.K)(0))
                    if wl.K * wl.d <= 50_000_000 else
                    workloads.TorchGradients(wl, dev, seed=rank)(0).cpu())
@@ -365,7 +380,7 @@ def run_gmc(args, wl, world, rank, local):
         torch.cuda.synchronize()
         e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
         e2e = {"value": wl.K * wl.d * args.steps * world / (e_ms / 1e3), "unit": UNIT,
-               "h2d_bytes_per_step": 4 * wl.K * wl.d, "d2h_bytes_per_step": 8 * 8,
+               "h2d_bytes_per_step": int(gb), "d2h_bytes_per_step": 8 * 8,
                "ms_per_step": e_ms / args.steps}
         del host
     gpu.close()
@@ -381,7 +396,7 @@ def run_gmc(args, wl, world, rank, local):
         "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": config_of(wl, args),
-        "hbm_gbs_step": 12.0 * wl.K * wl.d / (step_ms / 1e3) / 1e9,
+        "hbm_gbs_step": step_bytes(wl) / (step_ms / 1e3) / 1e9,
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": traffic, "algorithmic_bytes_per_launch": per_launch_bytes,

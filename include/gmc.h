@@ -213,6 +213,17 @@ int gmc_step(gmc_t h, const float* grads_dev, void* stream);
  * skip the read-back). */
 int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, void* stream);
 
+/* gmc_step_bf16 / gmc_step_host_bf16 -- gmc_step / gmc_step_host with the
+ * gradients in bfloat16: K x d row-major 16-bit values, each the upper half of
+ * an fp32 bit pattern, widened exactly to fp32 as they are read (the step's
+ * arithmetic is unchanged). Halves the gradient bytes the step reads (device)
+ * or moves over the host link (host). The pointer must be 2-byte aligned
+ * (GMC_EINVAL otherwise); ownership, ordering and errors as gmc_step /
+ * gmc_step_host. */
+int gmc_step_bf16(gmc_t h, const uint16_t* grads_bf16_dev, void* stream);
+int gmc_step_host_bf16(gmc_t h, const uint16_t* grads_bf16_host, uint64_t* step_stats_host,
+                       void* stream);
+
 /* gmc_get_params -- copy w_t (d floats) into w_dev_out (applying a pending
  * aggregation first, see gmc_step). */
 int gmc_get_params(gmc_t h, float* w_dev_out, void* stream);

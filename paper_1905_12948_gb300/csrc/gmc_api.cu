@@ -338,7 +338,11 @@ cudaError_t order_after_flush(gmc_ctx* h, cudaStream_t s, bool clear) {
 // sent) is left pending unless `eager`: the next step's bulk pass applies it
 // while it streams the tile, or flush() does when the state is read.
 // `direct`: grads is mapped host memory, read in place by the kernels.
-int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, bool direct = false) {
+int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, bool direct = false,
+                 bool bf16 = false) {
+  // fp32 rows, or bfloat16 rows (gmc_step_bf16) widened exactly as they are read
+  const float* grads = bf16 ? nullptr : static_cast<const float*>(grads_any);
+  const uint16_t* grads16 = bf16 ? static_cast<const uint16_t*>(grads_any) : nullptr;
   const double Kd = (double)h->K * (double)h->d;
   GMC_TRY(order_after_flush(h, s, true));
   GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
@@ -346,6 +350,8 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
   if (h->compressor != GMC_RBGS) {
     const bool approx = h->compressor == GMC_TOPK_APPROX;
     TopkArgs A = topk_args(h, grads);
+    A.grads16 = grads16;
+    A.bf16 = bf16 ? 1 : 0;
     A.g_direct = direct ? 1 : 0;
     A.pending = h->agg_pending ? 1 : 0;
     A.a_prev = h->a_pending;
@@ -353,7 +359,7 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
     const double kk = (double)h->K * (double)h->ksel;
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
     // read g, e (and the local momentum), write v over e (and the momentum)
-    GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, (A.local_mom ? 20.0 : 12.0) * Kd, s,
+    GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, ((A.local_mom ? 20.0 : 12.0) - (bf16 ? 2.0 : 0.0)) * Kd, s,
                   [&] { return launch_accumulate(A, h->grid_acc, s); }));
     h->agg_pending = false;
     GMC_TRY(timed(h, GMC_KERNEL_SELECT, 0.0, s, [&] {
@@ -378,13 +384,15 @@ int enqueue_step(gmc_ctx* h, const float* grads, cudaStream_t s, bool eager, boo
     pairs_add = approx ? 0ull : (unsigned long long)h->K * h->ksel;  // approximate: counted on the device
   } else {
     RbgsArgs A = rbgs_args(h, grads);
+    A.grads16 = grads16;
+    A.bf16 = bf16 ? 1 : 0;
     A.g_direct = direct ? 1 : 0;
     // restored state: w_t - w_{t-1} may be non-zero in any block (zero outside
     // the last union, where dlt holds it): flag every block as the last union's
     if (h->restored && h->t > 0) GMC_TRY(cudaMemsetAsync(A.uflag_prev, 1, (size_t)h->nb, s));
     GMC_TRY(cudaMemsetAsync(A.uflag_cur, 0, (size_t)h->nb, s));
     GMC_TRY(timed(h, GMC_KERNEL_RBGS_PICK, 0.0, s, [&] { return launch_rbgs_pick(A, s); }));
-    GMC_TRY(timed(h, GMC_KERNEL_RBGS_STEP, 12.0 * Kd, s,
+    GMC_TRY(timed(h, GMC_KERNEL_RBGS_STEP, (bf16 ? 10.0 : 12.0) * Kd, s,
                   [&] { return launch_rbgs_step(A, h->grid_rbgs, s); }));
   }
   if (h->detach_out) {
@@ -724,6 +732,31 @@ int reset_state(gmc_ctx* h, cudaStream_t s) {
   h->initialized = true;
   return GMC_OK;
 }
+
+// gmc_step_host for fp32 or bf16 gradient rows.
+int step_host(gmc_ctx* h, const void* grads_host, uint64_t* step_stats_host, cudaStream_t s, bool bf16) {
+  // page-locked host memory is mapped into the device's address space: the
+  // kernels read the gradients in place, each crossing the host link once
+  // while the pass runs; other host memory is copied to a staging buffer first
+  const void* mapped = nullptr;
+  int st;
+  if (cudaHostGetDevicePointer(const_cast<void**>(&mapped), const_cast<void*>(grads_host), 0) == cudaSuccess) {
+    st = enqueue_step(h, mapped, s, true, true, bf16);
+  } else {
+    cudaGetLastError();
+    const size_t n = (size_t)h->K * (size_t)h->d;
+    if (!h->gstage) {
+      cudaError_t err = dalloc(h, &h->gstage, n);
+      if (err != cudaSuccess) return status_of(err);
+    }
+    GMC_TRY(cudaMemcpyAsync(h->gstage, grads_host, n * (bf16 ? 2 : 4), cudaMemcpyHostToDevice, s));
+    st = enqueue_step(h, h->gstage, s, true, false, bf16);
+  }
+  if (st != GMC_OK) return st;
+  if (step_stats_host)
+    GMC_TRY(cudaMemcpyAsync(step_stats_host, h->step_ctr, sizeof(Counters), cudaMemcpyDeviceToHost, s));
+  return GMC_OK;
+}
 }  // namespace
 
 extern "C" {
@@ -744,32 +777,26 @@ int gmc_step(gmc_t h, const float* grads_dev, void* stream) {
   return enqueue_step(h, grads_dev, static_cast<cudaStream_t>(stream), false);
 }
 
+
 int gmc_step_host(gmc_t h, const float* grads_host, uint64_t* step_stats_host, void* stream) {
   if (!h || !grads_host) return GMC_EINVAL;
   if (!h->initialized) return GMC_ESTATE;
   DeviceGuard g(h->device);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // page-locked host memory is mapped into the device's address space: the
-  // kernels read the gradients in place, each crossing the host link once
-  // while the pass runs; other host memory is copied to a staging buffer first
-  const float* mapped = nullptr;
-  int st;
-  if (cudaHostGetDevicePointer((void**)&mapped, const_cast<float*>(grads_host), 0) == cudaSuccess) {
-    st = enqueue_step(h, mapped, s, true, true);
-  } else {
-    cudaGetLastError();
-    const size_t n = (size_t)h->K * (size_t)h->d;
-    if (!h->gstage) {
-      cudaError_t err = dalloc(h, &h->gstage, n);
-      if (err != cudaSuccess) return status_of(err);
-    }
-    GMC_TRY(cudaMemcpyAsync(h->gstage, grads_host, n * sizeof(float), cudaMemcpyHostToDevice, s));
-    st = enqueue_step(h, h->gstage, s, true);
-  }
-  if (st != GMC_OK) return st;
-  if (step_stats_host)
-    GMC_TRY(cudaMemcpyAsync(step_stats_host, h->step_ctr, sizeof(Counters), cudaMemcpyDeviceToHost, s));
-  return GMC_OK;
+  return step_host(h, grads_host, step_stats_host, static_cast<cudaStream_t>(stream), false);
+}
+
+int gmc_step_bf16(gmc_t h, const uint16_t* grads_bf16_dev, void* stream) {
+  if (!h || !grads_bf16_dev || (reinterpret_cast<uintptr_t>(grads_bf16_dev) & 1)) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  return enqueue_step(h, grads_bf16_dev, static_cast<cudaStream_t>(stream), false, false, true);
+}
+
+int gmc_step_host_bf16(gmc_t h, const uint16_t* grads_bf16_host, uint64_t* step_stats_host, void* stream) {
+  if (!h || !grads_bf16_host || (reinterpret_cast<uintptr_t>(grads_bf16_host) & 1)) return GMC_EINVAL;
+  if (!h->initialized) return GMC_ESTATE;
+  DeviceGuard g(h->device);
+  return step_host(h, grads_bf16_host, step_stats_host, static_cast<cudaStream_t>(stream), true);
 }
 
 int gmc_get_params(gmc_t h, float* w_dev_out, void* stream) {

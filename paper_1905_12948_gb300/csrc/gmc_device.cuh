@@ -66,6 +66,36 @@ __device__ __forceinline__ float accumulate(float e, float g, float c, float dl)
 __device__ __forceinline__ bool needs_dense(const WorkerSel& s, uint32_t ksel, uint32_t cap) {
   return s.count < ksel || s.count > cap || s.dense != 0;
 }
+// bfloat16 gradients: the upper 16 bits of an fp32 pattern, widened exactly.
+__device__ __forceinline__ float bf16_f32(uint32_t b) { return __uint_as_float(b << 16); }
+// Four consecutive bf16 values at p (2-byte aligned, shared or global memory).
+__device__ __forceinline__ float4 bf16x4(const uint16_t* p) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  uint32_t lo, hi;
+  if ((a & 7) == 0) {
+    const uint2 x = *reinterpret_cast<const uint2*>(p);
+    lo = x.x;
+    hi = x.y;
+  } else if ((a & 3) == 0) {
+    lo = *reinterpret_cast<const uint32_t*>(p);
+    hi = *reinterpret_cast<const uint32_t*>(p + 2);
+  } else {
+    lo = (uint32_t)p[0] | ((uint32_t)p[1] << 16);
+    hi = (uint32_t)p[2] | ((uint32_t)p[3] << 16);
+  }
+  return make_float4(__uint_as_float(lo << 16), __uint_as_float(lo & 0xffff0000u),
+                     __uint_as_float(hi << 16), __uint_as_float(hi & 0xffff0000u));
+}
+// Elements j .. j+3 of a bf16 row of d, zeros past d.
+__device__ __forceinline__ float4 load_g4_bf16(const uint16_t* g, int64_t j, int64_t d) {
+  if (j + 3 < d) return bf16x4(g + j);
+  float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (j < d) r.x = bf16_f32(g[j]);
+  if (j + 1 < d) r.y = bf16_f32(g[j + 1]);
+  if (j + 2 < d) r.z = bf16_f32(g[j + 2]);
+  return r;
+}
+
 // SplitMix64 (Steele, Lea & Flood, OOPSLA 2014): output function, the key of
 // step t's stream (stream 0 = shared by all workers, k+1 = worker k), the
 // stream's i-th draw, and [0, n) from a draw's top 32 bits by multiply-shift.

@@ -25,6 +25,8 @@ struct TopkArgs {
   float* e;                  // residuals / accumulator, K rows of ld floats
   int64_t ld;                // row stride of e (multiple of the tile)
   const float* grads;        // K x d, row stride d (caller memory)
+  const uint16_t* grads16;   // the same in bfloat16 (gmc_step_bf16), when bf16
+  int bf16;
   int64_t d;
   float* dlt;                // w_t - w_{t-1}, dense, zero outside the last union
   float* w;                  // parameters (ld floats)
@@ -110,6 +112,8 @@ struct RbgsArgs {
   float* e;
   int64_t ld;
   const float* grads;
+  const uint16_t* grads16;   // bfloat16 gradients (gmc_step_bf16), when bf16
+  int bf16;
   int64_t d;
   float* dlt;
   float* w;

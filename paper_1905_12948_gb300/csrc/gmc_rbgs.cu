@@ -101,6 +101,7 @@ __global__ void __launch_bounds__(kThreads) k_rbgs_pick(RbgsArgs A) {
 // ---------------------------------------------------------------------------
 // fused step: persistent blocks walk tiles of kRbgsTile elements
 // ---------------------------------------------------------------------------
+template <bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_rbgs_step(RbgsArgs A) {
   constexpr int U = kRbgsTile / (kThreads * 4);  // float4 groups per thread
   __shared__ unsigned long long ws[32];
@@ -142,6 +143,7 @@ __global__ void __launch_bounds__(kThreads) k_rbgs_step(RbgsArgs A) {
       const int32_t* rk = A.rank + (A.per_worker ? (int64_t)k * A.nb : 0);
       float* ek = A.e + (int64_t)k * A.ld;
       const float* gk = A.grads + (int64_t)k * A.d;
+      const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
       float* sk = A.slab + (int64_t)k * slab_ld;
       const int gm = g_mode(gk);
       float4 ev[U], gv[U];
@@ -149,7 +151,7 @@ __global__ void __launch_bounds__(kThreads) k_rbgs_step(RbgsArgs A) {
       for (int u = 0; u < U; ++u) {
         const int64_t j = t0 + u * (kThreads * 4) + threadIdx.x * 4;
         ev[u] = __ldcs(reinterpret_cast<const float4*>(ek + j));
-        gv[u] = load_g4(gk, j, A.d, gm);
+        gv[u] = kBf16 ? load_g4_bf16(gk16, j, A.d) : load_g4(gk, j, A.d, gm);
       }
 #pragma unroll
       for (int u = 0; u < U; ++u) {
@@ -275,6 +277,7 @@ struct Smem {
 };
 }  // namespace rbulk
 
+template <bool kBf16>
 __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A) {
   using namespace rbulk;
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -292,8 +295,10 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
   if (warp == kConsumers) {
     // ---- producer ----
     if (lane != 0) return;
-    const char* g_lo = reinterpret_cast<const char*>(A.grads);
-    const char* g_hi = reinterpret_cast<const char*>(A.grads + (int64_t)A.K * A.d);
+    // gradient rows of es-byte elements (fp32, or bf16 from gmc_step_bf16)
+    constexpr int es = kBf16 ? 2 : 4;
+    const char* g_lo = kBf16 ? reinterpret_cast<const char*>(A.grads16) : reinterpret_cast<const char*>(A.grads);
+    const char* g_hi = g_lo + (int64_t)A.K * A.d * es;
     uint32_t item = 0;
     bool ok = true;
     for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
@@ -306,11 +311,11 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
           break;
         }
         const float* esrc = A.e + (int64_t)k * A.ld + j0;
-        const uintptr_t ga = reinterpret_cast<uintptr_t>(A.grads + (int64_t)k * A.d + j0);
-        const uint32_t off = (uint32_t)(ga & 15) >> 2;
-        const char* gsrc = reinterpret_cast<const char*>(ga - off * 4);
-        const uint32_t gbytes = (uint32_t)(((nvalid + off) * 4 + 15) & ~int64_t(15));
-        const bool gbulk = !A.g_direct && (ga & 3) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
+        const uintptr_t ga = reinterpret_cast<uintptr_t>(g_lo + ((int64_t)k * A.d + j0) * es);
+        const uint32_t off = (uint32_t)(ga & 15) / es;  // leading elements before the row's tile
+        const char* gsrc = reinterpret_cast<const char*>(ga - off * es);
+        const uint32_t gbytes = (uint32_t)(((nvalid + off) * es + 15) & ~int64_t(15));
+        const bool gbulk = !A.g_direct && (ga % es) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
         sm.gmeta[s] = gbulk ? (int32_t)off : -1;
         mbar_arrive_expect_tx(&sm.full[s], kT * 4 + (gbulk ? gbytes : 0));
         bulk_load(sm.e[s], esrc, kT * 4, &sm.full[s]);
@@ -379,7 +384,12 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
         const int l = u * 128 + lane * 4;
         const float4 e4 = *reinterpret_cast<const float4*>(se + l);
         float4 g4;
-        if (off == 0) {
+        if constexpr (kBf16) {
+          if (off >= 0)
+            g4 = bf16x4(reinterpret_cast<const uint16_t*>(sm.g[s]) + off + warp * kSub + l);
+          else
+            g4 = load_g4_bf16(A.grads16 + (int64_t)k * A.d, s0 + l, A.d);
+        } else if (off == 0) {
           g4 = *reinterpret_cast<const float4*>(sg + l);
         } else if (off == 2) {
           const float2 a = *reinterpret_cast<const float2*>(sg + l);
@@ -474,15 +484,18 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
 cudaError_t configure_rbgs_kernels() {
   cudaError_t err = cudaFuncSetAttribute((const void*)k_rbgs_pick,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, kPickSmemWords * 4);
-  const cudaError_t e2 = cudaFuncSetAttribute((const void*)k_rbgs_bulk,
+  const cudaError_t e2 = cudaFuncSetAttribute((const void*)k_rbgs_bulk<false>,
                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               (int)sizeof(rbulk::Smem));
-  return err != cudaSuccess ? err : e2;
+  const cudaError_t e3 = cudaFuncSetAttribute((const void*)k_rbgs_bulk<true>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)sizeof(rbulk::Smem));
+  return err != cudaSuccess ? err : (e2 != cudaSuccess ? e2 : e3);
 }
 
 int rbgs_blocks_per_sm() {
   int n = 0;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_rbgs_step, kThreads, 0);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_rbgs_step<false>, kThreads, 0);
   return n > 0 ? n : 1;
 }
 
@@ -495,9 +508,15 @@ cudaError_t launch_rbgs_pick(const RbgsArgs& A, cudaStream_t s) {
 
 cudaError_t launch_rbgs_step(const RbgsArgs& A, int grid, cudaStream_t s) {
   if (A.bulk) {
-    k_rbgs_bulk<<<grid, rbulk::kThreadsAll, (int)sizeof(rbulk::Smem), s>>>(A);
+    if (A.bf16)
+      k_rbgs_bulk<true><<<grid, rbulk::kThreadsAll, (int)sizeof(rbulk::Smem), s>>>(A);
+    else
+      k_rbgs_bulk<false><<<grid, rbulk::kThreadsAll, (int)sizeof(rbulk::Smem), s>>>(A);
   } else {
-    k_rbgs_step<<<grid, kThreads, 0, s>>>(A);
+    if (A.bf16)
+      k_rbgs_step<true><<<grid, kThreads, 0, s>>>(A);
+    else
+      k_rbgs_step<false><<<grid, kThreads, 0, s>>>(A);
   }
   return cudaGetLastError();
 }

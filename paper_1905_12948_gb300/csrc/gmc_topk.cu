@@ -192,6 +192,7 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   }
   const float* ek = A.e + (int64_t)k * A.ld;
   const float* gk = A.grads + (int64_t)k * A.d;
+  const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
   uint32_t* keys = A.sample_keys + (int64_t)k * A.sample_stride;
   const int n_s = (int)A.n_sample;
   const uint64_t skey = sample_key(A);
@@ -210,12 +211,14 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
         const int64_t j = A.sample_pend[2 * A.sample_stride + i];
         const uint32_t m = A.sample_pend[i];
         ev[q] = ((m >> k) & 1u) ? 0.f : ek[j];
-        gv[q] = A.local_mom ? local_m(A, k, j, gk[j]) : (A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j]);
+        const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
+        gv[q] = A.local_mom ? local_m(A, k, j, g) : (A.gscale ? __fmul_rn(A.gs, g) : g);
         dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
       } else if (i < i_hi) {
         const int64_t j = sample_coord(A, skey, i);
         ev[q] = ek[j];
-        gv[q] = A.local_mom ? local_m(A, k, j, gk[j]) : (A.gscale ? __fmul_rn(A.gs, gk[j]) : gk[j]);
+        const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
+        gv[q] = A.local_mom ? local_m(A, k, j, g) : (A.gscale ? __fmul_rn(A.gs, g) : g);
         dv[q] = A.dlt[j];
         if (A.pending) {  // as if the previous step's aggregation were applied at j
           const uint32_t m = A.sample_pend[i];
@@ -656,7 +659,7 @@ __device__ __forceinline__ void write_group(const float v[4], uint32_t j, uint32
 // load/store version for small tiles; candidates share one region per worker
 // kLocal: the local-momentum baseline's instantiation (its momentum loads
 // need registers the other forms do without).
-template <int U, bool kLocal>
+template <int U, bool kLocal, bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
   constexpr int SUB = 128 * U;       // elements per warp and worker
   constexpr int T = kWarps * SUB;    // elements per tile
@@ -675,13 +678,15 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
       const uint32_t theta = A.sel[k].theta;
       float* ekt = A.e + (int64_t)k * A.ld + s0;
       const float* gk = A.grads + (int64_t)k * A.d;
+      const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
       const int gm = g_mode(gk);
       float4 ev[U], gv[U], mv[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const int l = u * 128 + lane * 4;
         ev[u] = __ldcs(reinterpret_cast<const float4*>(ekt + l));
-        gv[u] = scale_g(A, load_g4(gk, (int64_t)s0 + l, A.d, gm));
+        gv[u] = scale_g(A, kBf16 ? load_g4_bf16(gk16, (int64_t)s0 + l, A.d)
+                                 : load_g4(gk, (int64_t)s0 + l, A.d, gm));
         if (kLocal) mv[u] = __ldcs(reinterpret_cast<const float4*>(A.lm + (int64_t)k * A.ld + s0 + l));
       }
       if (kLocal) {
@@ -885,7 +890,7 @@ __device__ __forceinline__ uint32_t apply_pairs(const TopkArgs& A, uint32_t sub0
   return first ? l : ~0u;
 }
 
-template <bool kLocal>
+template <bool kLocal, bool kBf16>
 __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkArgs A) {
   using namespace bulk;
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -908,8 +913,10 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   if (warp == kProducer) {
     // ---- producer ----
     if (lane != 0) return;
-    const char* g_lo = reinterpret_cast<const char*>(A.grads);
-    const char* g_hi = reinterpret_cast<const char*>(A.grads + (int64_t)A.K * A.d);
+    // gradient rows of es-byte elements (fp32, or bf16 from gmc_step_bf16)
+    constexpr int es = kBf16 ? 2 : 4;
+    const char* g_lo = kBf16 ? reinterpret_cast<const char*>(A.grads16) : reinterpret_cast<const char*>(A.grads);
+    const char* g_hi = g_lo + (int64_t)A.K * A.d * es;
     uint32_t item = 0;
     bool ok = true;
     for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
@@ -922,11 +929,11 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
           break;
         }
         const float* esrc = A.e + (int64_t)k * A.ld + j0;
-        const uintptr_t ga = reinterpret_cast<uintptr_t>(A.grads + (int64_t)k * A.d + j0);
-        const uint32_t off = (uint32_t)(ga & 15) >> 2;
-        const char* gsrc = reinterpret_cast<const char*>(ga - off * 4);
-        const uint32_t gbytes = (uint32_t)(((nvalid + off) * 4 + 15) & ~int64_t(15));
-        const bool gbulk = !A.g_direct && (ga & 3) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
+        const uintptr_t ga = reinterpret_cast<uintptr_t>(g_lo + ((int64_t)k * A.d + j0) * es);
+        const uint32_t off = (uint32_t)(ga & 15) / es;  // leading elements before the row's tile
+        const char* gsrc = reinterpret_cast<const char*>(ga - off * es);
+        const uint32_t gbytes = (uint32_t)(((nvalid + off) * es + 15) & ~int64_t(15));
+        const bool gbulk = !A.g_direct && (ga % es) == 0 && gsrc >= g_lo && gsrc + gbytes <= g_hi;
         sm.gmeta[s] = gbulk ? (int32_t)off : -1;
         mbar_arrive_expect_tx(&sm.full[s], kT * 4 + (gbulk ? gbytes : 0));
         bulk_load(sm.e[s], esrc, kT * 4, &sm.full[s]);
@@ -1049,7 +1056,12 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         const int l = u * 128 + lane * 4;
         float4 e4 = *reinterpret_cast<const float4*>(se + l);
         float4 g4;
-        if (off == 0) {
+        if constexpr (kBf16) {
+          if (off >= 0)
+            g4 = bf16x4(reinterpret_cast<const uint16_t*>(sm.g[s]) + off + sw * kSub + l);
+          else
+            g4 = load_g4_bf16(A.grads16 + (int64_t)k * A.d, (int64_t)s0 + l, A.d);
+        } else if (off == 0) {
           g4 = *reinterpret_cast<const float4*>(sg + l);
         } else if (off == 2) {
           const float2 a = *reinterpret_cast<const float2*>(sg + l);
@@ -1768,14 +1780,22 @@ cudaError_t configure_topk_kernels() {
     const cudaError_t e2 = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (err == cudaSuccess) err = e2;
   };
-  set((const void*)k_accumulate<1, false>, 1024 * 12);
-  set((const void*)k_accumulate<2, false>, 2048 * 12);
-  set((const void*)k_accumulate<4, false>, 4096 * 12);
-  set((const void*)k_accumulate<1, true>, 1024 * 12);
-  set((const void*)k_accumulate<2, true>, 2048 * 12);
-  set((const void*)k_accumulate<4, true>, 4096 * 12);
-  set((const void*)k_accumulate_bulk<false>, bulk::smem_bytes(kBulkMaxK));
-  set((const void*)k_accumulate_bulk<true>, bulk::smem_bytes(kBulkMaxK));
+  set((const void*)k_accumulate<1, false, false>, 1024 * 12);
+  set((const void*)k_accumulate<2, false, false>, 2048 * 12);
+  set((const void*)k_accumulate<4, false, false>, 4096 * 12);
+  set((const void*)k_accumulate<1, true, false>, 1024 * 12);
+  set((const void*)k_accumulate<2, true, false>, 2048 * 12);
+  set((const void*)k_accumulate<4, true, false>, 4096 * 12);
+  set((const void*)k_accumulate<1, false, true>, 1024 * 12);
+  set((const void*)k_accumulate<2, false, true>, 2048 * 12);
+  set((const void*)k_accumulate<4, false, true>, 4096 * 12);
+  set((const void*)k_accumulate<1, true, true>, 1024 * 12);
+  set((const void*)k_accumulate<2, true, true>, 2048 * 12);
+  set((const void*)k_accumulate<4, true, true>, 4096 * 12);
+  set((const void*)k_accumulate_bulk<false, false>, bulk::smem_bytes(kBulkMaxK));
+  set((const void*)k_accumulate_bulk<true, false>, bulk::smem_bytes(kBulkMaxK));
+  set((const void*)k_accumulate_bulk<false, true>, bulk::smem_bytes(kBulkMaxK));
+  set((const void*)k_accumulate_bulk<true, true>, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_select_finish, 2 * kBucketCap * 4);
   set((const void*)k_sample_theta, kBucketCap * 4);
   return err;
@@ -1786,9 +1806,9 @@ int accumulate_blocks_per_sm(int tile) {
   int n = 0;
   const int smem = accumulate_smem_bytes(tile, kMaxK);
   switch (tile_u(tile)) {
-    case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<1, false>, kThreads, smem); break;
-    case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<2, false>, kThreads, smem); break;
-    default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<4, false>, kThreads, smem); break;
+    case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<1, false, false>, kThreads, smem); break;
+    case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<2, false, false>, kThreads, smem); break;
+    default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_accumulate<4, false, false>, kThreads, smem); break;
   }
   return n > 0 ? n : 1;
 }
@@ -1809,22 +1829,32 @@ cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+// The load/store pass's instantiation for the step's form and gradient type.
+template <int U>
+void launch_ls(const TopkArgs& A, int grid, int smem, cudaStream_t s) {
+  if (A.local_mom && A.bf16) k_accumulate<U, true, true><<<grid, kThreads, smem, s>>>(A);
+  else if (A.local_mom) k_accumulate<U, true, false><<<grid, kThreads, smem, s>>>(A);
+  else if (A.bf16) k_accumulate<U, false, true><<<grid, kThreads, smem, s>>>(A);
+  else k_accumulate<U, false, false><<<grid, kThreads, smem, s>>>(A);
+}
+
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
   const int smem = accumulate_smem_bytes(A.tile, A.K);
   if (use_bulk(A.tile)) {
-    if (A.local_mom)
-      k_accumulate_bulk<true><<<grid, bulk::kThreadsAll, smem, s>>>(A);
+    if (A.local_mom && A.bf16)
+      k_accumulate_bulk<true, true><<<grid, bulk::kThreadsAll, smem, s>>>(A);
+    else if (A.local_mom)
+      k_accumulate_bulk<true, false><<<grid, bulk::kThreadsAll, smem, s>>>(A);
+    else if (A.bf16)
+      k_accumulate_bulk<false, true><<<grid, bulk::kThreadsAll, smem, s>>>(A);
     else
-      k_accumulate_bulk<false><<<grid, bulk::kThreadsAll, smem, s>>>(A);
+      k_accumulate_bulk<false, false><<<grid, bulk::kThreadsAll, smem, s>>>(A);
     return cudaGetLastError();
   }
   switch (tile_u(A.tile)) {
-    case 1: A.local_mom ? k_accumulate<1, true><<<grid, kThreads, smem, s>>>(A)
-                        : k_accumulate<1, false><<<grid, kThreads, smem, s>>>(A); break;
-    case 2: A.local_mom ? k_accumulate<2, true><<<grid, kThreads, smem, s>>>(A)
-                        : k_accumulate<2, false><<<grid, kThreads, smem, s>>>(A); break;
-    default: A.local_mom ? k_accumulate<4, true><<<grid, kThreads, smem, s>>>(A)
-                         : k_accumulate<4, false><<<grid, kThreads, smem, s>>>(A); break;
+    case 1: launch_ls<1>(A, grid, smem, s); break;
+    case 2: launch_ls<2>(A, grid, smem, s); break;
+    default: launch_ls<4>(A, grid, smem, s); break;
   }
   return cudaGetLastError();
 }

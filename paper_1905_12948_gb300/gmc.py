@@ -42,6 +42,8 @@ _SIGNATURES = {
     "gmc_set_eta": (ctypes.c_int, [_c_p, _f32]),
     "gmc_set_select_mode": (ctypes.c_int, [_c_p, _i32]),
     "gmc_set_variant": (ctypes.c_int, [_c_p, _i32]),
+    "gmc_step_bf16": (ctypes.c_int, [_c_p, _c_p, _c_p]),
+    "gmc_step_host_bf16": (ctypes.c_int, [_c_p, _c_p, _c_p, _c_p]),
     "gmc_state_bytes": (_i64, [_c_p]),
     "gmc_save_state": (ctypes.c_int, [_c_p, _c_p, _i64]),
     "gmc_load_state": (ctypes.c_int, [_c_p, _c_p, _i64]),
@@ -177,19 +179,28 @@ class GMC:
                                        _stream_ptr(stream)), "gmc_set_params")
 
     def step(self, grads, stream=None) -> None:
+        """One step from device gradients: a K x d float32 CUDA tensor, or a
+        bfloat16 one (gmc_step_bf16: widened exactly, half the bytes)."""
         if tuple(grads.shape) != (self.K, self.d):
             raise ValueError("grads must have shape (K, d)")
+        if grads.dtype == self.torch.bfloat16:
+            _check(self.lib.gmc_step_bf16(self.h, _dev_ptr(grads, self.torch.bfloat16, "grads"),
+                                          _stream_ptr(stream)), "gmc_step_bf16")
+            return
         _check(self.lib.gmc_step(self.h, _dev_ptr(grads, self.torch.float32, "grads"),
                                  _stream_ptr(stream)), "gmc_step")
 
     def step_host(self, grads_host, stats_host=None, stream=None) -> None:
-        """One step from host gradients (pinned CPU float32 tensor K x d); the
-        step's counters land in stats_host (pinned CPU int64 tensor of 8)."""
+        """One step from host gradients (pinned CPU float32 or bfloat16 tensor
+        K x d); the step's counters land in stats_host (pinned CPU int64 tensor of 8)."""
         t = grads_host
-        if t.is_cuda or t.dtype != self.torch.float32 or not t.is_contiguous():
-            raise TypeError("grads_host must be a contiguous float32 CPU tensor")
+        if t.is_cuda or t.dtype not in (self.torch.float32, self.torch.bfloat16) or not t.is_contiguous():
+            raise TypeError("grads_host must be a contiguous float32 or bfloat16 CPU tensor")
+        if tuple(t.shape) != (self.K, self.d):
+            raise ValueError("grads_host must have shape (K, d)")
         sp = stats_host.data_ptr() if stats_host is not None else None
-        _check(self.lib.gmc_step_host(self.h, t.data_ptr(), sp, _stream_ptr(stream)), "gmc_step_host")
+        fn = self.lib.gmc_step_host_bf16 if t.dtype == self.torch.bfloat16 else self.lib.gmc_step_host
+        _check(fn(self.h, t.data_ptr(), sp, _stream_ptr(stream)), "gmc_step_host")
 
     # -- outputs --------------------------------------------------------------
     def params(self, stream=None):

@@ -53,6 +53,7 @@ class Workload:
     noniid: float = 0.0         # per-worker mean offset std as a multiple of the segment std
     iid_unit: bool = False      # gradients N(0,1) i.i.d., no segments
     w0_std: float = 0.01
+    grad_dtype: str = "f32"     # gradient input: "f32", or "bf16" (gmc_step_bf16: half the bytes)
     variant: str = "gmc"        # Alg. 1, the appendix's "server_momentum" (Alg. 3) / "lr_in_residual"
                                 # (Alg. 4), or the baseline "local_momentum" / "local_momentum_mfm"
 
@@ -84,6 +85,13 @@ WORKLOADS = [
     Workload("vgg16_alg4", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
              eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
              scale_lo=1e-4, scale_hi=1e-1, noniid=0.02, variant="lr_in_residual"),
+    # the vgg16 and resnet50 configurations with bfloat16 gradient input
+    Workload("vgg16_bf16", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
+             eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
+             scale_lo=1e-4, scale_hi=1e-1, noniid=0.02, grad_dtype="bf16"),
+    Workload("resnet50_bf16", d=25_557_032, K=32, compressor="rbgs", ratio=0.01, beta=0.9,
+             eta=0.1, steps=20, block=4096, lam=0.5, n_segments=161, noniid=0.02,
+             grad_dtype="bf16"),
     # and under the local-momentum baseline (DGC without / with momentum factor masking)
     Workload("vgg16_local", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
              eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
