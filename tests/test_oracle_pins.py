@@ -781,3 +781,38 @@ def test_p9_toy_quadratic_converges():
     d0 = float(np.linalg.norm(cfg["start"]))
     assert dist[500] < 1e-3 * d0
     assert max(dist[-1000:]) < 1e-4 * d0
+
+
+def _toy_distances(variant, d, s_fraction, start, steps=3000):
+    """Distances to the optimum w* = 0 of the two-worker quadratic of Sec. 3.2
+    (beta = 0.9, eta = 0.005, top-s), for one form of the step."""
+    i = np.arange(d)
+    wgt = (d - i).astype(np.float64)
+    o = GMC(d, 2, beta=0.9, eta=0.005, compressor=TOPK, ratio=s_fraction, variant=variant)
+    o.set_params(np.array(start, np.float32))
+    dist = []
+    for _ in range(steps):
+        w = o.w.astype(np.float64)
+        o.step(np.stack([2 * wgt * (w - (i + 1)), 2 * wgt * (w + (i + 1))]).astype(np.float32))
+        dist.append(float(np.linalg.norm(o.w.astype(np.float64))))
+    return np.array(dist)
+
+
+def test_p9b_toy_global_beats_local_momentum():
+    """Sec. 3.2, Figs. 1 and 2 (qualitative; parity unpinned: the figures carry
+    no numbers): GMC ends closer to the optimum than the local-momentum method
+    without masking, masking slows convergence down (d = 2, s = 0.5 d), and
+    for d = 20 GMC stays nearer the optimum than both local-momentum methods
+    at s = 0.1 d, 0.5 d and 0.8 d. The d = 20 start is not given in the paper;
+    this test reads it as 20 points evenly spaced from -1 to 2."""
+    cfg = _golden("toy_quadratic.json")
+    gmc = _toy_distances(oracle.ALG1, 2, 0.5, cfg["start"])
+    local = _toy_distances(oracle.LOCAL, 2, 0.5, cfg["start"])
+    mfm = _toy_distances(oracle.LOCAL_MFM, 2, 0.5, cfg["start"])
+    assert gmc[-1] < local[-1]
+    assert mfm[300] > gmc[300] and mfm[300] > local[300]
+    start = list(np.linspace(-1.0, 2.0, 20))
+    for s in (0.1, 0.5, 0.8):
+        tail = {v: _toy_distances(v, 20, s, start)[-1000:].mean()
+                for v in (oracle.ALG1, oracle.LOCAL, oracle.LOCAL_MFM)}
+        assert tail[oracle.ALG1] < tail[oracle.LOCAL] and tail[oracle.ALG1] < tail[oracle.LOCAL_MFM], (s, tail)
