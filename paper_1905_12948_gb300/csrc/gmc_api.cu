@@ -59,6 +59,8 @@ struct gmc_ctx {
   float* dlt = nullptr;
   WorkerSel* sel = nullptr;
   uint32_t* ghist = nullptr;
+  uint32_t* ghist2 = nullptr;  // K x 1024
+  bool sample_coop = false;    // the exact top-k's sample in one cooperative launch
   uint32_t* chist = nullptr;
   uint32_t* bucket = nullptr;  // K x 2*kBucketCap
   int sel_shift = 20;
@@ -249,6 +251,8 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.dense_mode = h->select_mode == GMC_SELECT_DENSE;
   A.sel = h->sel;
   A.ghist = h->ghist;
+  A.ghist2 = h->ghist2;
+  A.sample_coop = h->sample_coop ? 1 : 0;
   A.chist = h->chist;
   A.bucket = h->bucket;
   A.sel_shift = h->sel_shift;
@@ -555,11 +559,16 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     // select passes: about 2048 expected candidates per block
     const double expect = h->sample_chunks ? (double)d * h->sample_rank / (8.0 * kSampleChunks) : (double)h->ksel;
     const int64_t want = std::max<int64_t>(1, (int64_t)(expect / 2048.0));
-    h->sel_blocks = h->regions > 1 ? (int)std::min<int64_t>(h->regions, want)
+    // on the bulk path a warp visits candidate parts one after another, each a
+    // dependent load of its count and then of its keys: spread them over at
+    // least four blocks per SM's worth of warps
+    h->sel_blocks = h->regions > 1 ? (int)std::min<int64_t>(
+                                         h->regions, std::max<int64_t>(want, (4 * (int64_t)h->num_sms + K - 1) / K))
                                    : (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
     if (compressor == GMC_TOPK) h->n_sample = (uint32_t)(h->sample_chunks ? 8 * kSampleChunks : d);
     h->sample_stride = std::max<uint32_t>(kSampleSlots, (h->n_sample + 3) & ~3u);
     h->sample_blocks = (int)std::max<int64_t>(1, ((int64_t)h->n_sample + 2047) / 2048);
+    h->sample_coop = compressor == GMC_TOPK && sample_coop_fits(h->sample_blocks, K, h->num_sms);
     h->theta_blocks = (int)std::max<int64_t>(1, std::min<int64_t>(2 * h->num_sms / K + 1,
                                                                   ((int64_t)h->n_sample + 8191) / 8192));
     // relative-histogram bin width 2^sel_shift keys: near the k-th key a key
@@ -576,6 +585,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->dlt, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->sel, (size_t)K)) != cudaSuccess ||
         (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess ||
+        (err = dalloc(h, &h->ghist2, (size_t)K * 1024)) != cudaSuccess ||
         (err = dalloc(h, &h->chist, (size_t)K * kRelBins)) != cudaSuccess ||
         (err = dalloc(h, &h->bucket, (size_t)K * 2 * kBucketCap)) != cudaSuccess ||
         (err = dalloc(h, &h->sample_keys, (size_t)K * h->sample_stride)) != cudaSuccess ||

@@ -245,6 +245,35 @@ __device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity) {
   }
   return true;
 }
+// Barrier of the co-resident blocks (a cooperative launch) that share the
+// arrival counter ctr: each block arrives once per use, and waits until ctr
+// reaches target (its count of arrivals so far). Bounded: after 2 s it gives
+// up and returns false (the caller records kStatusTimeout). All threads of
+// the block must call it.
+__device__ __forceinline__ bool group_barrier(unsigned* ctr, unsigned target, unsigned* s_flag) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(ctr, 1u);
+    bool ok = true;
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    if (v < target) {
+      const uint64_t t0 = global_ns();
+      do {
+        __nanosleep(32);
+        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+        if (v < target && global_ns() - t0 > 2000000000ull) {
+          ok = false;
+          break;
+        }
+      } while (v < target);
+    }
+    *s_flag = ok ? 1u : 0u;
+  }
+  __syncthreads();
+  return *s_flag != 0u;
+}
 // Order this thread's generic-proxy shared-memory accesses before later
 // async-proxy (bulk copy) accesses to the same memory.
 __device__ __forceinline__ void fence_proxy_async() {

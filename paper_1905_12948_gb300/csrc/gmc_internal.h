@@ -74,6 +74,8 @@ struct TopkArgs {
   int dense_mode;            // GMC_SELECT_DENSE
   WorkerSel* sel;            // K entries
   uint32_t* ghist;           // K x kHistBins: the sample's histogram (zero between uses)
+  uint32_t* ghist2;          // K x 1024: its second digit in the first digit's bin (zero between uses)
+  int sample_coop;           // exact top-k: the sample in one cooperative launch (k_sample_coop)
   uint32_t* chist;           // K x kRelBins: the candidates' relative histogram (zeroed by the sample)
   uint32_t* bucket;          // K x 2*kBucketCap: keys, then indices of the k-th key's bin
   int sel_shift;             // log2 of the relative-histogram bin width (in keys)
@@ -183,6 +185,7 @@ int accumulate_blocks_per_sm(int tile);
 int rbgs_blocks_per_sm();
 int accumulate_smem_bytes(int tile, int K);
 cudaError_t configure_topk_kernels();
+bool sample_coop_fits(int blocks_per_worker, int K, int num_sms);
 cudaError_t configure_rbgs_kernels();
 
 constexpr int kRbgsTile = 4096;  // elements per tile of the fused RBGS kernel

@@ -331,6 +331,127 @@ __device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, u
 }
 
 // ---------------------------------------------------------------------------
+// The exact top-k's sample in one cooperative launch (all blocks co-resident):
+// the blocks of a worker form v at their slots (up to 8 per thread, kept in
+// registers), add their keys' first radix digit (bits 30..20) to the worker's
+// histogram, meet at a bounded barrier, find the bin of the r-th largest key,
+// add the second digit (bits 19..10) of their keys in that bin, meet again,
+// and read off theta = the two digits: a lower bound of the r-th largest
+// sampled key within 2^10 keys. No key is stored or read back.
+// ---------------------------------------------------------------------------
+constexpr int kCoopSlots = 8;  // sampled slots per thread
+
+__global__ void __launch_bounds__(kThreads) k_sample_coop(TopkArgs A) {
+  __shared__ uint32_t hist[kHistBins];
+  __shared__ uint32_t ws[32];
+  __shared__ uint32_t s_bin, s_rank, s_flag;
+  const int k = blockIdx.y;
+  WorkerSel& S = A.sel[k];
+  if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) A.big_tiles[0] = 0;
+  if (blockIdx.x == 0)  // this step's candidate histogram starts empty
+    for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) A.chist[(int64_t)k * kRelBins + b] = 0u;
+  if (A.dense_mode) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      S.theta = kNoCandidate;
+      S.count = 0;
+      S.dense = 0;
+    }
+    return;
+  }
+  const float* ek = A.e + (int64_t)k * A.ld;
+  const float* gk = A.grads + (int64_t)k * A.d;
+  const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
+  const int n_s = (int)A.n_sample;
+  const int per = (n_s + gridDim.x - 1) / gridDim.x;  // at most kCoopSlots * blockDim.x
+  const int i_lo = blockIdx.x * per;
+  const int i_hi = min(n_s, i_lo + per);
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0;
+  __syncthreads();
+  float ev[kCoopSlots], gv[kCoopSlots], dv[kCoopSlots];
+#pragma unroll
+  for (int q = 0; q < kCoopSlots; ++q) {
+    const int i = i_lo + q * blockDim.x + threadIdx.x;
+    ev[q] = gv[q] = dv[q] = 0.f;
+    if (i < i_hi) {
+      const int64_t j = sample_coord(A, 0ull, i);
+      ev[q] = ek[j];
+      const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
+      gv[q] = A.local_mom ? local_m(A, k, j, g) : (A.gscale ? __fmul_rn(A.gs, g) : g);
+      dv[q] = A.dlt[j];
+      if (A.pending) {  // as if the previous step's aggregation were applied at j
+        const uint32_t m = A.sample_pend[i];
+        if ((m >> k) & 1u) ev[q] = 0.f;
+        if (m) dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
+      }
+    }
+  }
+  uint32_t key[kCoopSlots];
+#pragma unroll
+  for (int q = 0; q < kCoopSlots; ++q) {
+    const int i = i_lo + q * blockDim.x + threadIdx.x;
+    key[q] = i < i_hi ? mag_key(accumulate(ev[q], gv[q], A.c, dv[q])) : 0xffffffffu;
+    warp_hist_add(hist, key[q] != 0xffffffffu ? (int)(key[q] >> 20) : -1);
+  }
+  __syncthreads();
+  uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
+  uint32_t* gh2 = A.ghist2 + (int64_t)k * 1024;
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
+    if (hist[b]) atomicAdd(&gh[b], hist[b]);
+  const unsigned n = gridDim.x;
+  bool ok = group_barrier(&S.done[3], n, &s_flag);
+  // the bin of the r-th largest key, and its rank there
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = __ldcg(&gh[b]);
+  if (threadIdx.x == 0) {
+    s_bin = 0;
+    s_rank = 0;
+  }
+  __syncthreads();
+  const uint32_t r = A.sample_rank < (uint32_t)n_s ? A.sample_rank : (uint32_t)n_s;
+  block_find_from_top(hist, kHistBins, r, ws, &s_bin, &s_rank);
+  const uint32_t b1 = s_bin, r1 = s_rank;
+  __syncthreads();
+  for (int b = threadIdx.x; b < 1024; b += blockDim.x) hist[b] = 0;
+  __syncthreads();
+#pragma unroll
+  for (int q = 0; q < kCoopSlots; ++q)
+    warp_hist_add(hist, (key[q] != 0xffffffffu && (key[q] >> 20) == b1) ? (int)((key[q] >> 10) & 1023u) : -1);
+  __syncthreads();
+  for (int b = threadIdx.x; b < 1024; b += blockDim.x)
+    if (hist[b]) atomicAdd(&gh2[b], hist[b]);
+  ok = group_barrier(&S.done[3], 2 * n, &s_flag) && ok;
+  for (int b = threadIdx.x; b < 1024; b += blockDim.x) hist[b] = __ldcg(&gh2[b]);
+  if (threadIdx.x == 0) {
+    s_bin = 0;
+    s_rank = 0;
+  }
+  __syncthreads();
+  block_find_from_top(hist, 1024, r1, ws, &s_bin, &s_rank);
+  if (threadIdx.x == 0) {
+    if (blockIdx.x == 0) {
+      // capped at the Inf key: every non-finite value is a candidate (and counted there)
+      S.theta = min((b1 << 20) | (s_bin << 10), 0x7f800000u);
+      S.count = 0;
+      S.dense = 0;
+    }
+    if (!ok) atomicOr(A.status, kStatusTimeout);
+    // the last block out clears the histograms and the counter for the next step
+    __threadfence();
+    s_flag = atomicAdd(&S.done[3], 1u) == 3 * n - 1 ? 1u : 0u;
+  }
+  __syncthreads();
+  if (s_flag) {
+    __threadfence();
+    for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) gh[b] = 0;
+    for (int b = threadIdx.x; b < 1024; b += blockDim.x) gh2[b] = 0;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      S.done[3] = 0;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Approximate top-s (Sec. 5.1): theta is the exact r-th largest sampled key.
 // Every block finds, from the sample's first-digit histogram, the bin that
 // holds it and collects that bin's keys from its slice of the sample (128 a
@@ -1278,7 +1399,9 @@ __global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
 }
 
 __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
-  extern __shared__ __align__(16) uint32_t fin[];  // kBucketCap keys + kBucketCap indices
+  // kBucketCap keys (the indices stay in the global bucket): 48 KB, so that
+  // four blocks fit on an SM and the grid runs in one wave
+  extern __shared__ __align__(16) uint32_t fin[];
   __shared__ uint32_t h[kHistBins];
   __shared__ uint32_t ws[32];
   __shared__ uint32_t s_last, s_bin, s_rank, s_n;
@@ -1356,11 +1479,7 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
     return;
   }
   uint32_t* keys = fin;
-  uint32_t* idxs = fin + kBucketCap;
-  for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) {
-    keys[i] = __ldcg(&bk[i]);
-    idxs[i] = __ldcg(&bk[kBucketCap + i]);
-  }
+  for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) keys[i] = __ldcg(&bk[i]);
   __syncthreads();
   uint32_t n_tie;
   const uint32_t T = smem_select(keys, n, want_rank, h, ws, &s_bin, &s_rank, &n_tie);
@@ -1371,7 +1490,7 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
     const uint32_t i = i0 + threadIdx.x;
     const bool tie = i < n && keys[i] == T;
-    const uint32_t j = tie ? idxs[i] : 0u;
+    const uint32_t j = tie ? __ldcg(&bk[kBucketCap + i]) : 0u;
     __syncthreads();
     if (tie) keys[atomicAdd(&s_n, 1u)] = j;
   }
@@ -1766,9 +1885,21 @@ __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uin
 }
 
 int tile_u(int tile) { return tile / (kWarps * 128); }
+
 bool use_bulk(int tile) { return tile == bulk::kT; }
 
 }  // namespace
+
+// Whether the exact top-k's sample (blocks_per_worker x K blocks) fits on the
+// GPU at once, as its cooperative launch requires.
+bool sample_coop_fits(int blocks_per_worker, int K, int num_sms) {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_sample_coop, kThreads, 0) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return (int64_t)n * num_sms >= (int64_t)blocks_per_worker * K;
+}
 
 int accumulate_smem_bytes(int tile, int K) {
   return use_bulk(tile) ? bulk::smem_bytes(K) : tile * 12;
@@ -1796,7 +1927,7 @@ cudaError_t configure_topk_kernels() {
   set((const void*)k_accumulate_bulk<true, false>, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_accumulate_bulk<false, true>, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_accumulate_bulk<true, true>, bulk::smem_bytes(kBulkMaxK));
-  set((const void*)k_select_finish, 2 * kBucketCap * 4);
+  set((const void*)k_select_finish, kBucketCap * 4);
   set((const void*)k_sample_theta, kBucketCap * 4);
   return err;
 }
@@ -1819,6 +1950,12 @@ cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
     k_sample_pending<<<(n_s + kThreads - 1) / kThreads, kThreads, 0, s>>>(A);
     const cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
+  }
+  if (A.sample_coop && !A.approx) {
+    TopkArgs a = A;
+    void* args[] = {&a};
+    return cudaLaunchCooperativeKernel((const void*)k_sample_coop, dim3(A.sample_blocks, A.K),
+                                       dim3(kThreads), args, 0, s);
   }
   k_sample<<<dim3(A.sample_blocks, A.K), kThreads, 0, s>>>(A);
   if (A.approx) {
@@ -1866,7 +2003,7 @@ cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t
     const cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
   }
-  k_select_finish<<<grid, kThreads, 2 * kBucketCap * 4, s>>>(A);
+  k_select_finish<<<grid, kThreads, kBucketCap * 4, s>>>(A);
   return cudaGetLastError();
 }
 
