@@ -289,6 +289,12 @@ int gmc_check(gmc_t h);
  * CUDA events on the step's stream; gmc_profile_read reports the totals. */
 int gmc_profile_enable(gmc_t h, int32_t on);
 
+/* gmc_profile_kernels -- which launches gmc_profile_enable brackets: bit k of
+ * kernel_mask selects kernel id k (GMC_KERNEL_*); default all. Each bracketed
+ * launch costs two event records on the stream, so timing only the kernels of
+ * interest keeps the step's own time undisturbed. */
+int gmc_profile_kernels(gmc_t h, uint32_t kernel_mask);
+
 /* gmc_profile_read -- synchronising. For kernel id `kernel` (GMC_KERNEL_*): the
  * summed device time in ms, the number of launches, and the algorithmic bytes
  * those launches had to move (the minimum traffic of the operation), since

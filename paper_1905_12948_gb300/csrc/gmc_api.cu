@@ -97,6 +97,7 @@ struct gmc_ctx {
   std::vector<void*> allocations;
   // profiling
   bool prof = false;
+  uint32_t prof_mask = 0xffffffffu;  // kernel ids bracketed by events while profiling
   std::vector<ProfRec> pending;
   std::vector<cudaEvent_t> free_events;
   double prof_ms[GMC_KERNEL_COUNT] = {};
@@ -172,7 +173,7 @@ cudaEvent_t take_event(gmc_ctx* h) {
 // Enqueue one kernel launch, bracketed by events when profiling is on.
 template <typename F>
 cudaError_t timed(gmc_ctx* h, int kernel, double bytes, cudaStream_t s, F&& launch) {
-  if (!h->prof) return launch();
+  if (!h->prof || !((h->prof_mask >> kernel) & 1u)) return launch();
   ProfRec r{kernel, take_event(h), take_event(h)};
   cudaEventRecord(r.start, s);
   cudaError_t err = launch();
@@ -1075,6 +1076,12 @@ int gmc_profile_enable(gmc_t h, int32_t on) {
     }
   }
   h->prof = on != 0;
+  return GMC_OK;
+}
+
+int gmc_profile_kernels(gmc_t h, uint32_t kernel_mask) {
+  if (!h) return GMC_EINVAL;
+  h->prof_mask = kernel_mask;
   return GMC_OK;
 }
 

@@ -42,6 +42,7 @@ _SIGNATURES = {
     "gmc_set_eta": (ctypes.c_int, [_c_p, _f32]),
     "gmc_set_select_mode": (ctypes.c_int, [_c_p, _i32]),
     "gmc_set_variant": (ctypes.c_int, [_c_p, _i32]),
+    "gmc_profile_kernels": (ctypes.c_int, [_c_p, ctypes.c_uint32]),
     "gmc_step_bf16": (ctypes.c_int, [_c_p, _c_p, _c_p]),
     "gmc_step_host_bf16": (ctypes.c_int, [_c_p, _c_p, _c_p, _c_p]),
     "gmc_state_bytes": (_i64, [_c_p]),
@@ -256,7 +257,10 @@ class GMC:
         return int(self.lib.gmc_check(self.h))
 
     # -- profiling ----------------------------------------------------------
-    def profile(self, on: bool = True) -> None:
+    def profile(self, on: bool = True, kernels=None) -> None:
+        """Bracket the step's launches with events (all kernels, or the named ones)."""
+        mask = 0xFFFFFFFF if kernels is None else sum(1 << KERNELS.index(k) for k in kernels)
+        _check(self.lib.gmc_profile_kernels(self.h, mask), "gmc_profile_kernels")
         _check(self.lib.gmc_profile_enable(self.h, int(on)), "gmc_profile_enable")
 
     def profile_read(self) -> dict:
