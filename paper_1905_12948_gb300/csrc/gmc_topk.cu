@@ -887,7 +887,7 @@ struct Smem {
   float g[kStages][kGLen];
   float dl[kSubTiles][kSub];               // w_t - w_{t-1} of a sub-tile
   uint32_t mk[kSubTiles][kSub];            // senders of the pending aggregation (bit k)
-  uint8_t own[kSubTiles][32];              // scratch: worker of each listed pair
+  uint8_t own[kConsumers][32];             // scratch of each consumer warp: worker of each listed pair
   uint32_t upos[kSubTiles][32];            // union coordinates of a sub-tile, one per lane
   uint32_t pflag[kSubTiles];               // per sub-tile: more than 32 pairs (per-element masks)
   uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
@@ -1074,10 +1074,9 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   const uint32_t lt = lanemask_lt();
   const int sw = warp & (kSubTiles - 1);  // sub-tile
   const int gp = warp / kSubTiles;         // workers k = gp, gp + 2, ...
-  const bool lead = gp == 0;               // forms the sub-tile's w_t - w_{t-1}
   float* dlw = sm.dl[sw];
   uint32_t* mkw = sm.mk[sw];
-  uint8_t* own = sm.own[sw];
+  uint8_t* own = sm.own[warp];
   // the sub-tile's part of the CTA's region, per worker: slots [part0, part0 + cap_part);
   // lane k counts worker k's candidates so far
   const uint32_t part0 = (blockIdx.x * kSubTiles + sw) * A.cap_part;
@@ -1088,20 +1087,21 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   uint32_t nonfinite = 0, uni = 0, chg = 0;
   bool ok = true;  // false after a bounded wait gave up: the items are skipped, the tile loop
                    // still runs (its named barriers need both warps of the sub-tile)
-  // fill the pipeline: pairs of tiles 0 and 1, w of tile 0, entries of tile 2
-  Pairs p0{kNone, 0.f, 0, 0u}, p1{kNone, 0.f, 0, 0u};
-  float w0 = 0.f;
-  uint2 c2 = make_uint2(0u, 0u);
-  if (lead) {
-    p0 = pipe_pairs(A, pipe_chunk(A, blockIdx.x, sw, lane), own, lane);
-    p1 = pipe_pairs(A, pipe_chunk(A, blockIdx.x + stride, sw, lane), own, lane);
-    w0 = pipe_w(A, p0, sm.Tp, sm.tip);
-    c2 = pipe_chunk(A, blockIdx.x + 2 * stride, sw, lane);
-  }
+  // The sub-tile's w_t - w_{t-1} is formed by one of its two warps, the
+  // tile's lead: warp gp leads the CTA's tiles n with n % 2 == gp, and
+  // pipelines the loads of its own tiles: the pairs of its next two, the w of
+  // its next one, the entries of the one after. Fill: its first three tiles.
+  const int64_t stride2 = 2 * stride;  // from one own tile to the next
+  const int64_t own0 = blockIdx.x + gp * stride;
+  Pairs p0 = pipe_pairs(A, pipe_chunk(A, own0, sw, lane), own, lane);
+  Pairs p1 = pipe_pairs(A, pipe_chunk(A, own0 + stride2, sw, lane), own, lane);
+  float w0 = pipe_w(A, p0, sm.Tp, sm.tip);
+  uint2 c2 = pipe_chunk(A, own0 + 2 * stride2, sw, lane);
   const uint32_t pair_bar = 1 + sw;  // named barrier of the sub-tile's two warps
   uint32_t n = 0;                    // tiles done
   for (int64_t tile = blockIdx.x; tile < A.n_tiles; tile += stride, ++n) {
     const uint32_t s0 = (uint32_t)(tile * kT) + sw * kSub;
+    const bool lead = (int)(n & 1u) == gp;
     // this sub-tile's w_t - w_{t-1}, and the pending senders (their residual
     // is +0): at most 32 union coordinates, one per lane (upos, umask), are
     // zeroed in each worker's stage before it is read; more use per-element masks
@@ -1134,10 +1134,10 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     float w1 = 0.f;
     Pairs p2{kNone, 0.f, 0, 0u};
     uint2 c3 = make_uint2(0u, 0u);
-    if (lead) {  // the next tiles' loads, in flight while this tile is processed
+    if (lead) {  // the loads of the lead's next own tiles, in flight meanwhile
       w1 = pipe_w(A, p1, sm.Tp, sm.tip);
       p2 = pipe_pairs(A, c2, own, lane);
-      c3 = pipe_chunk(A, tile + 3 * stride, sw, lane);
+      c3 = pipe_chunk(A, tile + 3 * stride2, sw, lane);
     }
     const int64_t rem = A.d - (int64_t)s0;
     const int lim = rem < kSub ? (int)rem : kSub;
