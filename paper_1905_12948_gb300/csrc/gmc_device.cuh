@@ -245,6 +245,13 @@ __device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity) {
   }
   return true;
 }
+// Programmatic dependent launch: a step's kernels are launched with
+// programmatic stream serialization, so one may be scheduled while the one
+// before it finishes; each waits here, before it touches memory, until its
+// predecessor's writes are visible. Without that launch attribute it returns
+// at once.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Barrier of the co-resident blocks (a cooperative launch) that share the
 // arrival counter ctr: each block arrives once per use, and waits until ctr
 // reaches target (its count of arrivals so far). Bounded: after 2 s it gives

@@ -152,6 +152,24 @@ struct DetachArgs {
   int k0, k1;                // workers [k0, k1)
 };
 
+// Launch with programmatic stream serialization (the kernel begins with
+// griddep_wait): its scheduling overlaps the end of the kernel before it.
+template <typename... P, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // Launch wrappers (each returns the cudaGetLastError of its launches).
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s);
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s);

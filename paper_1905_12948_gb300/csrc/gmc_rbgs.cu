@@ -49,6 +49,7 @@ __device__ __forceinline__ uint32_t block_of(int64_t j, const RbgsArgs& A) {
 // pick: one block per stream
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_rbgs_pick(RbgsArgs A) {
+  griddep_wait();
   extern __shared__ uint32_t bm_s[];
   __shared__ uint32_t ws[32];
   const int s = blockIdx.x;
@@ -103,6 +104,7 @@ __global__ void __launch_bounds__(kThreads) k_rbgs_pick(RbgsArgs A) {
 // ---------------------------------------------------------------------------
 template <bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_rbgs_step(RbgsArgs A) {
+  griddep_wait();
   constexpr int U = kRbgsTile / (kThreads * 4);  // float4 groups per thread
   __shared__ unsigned long long ws[32];
   uint32_t nonfinite = 0;
@@ -219,6 +221,7 @@ __global__ void __launch_bounds__(kThreads) k_rbgs_step(RbgsArgs A) {
 
 // (index, value) pairs of worker k's last C(.), in ascending index order.
 __global__ void k_rbgs_expand(RbgsArgs A, int k, uint32_t* idx_out, float* val_out) {
+  griddep_wait();
   const int64_t n = A.m * A.B;
   const int32_t* blk = A.blocks + (A.per_worker ? (int64_t)k * A.m : 0);
   const float* sk = A.slab + (int64_t)k * n;
@@ -235,6 +238,7 @@ __global__ void k_rbgs_expand(RbgsArgs A, int k, uint32_t* idx_out, float* val_o
 
 // GMC+ detach: out[k][j] = w[j] - b * e[k][j] (Alg. 2).
 __global__ void k_detach(DetachArgs A) {
+  griddep_wait();
   const int k = A.k0 + blockIdx.y;
   const float* ek = A.e + (int64_t)k * A.ld;
   float* ok = A.out + (int64_t)(k - A.k0) * A.out_ld;
@@ -244,6 +248,7 @@ __global__ void k_detach(DetachArgs A) {
 }
 
 __global__ void k_finalize(Counters* step, Counters* total, unsigned long long pairs_add) {
+  griddep_wait();
   if (threadIdx.x == 0) {
     step->v[kPairs] += pairs_add;
     step->v[kSteps] = 1;
@@ -279,6 +284,7 @@ struct Smem {
 
 template <bool kBf16>
 __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A) {
+  griddep_wait();
   using namespace rbulk;
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
@@ -502,23 +508,17 @@ int rbgs_blocks_per_sm() {
 cudaError_t launch_rbgs_pick(const RbgsArgs& A, cudaStream_t s) {
   const int64_t nbw = (A.nb + 31) / 32;
   const int smem = nbw <= kPickSmemWords ? (int)(nbw * 4) : 0;
-  k_rbgs_pick<<<A.per_worker ? A.K : 1, kThreads, smem, s>>>(A);
+  const cudaError_t err = launch_pdl(k_rbgs_pick, dim3(A.per_worker ? A.K : 1), dim3(kThreads), smem, s, A);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
 cudaError_t launch_rbgs_step(const RbgsArgs& A, int grid, cudaStream_t s) {
   if (A.bulk) {
-    if (A.bf16)
-      k_rbgs_bulk<true><<<grid, rbulk::kThreadsAll, (int)sizeof(rbulk::Smem), s>>>(A);
-    else
-      k_rbgs_bulk<false><<<grid, rbulk::kThreadsAll, (int)sizeof(rbulk::Smem), s>>>(A);
-  } else {
-    if (A.bf16)
-      k_rbgs_step<true><<<grid, kThreads, 0, s>>>(A);
-    else
-      k_rbgs_step<false><<<grid, kThreads, 0, s>>>(A);
+    return launch_pdl(A.bf16 ? k_rbgs_bulk<true> : k_rbgs_bulk<false>, dim3(grid), dim3(rbulk::kThreadsAll),
+                      sizeof(rbulk::Smem), s, A);
   }
-  return cudaGetLastError();
+  return launch_pdl(A.bf16 ? k_rbgs_step<true> : k_rbgs_step<false>, dim3(grid), dim3(kThreads), 0, s, A);
 }
 
 cudaError_t launch_rbgs_expand(const RbgsArgs& A, int k, uint32_t* idx_out, float* val_out,
@@ -532,13 +532,15 @@ cudaError_t launch_rbgs_expand(const RbgsArgs& A, int k, uint32_t* idx_out, floa
 cudaError_t launch_detach(const DetachArgs& A, cudaStream_t s) {
   const int64_t blocks = (A.d + 255) / 256;
   const dim3 grid((unsigned)(blocks < 1024 ? blocks : 1024), (unsigned)(A.k1 - A.k0));
-  k_detach<<<grid, 256, 0, s>>>(A);
+  const cudaError_t err = launch_pdl(k_detach, dim3(grid), dim3(256), 0, s, A);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(Counters* step, Counters* total, unsigned long long pairs_add,
                             cudaStream_t s) {
-  k_finalize<<<1, 32, 0, s>>>(step, total, pairs_add);
+  const cudaError_t err = launch_pdl(k_finalize, dim3(1), dim3(32), 0, s, step, total, pairs_add);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 

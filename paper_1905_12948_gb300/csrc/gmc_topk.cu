@@ -123,6 +123,7 @@ __device__ __forceinline__ uint64_t sample_key(const TopkArgs& A) {
 // slot's coordinate, and the step's w_t - w_{t-1} there (from dlt when no
 // aggregation is pending), for k_sample to read in order.
 __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
+  griddep_wait();
   __shared__ uint32_t Tp[kMaxK], tip[kMaxK];
   for (int kk = threadIdx.x; kk < A.K; kk += blockDim.x) {  // the previous step's selections
     Tp[kk] = A.sel[kk].T;
@@ -174,6 +175,7 @@ __device__ __forceinline__ int rel_bin(uint32_t key, uint32_t theta, int shift) 
 // had been applied (residual +0 where the worker sent, the pending delta).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
+  griddep_wait();
   __shared__ uint32_t hist[kHistBins];
   __shared__ uint32_t ws[32];
   __shared__ uint32_t s_last, s_bin, s_rank;
@@ -342,6 +344,7 @@ __device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, u
 constexpr int kCoopSlots = 8;  // sampled slots per thread
 
 __global__ void __launch_bounds__(kThreads) k_sample_coop(TopkArgs A) {
+  griddep_wait();
   __shared__ uint32_t hist[kHistBins];
   __shared__ uint32_t ws[32];
   __shared__ uint32_t s_bin, s_rank, s_flag;
@@ -460,6 +463,7 @@ __global__ void __launch_bounds__(kThreads) k_sample_coop(TopkArgs A) {
 // two remaining radix digits over the whole sample.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_sample_theta(TopkArgs A) {
+  griddep_wait();
   extern __shared__ __align__(16) uint32_t fin[];  // kBucketCap keys
   __shared__ uint32_t h[kHistBins];
   __shared__ uint32_t ws[32];
@@ -782,6 +786,7 @@ __device__ __forceinline__ void write_group(const float v[4], uint32_t j, uint32
 // need registers the other forms do without).
 template <int U, bool kLocal, bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
+  griddep_wait();
   constexpr int SUB = 128 * U;       // elements per warp and worker
   constexpr int T = kWarps * SUB;    // elements per tile
   extern __shared__ __align__(16) unsigned char smem[];
@@ -1013,6 +1018,7 @@ __device__ __forceinline__ uint32_t apply_pairs(const TopkArgs& A, uint32_t sub0
 
 template <bool kLocal, bool kBf16>
 __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkArgs A) {
+  griddep_wait();
   using namespace bulk;
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
@@ -1368,6 +1374,7 @@ __device__ __forceinline__ void candidate_part(const TopkArgs& A, int k, int p, 
 // The candidate histogram of the load/store pass (the bulk pass counts its
 // candidates into chist as they leave its staging lines).
 __global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
+  griddep_wait();
   __shared__ uint32_t h[kRelBins];
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
@@ -1399,6 +1406,7 @@ __global__ void __launch_bounds__(kThreads) k_select_hist(TopkArgs A) {
 }
 
 __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
+  griddep_wait();
   // kBucketCap keys (the indices stay in the global bucket): 48 KB, so that
   // four blocks fit on an SM and the grid runs in one wave
   extern __shared__ __align__(16) uint32_t fin[];
@@ -1520,6 +1528,7 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
 // overflowed, leaves the worker to the dense path.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_select_approx(TopkArgs A) {
+  griddep_wait();
   __shared__ uint32_t s_zero;
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
@@ -1560,6 +1569,7 @@ __global__ void __launch_bounds__(kThreads) k_select_approx(TopkArgs A) {
 // the exact top-`limit`.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
+  griddep_wait();
   const int k = blockIdx.x;
   WorkerSel& S = A.sel[k];
   if (A.approx ? S.dense == 0 : !needs_dense(S, A.ksel, A.cap)) return;
@@ -1717,6 +1727,7 @@ __device__ __forceinline__ void sent_part(const TopkArgs& A, int k, int p, int n
 }
 
 __global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A) {
+  griddep_wait();
   const int k = blockIdx.y;
   const uint32_t T = A.sel[k].T, tidx = A.sel[k].t_idx;
   const uint32_t bit = 1u << k;
@@ -1746,6 +1757,7 @@ __global__ void __launch_bounds__(kThreads) k_mark(TopkArgs A) {
 }
 
 __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
+  griddep_wait();
   const int k = blockIdx.y;
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
@@ -1806,6 +1818,7 @@ __global__ void __launch_bounds__(kThreads) k_owner_sum(TopkArgs A) {
 // dlt by the aggregate on the union, +0 elsewhere); then mom = w_{t+1} - w_t
 // (what fl(w_{t+1} - w_t) gives the next step) and dlt back to zero.
 __global__ void __launch_bounds__(kThreads) k_server_update(TopkArgs A) {
+  griddep_wait();
   unsigned long long changed = 0;
   const int64_t n4 = A.d >> 2;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -1845,6 +1858,7 @@ __global__ void __launch_bounds__(kThreads) k_server_update(TopkArgs A) {
 // sent candidates, tile by tile, sub-chunk by sub-chunk.
 __global__ void __launch_bounds__(1024) k_gather_selected(TopkArgs A, int k, uint32_t* idx_out,
                                                           float* val_out) {
+  griddep_wait();
   __shared__ uint32_t ws[32];
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
@@ -1947,8 +1961,7 @@ int accumulate_blocks_per_sm(int tile) {
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
   if ((A.pending || A.approx) && !A.dense_mode) {
     const int n_s = (int)A.n_sample;
-    k_sample_pending<<<(n_s + kThreads - 1) / kThreads, kThreads, 0, s>>>(A);
-    const cudaError_t err = cudaGetLastError();
+    const cudaError_t err = launch_pdl(k_sample_pending, dim3((n_s + kThreads - 1) / kThreads), dim3(kThreads), 0, s, A);
     if (err != cudaSuccess) return err;
   }
   if (A.sample_coop && !A.approx) {
@@ -1957,74 +1970,59 @@ cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
     return cudaLaunchCooperativeKernel((const void*)k_sample_coop, dim3(A.sample_blocks, A.K),
                                        dim3(kThreads), args, 0, s);
   }
-  k_sample<<<dim3(A.sample_blocks, A.K), kThreads, 0, s>>>(A);
-  if (A.approx) {
-    const cudaError_t err = cudaGetLastError();
-    if (err != cudaSuccess) return err;
-    k_sample_theta<<<dim3(A.theta_blocks, A.K), kThreads, kBucketCap * 4, s>>>(A);
-  }
-  return cudaGetLastError();
+  const cudaError_t err = launch_pdl(k_sample, dim3(A.sample_blocks, A.K), dim3(kThreads), 0, s, A);
+  if (err != cudaSuccess || !A.approx) return err;
+  return launch_pdl(k_sample_theta, dim3(A.theta_blocks, A.K), dim3(kThreads), kBucketCap * 4, s, A);
 }
 
 // The load/store pass's instantiation for the step's form and gradient type.
 template <int U>
-void launch_ls(const TopkArgs& A, int grid, int smem, cudaStream_t s) {
-  if (A.local_mom && A.bf16) k_accumulate<U, true, true><<<grid, kThreads, smem, s>>>(A);
-  else if (A.local_mom) k_accumulate<U, true, false><<<grid, kThreads, smem, s>>>(A);
-  else if (A.bf16) k_accumulate<U, false, true><<<grid, kThreads, smem, s>>>(A);
-  else k_accumulate<U, false, false><<<grid, kThreads, smem, s>>>(A);
+cudaError_t launch_ls(const TopkArgs& A, int grid, int smem, cudaStream_t s) {
+  if (A.local_mom && A.bf16) return launch_pdl(k_accumulate<U, true, true>, dim3(grid), dim3(kThreads), smem, s, A);
+  if (A.local_mom) return launch_pdl(k_accumulate<U, true, false>, dim3(grid), dim3(kThreads), smem, s, A);
+  if (A.bf16) return launch_pdl(k_accumulate<U, false, true>, dim3(grid), dim3(kThreads), smem, s, A);
+  return launch_pdl(k_accumulate<U, false, false>, dim3(grid), dim3(kThreads), smem, s, A);
 }
 
 cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
   const int smem = accumulate_smem_bytes(A.tile, A.K);
   if (use_bulk(A.tile)) {
-    if (A.local_mom && A.bf16)
-      k_accumulate_bulk<true, true><<<grid, bulk::kThreadsAll, smem, s>>>(A);
-    else if (A.local_mom)
-      k_accumulate_bulk<true, false><<<grid, bulk::kThreadsAll, smem, s>>>(A);
-    else if (A.bf16)
-      k_accumulate_bulk<false, true><<<grid, bulk::kThreadsAll, smem, s>>>(A);
-    else
-      k_accumulate_bulk<false, false><<<grid, bulk::kThreadsAll, smem, s>>>(A);
-    return cudaGetLastError();
+    const dim3 g(grid), b(bulk::kThreadsAll);
+    if (A.local_mom && A.bf16) return launch_pdl(k_accumulate_bulk<true, true>, g, b, smem, s, A);
+    if (A.local_mom) return launch_pdl(k_accumulate_bulk<true, false>, g, b, smem, s, A);
+    if (A.bf16) return launch_pdl(k_accumulate_bulk<false, true>, g, b, smem, s, A);
+    return launch_pdl(k_accumulate_bulk<false, false>, g, b, smem, s, A);
   }
   switch (tile_u(A.tile)) {
-    case 1: launch_ls<1>(A, grid, smem, s); break;
-    case 2: launch_ls<2>(A, grid, smem, s); break;
-    default: launch_ls<4>(A, grid, smem, s); break;
+    case 1: return launch_ls<1>(A, grid, smem, s);
+    case 2: return launch_ls<2>(A, grid, smem, s);
+    default: return launch_ls<4>(A, grid, smem, s);
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s) {
   const dim3 grid(blocks_per_worker, A.K);
   if (A.regions == 1) {  // the bulk pass histogrammed its candidates already
-    k_select_hist<<<grid, kThreads, 0, s>>>(A);
-    const cudaError_t err = cudaGetLastError();
+    const cudaError_t err = launch_pdl(k_select_hist, grid, dim3(kThreads), 0, s, A);
     if (err != cudaSuccess) return err;
   }
-  k_select_finish<<<grid, kThreads, kBucketCap * 4, s>>>(A);
-  return cudaGetLastError();
+  return launch_pdl(k_select_finish, grid, dim3(kThreads), kBucketCap * 4, s, A);
 }
 
 cudaError_t launch_select_approx(const TopkArgs& A, cudaStream_t s) {
-  k_select_approx<<<dim3(1, A.K), kThreads, 0, s>>>(A);
-  return cudaGetLastError();
+  return launch_pdl(k_select_approx, dim3(1, A.K), dim3(kThreads), 0, s, A);
 }
 
 cudaError_t launch_select_dense(const TopkArgs& A, cudaStream_t s) {
-  k_select_dense<<<A.K, 1024, 0, s>>>(A);
-  return cudaGetLastError();
+  return launch_pdl(k_select_dense, dim3(A.K), dim3(1024), 0, s, A);
 }
 
 cudaError_t launch_mark(const TopkArgs& A, int grid, cudaStream_t s) {
-  k_mark<<<dim3(grid, A.K), kThreads, 0, s>>>(A);
-  return cudaGetLastError();
+  return launch_pdl(k_mark, dim3(grid, A.K), dim3(kThreads), 0, s, A);
 }
 
 cudaError_t launch_owner_sum(const TopkArgs& A, int grid, cudaStream_t s) {
-  k_owner_sum<<<dim3(grid, A.K), kThreads, 0, s>>>(A);
-  return cudaGetLastError();
+  return launch_pdl(k_owner_sum, dim3(grid, A.K), dim3(kThreads), 0, s, A);
 }
 
 cudaError_t launch_server_update(const TopkArgs& A, cudaStream_t s) {
@@ -2035,8 +2033,7 @@ cudaError_t launch_server_update(const TopkArgs& A, cudaStream_t s) {
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int64_t want = (A.d / 4 + kThreads - 1) / kThreads;
   const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sms * std::max(n, 1)));
-  k_server_update<<<grid, kThreads, 0, s>>>(A);
-  return cudaGetLastError();
+  return launch_pdl(k_server_update, dim3(grid), dim3(kThreads), 0, s, A);
 }
 
 cudaError_t launch_gather_selected(const TopkArgs& A, int k, uint32_t* idx_out, float* val_out,
