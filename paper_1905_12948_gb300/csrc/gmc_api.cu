@@ -59,8 +59,6 @@ struct gmc_ctx {
   float* dlt = nullptr;
   WorkerSel* sel = nullptr;
   uint32_t* ghist = nullptr;
-  uint32_t* ghist2 = nullptr;  // K x 1024
-  bool sample_coop = false;    // the exact top-k's sample in one cooperative launch
   uint32_t* chist = nullptr;
   uint32_t* bucket = nullptr;  // K x 2*kBucketCap
   int sel_shift = 20;
@@ -91,6 +89,7 @@ struct gmc_ctx {
   uint8_t* uflag[2] = {nullptr, nullptr};
   float* slab = nullptr;
   Counters* step_ctr = nullptr;
+  uint32_t* tile_ctr = nullptr;  // tiles claimed by the persistent passes
   Counters* total_ctr = nullptr;
   unsigned* status = nullptr;
   float* gstage = nullptr;
@@ -229,7 +228,7 @@ void set_constants(gmc_ctx* h, TopkArgs* A) {
 
 // Arguments of step t's top-k kernels; chunk buffers alternate with the parity of t.
 TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
-  TopkArgs A;
+  TopkArgs A{};
   std::memset(&A, 0, sizeof(A));
   const int cur = (int)(t & 1), prev = cur ^ 1;
   A.e = h->e;
@@ -252,8 +251,6 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.dense_mode = h->select_mode == GMC_SELECT_DENSE;
   A.sel = h->sel;
   A.ghist = h->ghist;
-  A.ghist2 = h->ghist2;
-  A.sample_coop = h->sample_coop ? 1 : 0;
   A.chist = h->chist;
   A.bucket = h->bucket;
   A.sel_shift = h->sel_shift;
@@ -283,6 +280,7 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.a_prev = A.a;
   A.chunk_prev = h->chunk[prev];
   A.step_ctr = h->step_ctr;
+  A.tile_ctr = h->tile_ctr;
   A.status = h->status;
   return A;
 }
@@ -319,6 +317,7 @@ RbgsArgs rbgs_args(gmc_ctx* h, const float* grads) {
   A.slab = h->slab;
   A.has_prev = h->t > 0;
   A.step_ctr = h->step_ctr;
+  A.tile_ctr = h->tile_ctr;
   A.status = h->status;
   return A;
 }
@@ -350,8 +349,11 @@ int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, 
   const uint16_t* grads16 = bf16 ? static_cast<const uint16_t*>(grads_any) : nullptr;
   const double Kd = (double)h->K * (double)h->d;
   GMC_TRY(order_after_flush(h, s, true));
-  GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
+  // the exact top-k's sample kernel clears the step's counters itself (a
+  // memset between two kernels would keep the second from starting early)
+  if (h->compressor != GMC_TOPK) GMC_TRY(cudaMemsetAsync(h->step_ctr, 0, sizeof(Counters), s));
   unsigned long long pairs_add = 0;
+  bool finalized = false;  // the step's counters already added up by its last kernel
   if (h->compressor != GMC_RBGS) {
     const bool approx = h->compressor == GMC_TOPK_APPROX;
     TopkArgs A = topk_args(h, grads);
@@ -362,6 +364,11 @@ int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, 
     A.a_prev = h->a_pending;
     const bool defer = h->tile == kBulkTile && !eager && !h->detach_out && !A.server_mom && !A.mfm;
     const double kk = (double)h->K * (double)h->ksel;
+    pairs_add = approx ? 0ull : (unsigned long long)h->K * h->ksel;  // approximate: counted on the device
+    // deferred: the dense select is the step's last launch and ends it
+    A.finalize = defer ? 1 : 0;
+    A.pairs_add = pairs_add;
+    finalized = defer;
     GMC_TRY(timed(h, GMC_KERNEL_SAMPLE, 0.0, s, [&] { return launch_sample(A, s); }));
     // read g, e (and the local momentum), write v over e (and the momentum)
     GMC_TRY(timed(h, GMC_KERNEL_ACCUMULATE, ((A.local_mom ? 20.0 : 12.0) - (bf16 ? 2.0 : 0.0)) * Kd, s,
@@ -386,7 +393,6 @@ int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, 
         return err;
       }));
     }
-    pairs_add = approx ? 0ull : (unsigned long long)h->K * h->ksel;  // approximate: counted on the device
   } else {
     RbgsArgs A = rbgs_args(h, grads);
     A.grads16 = grads16;
@@ -404,8 +410,9 @@ int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, 
     DetachArgs D{h->w, h->e, h->ld, h->d, detach_b(h), h->detach_out, h->detach_ld, 0, h->K};
     GMC_TRY(timed(h, GMC_KERNEL_DETACH, 8.0 * Kd + 4.0 * h->d, s, [&] { return launch_detach(D, s); }));
   }
-  GMC_TRY(timed(h, GMC_KERNEL_OTHER, 0.0, s,
-                [&] { return launch_finalize(h->step_ctr, h->total_ctr, pairs_add, s); }));
+  if (!finalized)
+    GMC_TRY(timed(h, GMC_KERNEL_OTHER, 0.0, s,
+                  [&] { return launch_finalize(h->step_ctr, h->total_ctr, pairs_add, s); }));
   if (h->ev_step) GMC_TRY(cudaEventRecord(h->ev_step, s));
   h->t += 1;
   h->restored = false;
@@ -569,7 +576,6 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     if (compressor == GMC_TOPK) h->n_sample = (uint32_t)(h->sample_chunks ? 8 * kSampleChunks : d);
     h->sample_stride = std::max<uint32_t>(kSampleSlots, (h->n_sample + 3) & ~3u);
     h->sample_blocks = (int)std::max<int64_t>(1, ((int64_t)h->n_sample + 2047) / 2048);
-    h->sample_coop = compressor == GMC_TOPK && sample_coop_fits(h->sample_blocks, K, h->num_sms);
     h->theta_blocks = (int)std::max<int64_t>(1, std::min<int64_t>(2 * h->num_sms / K + 1,
                                                                   ((int64_t)h->n_sample + 8191) / 8192));
     // relative-histogram bin width 2^sel_shift keys: near the k-th key a key
@@ -586,7 +592,6 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->dlt, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->sel, (size_t)K)) != cudaSuccess ||
         (err = dalloc(h, &h->ghist, (size_t)K * kHistBins)) != cudaSuccess ||
-        (err = dalloc(h, &h->ghist2, (size_t)K * 1024)) != cudaSuccess ||
         (err = dalloc(h, &h->chist, (size_t)K * kRelBins)) != cudaSuccess ||
         (err = dalloc(h, &h->bucket, (size_t)K * 2 * kBucketCap)) != cudaSuccess ||
         (err = dalloc(h, &h->sample_keys, (size_t)K * h->sample_stride)) != cudaSuccess ||
@@ -634,6 +639,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
       return fail(err);
   }
   if ((err = dalloc(h, &h->step_ctr, 1)) != cudaSuccess ||
+      (err = dalloc(h, &h->tile_ctr, 1)) != cudaSuccess ||
       (err = dalloc(h, &h->total_ctr, 1)) != cudaSuccess ||
       (err = dalloc(h, &h->status, 1)) != cudaSuccess)
     return fail(err);

@@ -31,7 +31,8 @@ struct WorkerSel {
   uint32_t ties;     // candidates equal to T
   uint32_t t_idx;    // a candidate equal to T is kept iff its index <= t_idx
   uint32_t dense;    // 1: this worker's selection is made by the dense path
-  uint32_t done[4];  // finished-block counters: the two select passes, -, the sample
+  uint32_t done[4];  // finished-block counters: -, the select finish, the approximate
+                     // top-s threshold, and (worker 0's) the dense select's blocks
   uint32_t count_bucket;  // candidates collected from the k-th key's bin
   uint32_t nsel;     // approximate top-s: components sent (the count varies by step)
   uint32_t pad;
@@ -43,6 +44,16 @@ struct Counters {
 };
 enum CounterSlot { kSteps = 0, kPairs = 1, kNnz = 2, kUnion = 3, kChanged = 4,
                    kFallbacks = 5, kNonfinite = 6 };
+// The end of a step (one thread, after every kernel of the step that counts):
+// the pairs counted on the host, the step mark, and the step into the totals.
+// The step's counts may come from other blocks of the calling kernel: they
+// are read from L2.
+__device__ __forceinline__ void finalize_counters(Counters* step, Counters* total,
+                                                  unsigned long long pairs_add) {
+  step->v[kPairs] = __ldcg(&step->v[kPairs]) + pairs_add;
+  step->v[kSteps] = 1;
+  for (int i = 0; i < 8; ++i) total->v[i] += __ldcg(&step->v[i]);
+}
 
 // Device status bits (gmc_check).
 constexpr unsigned kStatusNonfinite = 1u;
@@ -252,35 +263,30 @@ __device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity) {
 // at once.
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
-// Barrier of the co-resident blocks (a cooperative launch) that share the
-// arrival counter ctr: each block arrives once per use, and waits until ctr
-// reaches target (its count of arrivals so far). Bounded: after 2 s it gives
-// up and returns false (the caller records kStatusTimeout). All threads of
-// the block must call it.
-__device__ __forceinline__ bool group_barrier(unsigned* ctr, unsigned target, unsigned* s_flag) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(ctr, 1u);
-    bool ok = true;
-    unsigned v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
-    if (v < target) {
-      const uint64_t t0 = global_ns();
-      do {
-        __nanosleep(32);
-        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
-        if (v < target && global_ns() - t0 > 2000000000ull) {
-          ok = false;
-          break;
-        }
-      } while (v < target);
-    }
-    *s_flag = ok ? 1u : 0u;
-  }
-  __syncthreads();
-  return *s_flag != 0u;
+// Tiles of a persistent streaming pass. A CTA's first kFixed tiles are fixed,
+// blockIdx.x + n * gridDim.x; every later one is claimed from a counter that
+// the step's previous kernel zeroed, kFixed - 1 tiles before the CTA starts
+// it, so that a CTA whose streams run faster takes more tiles and all of them
+// finish together. The CTA's producer thread, when it starts its tile n,
+// publishes the claim it made at tile n - 1 (for tile n - 1 + kFixed) in
+// tq[(n - 1 + kFixed) % kQ], and then claims the next one; a thread reads
+// tq[m % kQ] only after it has synchronised with the producer's start of tile
+// m + 1 - kFixed. kQ must exceed the tiles between the oldest slot a thread
+// may still read and the newest the producer may write.
+template <int kFixed, int kQ>
+__device__ __forceinline__ int64_t tile_at(const uint32_t* tq, uint32_t n) {
+  return n < (uint32_t)kFixed ? (int64_t)blockIdx.x + (int64_t)n * gridDim.x : (int64_t)tq[n % kQ];
 }
+// The producer's part at the start of its tile n: returns the tile.
+template <int kFixed, int kQ>
+__device__ __forceinline__ int64_t tile_claim(uint32_t* tq, uint32_t n, uint32_t* ctr, uint32_t& claim,
+                                              int64_t n_tiles) {
+  if (n > 0) tq[(n - 1 + kFixed) % kQ] = (uint32_t)kFixed * gridDim.x + claim;
+  const int64_t tile = tile_at<kFixed, kQ>(tq, n);
+  if (tile < n_tiles) claim = atomicAdd(ctr, 1u);
+  return tile;
+}
+
 // Order this thread's generic-proxy shared-memory accesses before later
 // async-proxy (bulk copy) accesses to the same memory.
 __device__ __forceinline__ void fence_proxy_async() {

@@ -57,7 +57,7 @@ struct TopkArgs {
   uint32_t* rcount;          // K x regions x kChunksPerTile: candidates written in each part
   uint32_t sample_rank;      // rank of the sampled threshold
   int sample_chunks;         // 0 = sample every element (or the approximate top-s sample)
-  int sample_blocks;         // blocks per worker of the sample kernel
+  int sample_blocks;         // blocks per worker of the approximate top-s sample (k_sample)
   uint32_t n_sample;         // sampled positions per worker
   uint32_t sample_stride;    // per-worker stride of sample_keys; offset of the delta half of sample_pend
   // Approximate top-s (Sec. 5.1): the sample is one position per stratum of
@@ -73,9 +73,7 @@ struct TopkArgs {
   int dense_prev;            // restored state: w_t - w_{t-1} is in dlt over [0, d), no pair lists
   int dense_mode;            // GMC_SELECT_DENSE
   WorkerSel* sel;            // K entries
-  uint32_t* ghist;           // K x kHistBins: the sample's histogram (zero between uses)
-  uint32_t* ghist2;          // K x 1024: its second digit in the first digit's bin (zero between uses)
-  int sample_coop;           // exact top-k: the sample in one cooperative launch (k_sample_coop)
+  uint32_t* ghist;           // K x kHistBins: the approximate top-s sample's histogram (zero between uses)
   uint32_t* chist;           // K x kRelBins: the candidates' relative histogram (zeroed by the sample)
   uint32_t* bucket;          // K x 2*kBucketCap: keys, then indices of the k-th key's bin
   int sel_shift;             // log2 of the relative-histogram bin width (in keys)
@@ -100,6 +98,9 @@ struct TopkArgs {
   Counters* total_ctr;       // running totals: the deferred aggregation counts there
   Counters* step_ctr;
   unsigned* status;
+  uint32_t* tile_ctr;        // tiles claimed by k_accumulate_bulk (zeroed by the sample kernel)
+  int finalize;              // k_select_dense ends the step: adds step_ctr (+ pairs_add pairs) to the totals
+  unsigned long long pairs_add;
 };
 
 // Slot of sub-chunk (k, tile, w) in the sub-chunk tables: a tile's entries are
@@ -137,6 +138,7 @@ struct RbgsArgs {
   int has_prev;
   int bulk;                  // k_rbgs_bulk (bulk copies through shared memory), else k_rbgs_step
   int g_direct;              // grads is mapped host memory: read it with loads, not bulk copies
+  uint32_t* tile_ctr;        // tiles claimed by k_rbgs_bulk (zeroed by k_rbgs_pick)
   Counters* step_ctr;
   unsigned* status;
 };
@@ -203,7 +205,6 @@ int accumulate_blocks_per_sm(int tile);
 int rbgs_blocks_per_sm();
 int accumulate_smem_bytes(int tile, int K);
 cudaError_t configure_topk_kernels();
-bool sample_coop_fits(int blocks_per_worker, int K, int num_sms);
 cudaError_t configure_rbgs_kernels();
 
 constexpr int kRbgsTile = 4096;  // elements per tile of the fused RBGS kernel

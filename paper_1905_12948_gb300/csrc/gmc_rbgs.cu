@@ -50,6 +50,7 @@ __device__ __forceinline__ uint32_t block_of(int64_t j, const RbgsArgs& A) {
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_rbgs_pick(RbgsArgs A) {
   griddep_wait();
+  if (blockIdx.x == 0 && threadIdx.x == 0) *A.tile_ctr = 0u;  // the fused pass claims its tiles from it
   extern __shared__ uint32_t bm_s[];
   __shared__ uint32_t ws[32];
   const int s = blockIdx.x;
@@ -249,11 +250,7 @@ __global__ void k_detach(DetachArgs A) {
 
 __global__ void k_finalize(Counters* step, Counters* total, unsigned long long pairs_add) {
   griddep_wait();
-  if (threadIdx.x == 0) {
-    step->v[kPairs] += pairs_add;
-    step->v[kSteps] = 1;
-    for (int i = 0; i < 8; ++i) total->v[i] += step->v[i];
-  }
+  if (threadIdx.x == 0) finalize_counters(step, total, pairs_add);
 }
 
 
@@ -263,7 +260,10 @@ __global__ void k_finalize(Counters* step, Counters* total, unsigned long long p
 // each (tile, worker) item's cp.async.bulk copies of e and g into the ring;
 // sixteen consumer warps each own 256 elements of every tile and run through
 // the K workers in ascending order (the aggregate adds in that order).
-// Producer and consumers meet only at mbarriers; every wait is bounded.
+// Producer and consumers meet only at mbarriers; every wait is bounded. A
+// CTA's first two tiles are fixed and every later one is claimed from a
+// counter (tile_at, tile_claim), so that CTAs whose streams run faster take
+// more tiles and all of them finish together.
 // ---------------------------------------------------------------------------
 namespace rbulk {
 constexpr int kT = kRbgsTile;
@@ -279,7 +279,16 @@ struct Smem {
   uint64_t full[kStages];                  // e, g landed (1 arrival + tx bytes)
   uint64_t empty[kStages];                 // all consumer warps read the stage
   int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
+  uint32_t tq[8];                          // claimed tiles (tile_at)
 };
+// Tiles: the first two of a CTA fixed, the rest claimed one tile ahead of the
+// producer's start of the tile before it. A consumer reads a tile's slot at
+// its start, after waiting on the previous tile's items (the producer's start
+// of that tile is two tiles on from the claim's); the producer runs at most
+// kStages items (tiles, for K = 1) ahead of the slowest consumer.
+constexpr int kFixed = 2;
+constexpr int kQ = 8;
+static_assert(kQ > kStages + kFixed, "the producer may overwrite a claimed tile not yet read");
 }  // namespace rbulk
 
 template <bool kBf16>
@@ -305,9 +314,11 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
     constexpr int es = kBf16 ? 2 : 4;
     const char* g_lo = kBf16 ? reinterpret_cast<const char*>(A.grads16) : reinterpret_cast<const char*>(A.grads);
     const char* g_hi = g_lo + (int64_t)A.K * A.d * es;
-    uint32_t item = 0;
+    uint32_t item = 0, claim = 0;
     bool ok = true;
-    for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+    for (uint32_t n = 0; ok; ++n) {
+      const int64_t tile = tile_claim<kFixed, kQ>(sm.tq, n, A.tile_ctr, claim, A.n_tiles);
+      if (tile >= A.n_tiles) break;
       const int64_t j0 = tile * kT;
       const int64_t nvalid = A.d - j0 < kT ? A.d - j0 : kT;
       for (int k = 0; k < A.K; ++k, ++item) {
@@ -343,7 +354,9 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
   unsigned long long pairs = 0, nnz = 0, uni = 0, changed = 0;
   uint32_t item = 0;
   bool ok = true;
-  for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+  for (uint32_t n = 0; ok; ++n) {
+    const int64_t tile = tile_at<kFixed, kQ>(sm.tq, n);
+    if (tile >= A.n_tiles) break;
     const int64_t s0 = tile * kT + warp * kSub;
     const int64_t rem = A.d - s0;
     const int lim = rem < kSub ? (rem > 0 ? (int)rem : 0) : kSub;

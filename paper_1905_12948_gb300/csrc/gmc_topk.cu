@@ -20,6 +20,8 @@
 // selected set is the first k elements under (key descending, index ascending).
 #include <algorithm>
 
+#include <cooperative_groups.h>
+
 #include "gmc_internal.h"
 
 namespace gmc {
@@ -169,19 +171,21 @@ __device__ __forceinline__ int rel_bin(uint32_t key, uint32_t theta, int shift) 
 }
 
 // ---------------------------------------------------------------------------
-// sample: blocks spread over the workers' samples; the last block of a worker
-// fixes two radix digits of the sample's r-th largest key. Where the previous
-// step's aggregation is pending, the sampled accumulator is formed as if it
-// had been applied (residual +0 where the worker sent, the pending delta).
+// Sample of the approximate top-s (Sec. 5.1): blocks spread over the workers'
+// samples store every sampled key and add its first radix digit to the
+// worker's histogram, for k_sample_theta. The accumulator at a sampled
+// coordinate is formed as if the previous step's aggregation had been applied
+// (residual +0 where the worker sent, the pending delta).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   griddep_wait();
   __shared__ uint32_t hist[kHistBins];
-  __shared__ uint32_t ws[32];
-  __shared__ uint32_t s_last, s_bin, s_rank;
   const int k = blockIdx.y;
   WorkerSel& S = A.sel[k];
-  if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) A.big_tiles[0] = 0;
+  if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) {
+    A.big_tiles[0] = 0;
+    *A.tile_ctr = 0u;  // the bulk pass claims its tiles from zero
+  }
   if (blockIdx.x == 0)  // this step's candidate histogram starts empty
     for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) A.chist[(int64_t)k * kRelBins + b] = 0u;
   if (A.dense_mode) {
@@ -197,7 +201,6 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
   uint32_t* keys = A.sample_keys + (int64_t)k * A.sample_stride;
   const int n_s = (int)A.n_sample;
-  const uint64_t skey = sample_key(A);
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0;
   __syncthreads();
   const int per = (n_s + gridDim.x - 1) / gridDim.x;
@@ -209,24 +212,13 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
     for (int q = 0; q < 8; ++q) {
       const int i = i0 + q * blockDim.x + threadIdx.x;
       ev[q] = gv[q] = dv[q] = 0.f;
-      if (i < i_hi && A.approx) {  // coordinate, senders and w_t - w_{t-1} from k_sample_pending
+      if (i < i_hi) {  // coordinate, senders and w_t - w_{t-1} from k_sample_pending
         const int64_t j = A.sample_pend[2 * A.sample_stride + i];
         const uint32_t m = A.sample_pend[i];
         ev[q] = ((m >> k) & 1u) ? 0.f : ek[j];
         const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
         gv[q] = A.local_mom ? local_m(A, k, j, g) : (A.gscale ? __fmul_rn(A.gs, g) : g);
         dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
-      } else if (i < i_hi) {
-        const int64_t j = sample_coord(A, skey, i);
-        ev[q] = ek[j];
-        const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
-        gv[q] = A.local_mom ? local_m(A, k, j, g) : (A.gscale ? __fmul_rn(A.gs, g) : g);
-        dv[q] = A.dlt[j];
-        if (A.pending) {  // as if the previous step's aggregation were applied at j
-          const uint32_t m = A.sample_pend[i];
-          if ((m >> k) & 1u) ev[q] = 0.f;
-          if (m) dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
-        }
       }
     }
 #pragma unroll
@@ -245,58 +237,7 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
     if (hist[b]) atomicAdd(&gh[b], hist[b]);
-  if (A.approx) return;  // k_sample_theta fixes theta exactly
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(&S.done[3], 1u) == gridDim.x - 1) ? 1u : 0u;
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) {
-    hist[b] = __ldcg(&gh[b]);
-    gh[b] = 0;
-  }
-  if (threadIdx.x == 0) {
-    S.done[3] = 0;
-    s_bin = 0;
-    s_rank = 0;
-  }
-  __syncthreads();
-  uint32_t r = A.sample_rank < (uint32_t)n_s ? A.sample_rank : (uint32_t)n_s;
-  block_find_from_top(hist, kHistBins, r, ws, &s_bin, &s_rank);
-  const uint32_t b1 = s_bin;
-  r = s_rank;
-  for (int b = threadIdx.x; b < 1024; b += blockDim.x) hist[b] = 0;
-  __syncthreads();
-  // second digit over all the worker's sample keys (n_s is a multiple of 8 or
-  // at most kSampleAll; keys are 16-byte aligned): 16 keys per thread per round
-  for (int i0 = 0; i0 < n_s; i0 += 16 * blockDim.x) {
-    uint32_t kv[16];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int i = i0 + (q * blockDim.x + threadIdx.x) * 4;
-      if (i + 3 < n_s) {
-        const uint4 x = __ldcg(reinterpret_cast<const uint4*>(keys + i));
-        kv[4 * q] = x.x; kv[4 * q + 1] = x.y; kv[4 * q + 2] = x.z; kv[4 * q + 3] = x.w;
-      } else {
-#pragma unroll
-        for (int t = 0; t < 4; ++t) kv[4 * q + t] = i + t < n_s ? __ldcg(keys + i + t) : 0xffffffffu;
-      }
-    }
-#pragma unroll
-    for (int t = 0; t < 16; ++t) {
-      const uint32_t key = kv[t];
-      warp_hist_add(hist, (key != 0xffffffffu && (key >> 20) == b1) ? (int)((key >> 10) & 1023u) : -1);
-    }
-  }
-  __syncthreads();
-  block_find_from_top(hist, 1024, r, ws, &s_bin, &s_rank);
-  if (threadIdx.x == 0) {
-    // capped at the Inf key: every non-finite value is a candidate (and counted there)
-    S.theta = min((b1 << 20) | (s_bin << 10), 0x7f800000u);
-    S.count = 0;
-    S.dense = 0;
-  }
+  // k_sample_theta fixes theta exactly from the keys and this histogram
 }
 
 // Radix select in shared memory: the r-th largest of n values (digits 11/10/10).
@@ -333,49 +274,72 @@ __device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, u
 }
 
 // ---------------------------------------------------------------------------
-// The exact top-k's sample in one cooperative launch (all blocks co-resident):
-// the blocks of a worker form v at their slots (up to 8 per thread, kept in
-// registers), add their keys' first radix digit (bits 30..20) to the worker's
-// histogram, meet at a bounded barrier, find the bin of the r-th largest key,
-// add the second digit (bits 19..10) of their keys in that bin, meet again,
-// and read off theta = the two digits: a lower bound of the r-th largest
-// sampled key within 2^10 keys. No key is stored or read back.
+// The exact top-k's sample with one thread-block cluster per worker (its CTAs
+// are co-scheduled by the hardware). Each CTA forms v at its slots (up to 8 per
+// thread, kept in registers) and adds its keys' first radix digit (bits
+// 30..20) into the histogram held in the shared memory of the cluster's first
+// CTA; after a cluster barrier every CTA reads it back and finds the bin of
+// the r-th largest key, adds the second digit (bits 19..10) of its keys in
+// that bin into a second histogram there, and after another barrier the first
+// CTA reads off theta = the two digits: a lower bound of the r-th largest
+// sampled key within 2^10 keys. Distributed shared memory and hardware
+// barriers only: no global scratch, no spin-wait.
 // ---------------------------------------------------------------------------
-constexpr int kCoopSlots = 8;  // sampled slots per thread
+namespace scl {
+constexpr int kCtas = 8;                                    // CTAs per cluster, one cluster per worker
+constexpr int kThreadsC = 512;
+constexpr int kSlots = kSampleSlots / (kCtas * kThreadsC);  // sampled slots per thread
+static_assert(kSlots * kCtas * kThreadsC == kSampleSlots, "the cluster covers the whole sample");
+static_assert(kHistBins % kThreadsC == 0 && 1024 % kThreadsC == 0, "histograms split evenly over a block");
+}  // namespace scl
 
-__global__ void __launch_bounds__(kThreads) k_sample_coop(TopkArgs A) {
+__global__ void __cluster_dims__(scl::kCtas, 1, 1) __launch_bounds__(scl::kThreadsC)
+    k_sample_cluster(TopkArgs A) {
+  using namespace scl;
   griddep_wait();
-  __shared__ uint32_t hist[kHistBins];
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  __shared__ uint32_t hist[kHistBins];  // this CTA's counts
+  __shared__ uint32_t red1[kHistBins];  // first CTA: the cluster's first-digit counts
+  __shared__ uint32_t red2[1024];       // first CTA: the cluster's second digits in the bin b1
   __shared__ uint32_t ws[32];
-  __shared__ uint32_t s_bin, s_rank, s_flag;
+  __shared__ uint32_t s_bin, s_rank;
   const int k = blockIdx.y;
+  const unsigned crank = cl.block_rank();
   WorkerSel& S = A.sel[k];
-  if (blockIdx.x == 0 && k == 0 && threadIdx.x == 0) A.big_tiles[0] = 0;
-  if (blockIdx.x == 0)  // this step's candidate histogram starts empty
+  if (crank == 0 && k == 0) {  // the step's first kernel that counts: its counters start at zero
+    if (threadIdx.x == 0) {
+      A.big_tiles[0] = 0;
+      *A.tile_ctr = 0u;  // and the bulk pass claims its tiles from zero
+    }
+    if (threadIdx.x < 8) A.step_ctr->v[threadIdx.x] = 0ull;
+  }
+  if (crank == 0)  // this step's candidate histogram starts empty
     for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) A.chist[(int64_t)k * kRelBins + b] = 0u;
-  if (A.dense_mode) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) {
+  if (A.dense_mode) {  // uniform over the grid: no CTA reaches a cluster barrier
+    if (crank == 0 && threadIdx.x == 0) {
       S.theta = kNoCandidate;
       S.count = 0;
       S.dense = 0;
     }
     return;
   }
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) {
+    hist[b] = 0;
+    red1[b] = 0;
+  }
+  for (int b = threadIdx.x; b < 1024; b += blockDim.x) red2[b] = 0;
   const float* ek = A.e + (int64_t)k * A.ld;
   const float* gk = A.grads + (int64_t)k * A.d;
   const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
-  const int n_s = (int)A.n_sample;
-  const int per = (n_s + gridDim.x - 1) / gridDim.x;  // at most kCoopSlots * blockDim.x
-  const int i_lo = blockIdx.x * per;
-  const int i_hi = min(n_s, i_lo + per);
-  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0;
-  __syncthreads();
-  float ev[kCoopSlots], gv[kCoopSlots], dv[kCoopSlots];
+  const int n_s = (int)A.n_sample;  // at most kSampleSlots
+  const int i_lo = (int)crank * (kSlots * kThreadsC);
+  float ev[kSlots], gv[kSlots], dv[kSlots];
 #pragma unroll
-  for (int q = 0; q < kCoopSlots; ++q) {
-    const int i = i_lo + q * blockDim.x + threadIdx.x;
+  for (int q = 0; q < kSlots; ++q) {
+    const int i = i_lo + q * kThreadsC + threadIdx.x;
     ev[q] = gv[q] = dv[q] = 0.f;
-    if (i < i_hi) {
+    if (i < n_s) {
       const int64_t j = sample_coord(A, 0ull, i);
       ev[q] = ek[j];
       const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
@@ -388,22 +352,21 @@ __global__ void __launch_bounds__(kThreads) k_sample_coop(TopkArgs A) {
       }
     }
   }
-  uint32_t key[kCoopSlots];
+  uint32_t key[kSlots];
 #pragma unroll
-  for (int q = 0; q < kCoopSlots; ++q) {
-    const int i = i_lo + q * blockDim.x + threadIdx.x;
-    key[q] = i < i_hi ? mag_key(accumulate(ev[q], gv[q], A.c, dv[q])) : 0xffffffffu;
+  for (int q = 0; q < kSlots; ++q) {
+    const int i = i_lo + q * kThreadsC + threadIdx.x;
+    key[q] = i < n_s ? mag_key(accumulate(ev[q], gv[q], A.c, dv[q])) : 0xffffffffu;
     warp_hist_add(hist, key[q] != 0xffffffffu ? (int)(key[q] >> 20) : -1);
   }
-  __syncthreads();
-  uint32_t* gh = A.ghist + (int64_t)k * kHistBins;
-  uint32_t* gh2 = A.ghist2 + (int64_t)k * 1024;
+  // every CTA of the cluster runs and has zeroed its histograms before any remote add
+  cl.sync();
+  uint32_t* r1 = cl.map_shared_rank(red1, 0);
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
-    if (hist[b]) atomicAdd(&gh[b], hist[b]);
-  const unsigned n = gridDim.x;
-  bool ok = group_barrier(&S.done[3], n, &s_flag);
-  // the bin of the r-th largest key, and its rank there
-  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = __ldcg(&gh[b]);
+    if (hist[b]) atomicAdd(&r1[b], hist[b]);
+  cl.sync();
+  // the bin of the r-th largest key and its rank there (every CTA alike)
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = r1[b];
   if (threadIdx.x == 0) {
     s_bin = 0;
     s_rank = 0;
@@ -411,46 +374,30 @@ __global__ void __launch_bounds__(kThreads) k_sample_coop(TopkArgs A) {
   __syncthreads();
   const uint32_t r = A.sample_rank < (uint32_t)n_s ? A.sample_rank : (uint32_t)n_s;
   block_find_from_top(hist, kHistBins, r, ws, &s_bin, &s_rank);
-  const uint32_t b1 = s_bin, r1 = s_rank;
-  __syncthreads();
+  const uint32_t b1 = s_bin, rr = s_rank;
   for (int b = threadIdx.x; b < 1024; b += blockDim.x) hist[b] = 0;
   __syncthreads();
 #pragma unroll
-  for (int q = 0; q < kCoopSlots; ++q)
+  for (int q = 0; q < kSlots; ++q)
     warp_hist_add(hist, (key[q] != 0xffffffffu && (key[q] >> 20) == b1) ? (int)((key[q] >> 10) & 1023u) : -1);
   __syncthreads();
+  uint32_t* r2 = cl.map_shared_rank(red2, 0);
   for (int b = threadIdx.x; b < 1024; b += blockDim.x)
-    if (hist[b]) atomicAdd(&gh2[b], hist[b]);
-  ok = group_barrier(&S.done[3], 2 * n, &s_flag) && ok;
-  for (int b = threadIdx.x; b < 1024; b += blockDim.x) hist[b] = __ldcg(&gh2[b]);
+    if (hist[b]) atomicAdd(&r2[b], hist[b]);
+  // after this barrier no CTA touches another's shared memory
+  cl.sync();
+  if (crank != 0) return;
   if (threadIdx.x == 0) {
     s_bin = 0;
     s_rank = 0;
   }
   __syncthreads();
-  block_find_from_top(hist, 1024, r1, ws, &s_bin, &s_rank);
+  block_find_from_top(red2, 1024, rr, ws, &s_bin, &s_rank);
   if (threadIdx.x == 0) {
-    if (blockIdx.x == 0) {
-      // capped at the Inf key: every non-finite value is a candidate (and counted there)
-      S.theta = min((b1 << 20) | (s_bin << 10), 0x7f800000u);
-      S.count = 0;
-      S.dense = 0;
-    }
-    if (!ok) atomicOr(A.status, kStatusTimeout);
-    // the last block out clears the histograms and the counter for the next step
-    __threadfence();
-    s_flag = atomicAdd(&S.done[3], 1u) == 3 * n - 1 ? 1u : 0u;
-  }
-  __syncthreads();
-  if (s_flag) {
-    __threadfence();
-    for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) gh[b] = 0;
-    for (int b = threadIdx.x; b < 1024; b += blockDim.x) gh2[b] = 0;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      __threadfence();
-      S.done[3] = 0;
-    }
+    // capped at the Inf key: every non-finite value is a candidate (and counted there)
+    S.theta = min((b1 << 20) | (s_bin << 10), 0x7f800000u);
+    S.count = 0;
+    S.dense = 0;
   }
 }
 
@@ -877,10 +824,20 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 // tile n+1, the pairs of tile n+2 and the sub-chunk entries of tile n+3, so
 // no latency lies on its path. A sub-tile with more than 32 pairs takes the
 // direct path (stage_pending_warp / stage_delta_warp).
+//
+// A CTA's first tiles are fixed and every later one is claimed from a counter
+// (tile_at, tile_claim), so that CTAs whose streams run faster take more
+// tiles and all of them finish together.
 // ---------------------------------------------------------------------------
 namespace bulk {
 constexpr int kT = kBulkTile;
 constexpr int kStages = 4;                 // shared-memory ring of (e, g) tiles
+// Each worker-parity warp group has its own kGroupStages of the ring, which it
+// reads in order: an mbarrier wait by phase parity can only tell the phase it
+// waits for from the one before, so no warp may wait on a stage two phases
+// ahead, as it could if the groups shared stages (an odd K, or a ring whose
+// size is not twice a group's share).
+constexpr int kGroupStages = kStages / 2;
 constexpr int kSubTiles = kChunksPerTile;  // 8 sub-tiles of 512 elements
 constexpr int kSub = kT / kSubTiles;       // 512
 constexpr int kConsumers = 2 * kSubTiles;  // warps 0..15: sub-tile w & 7, workers of parity w >> 3
@@ -900,9 +857,21 @@ struct Smem {
   int32_t gmeta[kStages];                  // leading floats in the g stage, -1 = not copied
   uint32_t theta[kMaxK];
   uint32_t Tp[kMaxK], tip[kMaxK];          // the previous step's selection (T, t_idx) per worker
+  uint32_t tq[16];                         // claimed tiles (tile_at)
+  uint32_t next[kSubTiles];                // per sub-tile: the next tile of its two warps
   // followed by the candidate staging lines: per consumer warp and worker, 32
   // indices then 32 values (staging_bytes)
 };
+// Tiles: a CTA's first five fixed, the rest claimed four tiles ahead of the
+// producer's start of the tile before it. Only the lead warp of a sub-tile
+// (it has worker 0's items) reads the queue; the earliest read of a slot is
+// its load of tile n + 3's sub-chunk entries during tile n, after it waited
+// on an item of tile n - 1, whose issue followed the producer's publishing of
+// slots up to n + 3. The producer runs at most kStages items (tiles, for
+// K <= 2) ahead of the slowest consumer.
+constexpr int kFixed = 5;
+constexpr int kQ = 16;
+static_assert(kQ > kStages + kFixed, "the producer may overwrite a claimed tile not yet read");
 // Dynamic shared memory of the bulk pass for K workers.
 __host__ __device__ constexpr int smem_bytes(int K) {
   return (int)((sizeof(Smem) + 127) / 128 * 128) + kSubTiles * K * 64 * 4;
@@ -1026,7 +995,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], kSubTiles);  // the eight warps of the item's worker parity
+      mbar_init(&sm.empty[s], kSubTiles);  // the eight warps of the stage's worker parity
     }
     fence_mbar_init();
   }
@@ -1044,13 +1013,17 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     constexpr int es = kBf16 ? 2 : 4;
     const char* g_lo = kBf16 ? reinterpret_cast<const char*>(A.grads16) : reinterpret_cast<const char*>(A.grads);
     const char* g_hi = g_lo + (int64_t)A.K * A.d * es;
-    uint32_t item = 0;
+    uint32_t issued[2] = {0u, 0u};  // items issued to each worker-parity group
+    uint32_t claim = 0;
     bool ok = true;
-    for (int64_t tile = blockIdx.x; ok && tile < A.n_tiles; tile += gridDim.x) {
+    for (uint32_t n = 0; ok; ++n) {
+      const int64_t tile = tile_claim<kFixed, kQ>(sm.tq, n, A.tile_ctr, claim, A.n_tiles);
+      if (tile >= A.n_tiles) break;
       const int64_t j0 = tile * kT;
       const int64_t nvalid = A.d - j0 < kT ? A.d - j0 : kT;
-      for (int k = 0; k < A.K; ++k, ++item) {
-        const uint32_t s = item % kStages, r = item / kStages;
+      for (int k = 0; k < A.K; ++k) {
+        const uint32_t grp = (uint32_t)k & 1u, c = issued[grp];
+        const uint32_t s = grp * kGroupStages + c % kGroupStages, r = c / kGroupStages;
         if (r > 0 && !wait_bounded(&sm.empty[s], (r - 1) & 1)) {
           ok = false;
           break;
@@ -1065,13 +1038,17 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         mbar_arrive_expect_tx(&sm.full[s], kT * 4 + (gbulk ? gbytes : 0));
         bulk_load(sm.e[s], esrc, kT * 4, &sm.full[s]);
         if (gbulk) bulk_load(sm.g[s], gsrc, gbytes, &sm.full[s]);
+        issued[grp] = c + 1;
       }
     }
     if (!ok) {
       atomicOr(A.status, kStatusTimeout);
       // let the copies already issued land before the CTA's shared memory goes away
-      const uint32_t first = item > (uint32_t)kStages ? item - kStages : 0u;
-      for (uint32_t i = first; i < item; ++i) wait_bounded(&sm.full[i % kStages], (i / kStages) & 1);
+      for (uint32_t grp = 0; grp < 2; ++grp) {
+        const uint32_t c1 = issued[grp], c0 = c1 > (uint32_t)kGroupStages ? c1 - kGroupStages : 0u;
+        for (uint32_t c = c0; c < c1; ++c)
+          wait_bounded(&sm.full[grp * kGroupStages + c % kGroupStages], (c / kGroupStages) & 1);
+      }
     }
     return;
   }
@@ -1089,25 +1066,31 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   uint32_t* stg = reinterpret_cast<uint32_t*>(smem_raw + (sizeof(Smem) + 127) / 128 * 128) +
                   sw * A.K * 64;
   uint32_t run = 0;
-  const int64_t stride = gridDim.x;
+  uint32_t taken = 0;  // items of this warp's group read so far (its stages, in order)
   uint32_t nonfinite = 0, uni = 0, chg = 0;
   bool ok = true;  // false after a bounded wait gave up: the items are skipped, the tile loop
                    // still runs (its named barriers need both warps of the sub-tile)
-  // The sub-tile's w_t - w_{t-1} is formed by one of its two warps, the
-  // tile's lead: warp gp leads the CTA's tiles n with n % 2 == gp, and
-  // pipelines the loads of its own tiles: the pairs of its next two, the w of
-  // its next one, the entries of the one after. Fill: its first three tiles.
-  const int64_t stride2 = 2 * stride;  // from one own tile to the next
-  const int64_t own0 = blockIdx.x + gp * stride;
-  Pairs p0 = pipe_pairs(A, pipe_chunk(A, own0, sw, lane), own, lane);
-  Pairs p1 = pipe_pairs(A, pipe_chunk(A, own0 + stride2, sw, lane), own, lane);
-  float w0 = pipe_w(A, p0, sm.Tp, sm.tip);
-  uint2 c2 = pipe_chunk(A, own0 + 2 * stride2, sw, lane);
+  // The sub-tile's w_t - w_{t-1} is formed by one of its two warps, the lead
+  // (the warp of the even workers), which pipelines the loads of the CTA's
+  // next tiles: while it works on tile n it loads w for tile n + 1, the pairs
+  // of tile n + 2 and the sub-chunk entries of tile n + 3. Fill: tiles 0-2.
+  const bool lead = gp == 0;
+  Pairs p0{kNone, 0.f, 0, 0u}, p1{kNone, 0.f, 0, 0u};
+  float w0 = 0.f;
+  uint2 c2 = make_uint2(0u, 0u);
+  if (lead) {
+    p0 = pipe_pairs(A, pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, 0), sw, lane), own, lane);
+    p1 = pipe_pairs(A, pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, 1), sw, lane), own, lane);
+    w0 = pipe_w(A, p0, sm.Tp, sm.tip);
+    c2 = pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, 2), sw, lane);
+  }
   const uint32_t pair_bar = 1 + sw;  // named barrier of the sub-tile's two warps
-  uint32_t n = 0;                    // tiles done
-  for (int64_t tile = blockIdx.x; tile < A.n_tiles; tile += stride, ++n) {
+  // The sub-tile's two warps take their next tile from one read of its
+  // queue slot (sm.next), so that both leave the loop together: the named
+  // barriers need both. A warp whose wait gave up ends the CTA's tiles.
+  int64_t tile = tile_at<kFixed, kQ>(sm.tq, 0);
+  for (uint32_t n = 0; tile < A.n_tiles; ++n) {  // n: tiles done
     const uint32_t s0 = (uint32_t)(tile * kT) + sw * kSub;
-    const bool lead = (int)(n & 1u) == gp;
     // this sub-tile's w_t - w_{t-1}, and the pending senders (their residual
     // is +0): at most 32 union coordinates, one per lane (upos, umask), are
     // zeroed in each worker's stage before it is read; more use per-element masks
@@ -1135,15 +1118,18 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     float4 dl4[kSub / 128];
 #pragma unroll
     for (int u = 0; u < kSub / 128; ++u) dl4[u] = *reinterpret_cast<const float4*>(dlw + u * 128 + lane * 4);
+    if (lead && lane == 0)  // the slot of tile n + 1 was published before tile n - 3's items
+      sm.next[sw] = (!ok || n + 1 >= (uint64_t)A.n_tiles) ? (uint32_t)A.n_tiles
+                                                          : (uint32_t)tile_at<kFixed, kQ>(sm.tq, n + 1);
     // the lead warp rewrites the sub-tile's buffers for the next tile only after this
     asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
     float w1 = 0.f;
     Pairs p2{kNone, 0.f, 0, 0u};
     uint2 c3 = make_uint2(0u, 0u);
-    if (lead) {  // the loads of the lead's next own tiles, in flight meanwhile
+    if (lead) {  // the next tiles' loads, in flight while this tile is processed
       w1 = pipe_w(A, p1, sm.Tp, sm.tip);
       p2 = pipe_pairs(A, c2, own, lane);
-      c3 = pipe_chunk(A, tile + 3 * stride2, sw, lane);
+      c3 = pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, n + 3), sw, lane);
     }
     const int64_t rem = A.d - (int64_t)s0;
     const int lim = rem < kSub ? (int)rem : kSub;
@@ -1155,8 +1141,8 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
       for (int i = 0; i < 4; ++i) valid |= (u * 128 + lane * 4 + i < lim ? 1u : 0u) << (4 * u + i);
     uint2 bc_lane = make_uint2(0u, 0u);
     for (int k = gp; ok && k < A.K; k += 2) {
-      const uint32_t item = n * (uint32_t)A.K + (uint32_t)k;
-      const uint32_t s = item % kStages, r = item / kStages;
+      const uint32_t s = gp * kGroupStages + taken % kGroupStages, r = taken / kGroupStages;
+      ++taken;
       float4 mv[kSub / 128];  // the local-momentum baseline: m loaded while the stage lands
       if (kLocal) {
 #pragma unroll
@@ -1306,6 +1292,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     }
     // the per-element masks of a many-sender sub-tile stay in use until both warps are done
     if (many) asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+    tile = (int64_t)sm.next[sw];  // written before this tile's second barrier, rewritten after the next one's first
   }
   if (!ok) atomicOr(A.status, kStatusTimeout);
   if (A.pending) {  // the previous step's counts, straight into the totals
@@ -1568,9 +1555,7 @@ __global__ void __launch_bounds__(kThreads) k_select_approx(TopkArgs A) {
 // approximate top-s: every key >= theta when at most `limit` reach it, else
 // the exact top-`limit`.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
-  griddep_wait();
-  const int k = blockIdx.x;
+__device__ __forceinline__ void select_dense_worker(const TopkArgs& A, const int k) {
   WorkerSel& S = A.sel[k];
   if (A.approx ? S.dense == 0 : !needs_dense(S, A.ksel, A.cap)) return;
   __shared__ uint32_t h[kHistBins];
@@ -1697,6 +1682,27 @@ __global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
     atomicAdd(&A.step_ctr->v[kFallbacks], 1ull);
     atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(nsel - zeros));
     if (A.approx) atomicAdd(&A.step_ctr->v[kPairs], (unsigned long long)nsel);
+  }
+}
+
+// One block per worker. When it is the step's last launch (A.finalize), the
+// last block out also adds the step's counters to the totals (k_finalize's
+// work, one launch fewer).
+__global__ void __launch_bounds__(1024) k_select_dense(TopkArgs A) {
+  griddep_wait();
+  select_dense_worker(A, blockIdx.x);
+  if (!A.finalize) return;
+  __shared__ uint32_t s_last;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(&A.sel[0].done[3], 1u) == gridDim.x - 1 ? 1u : 0u;
+  }
+  __syncthreads();
+  if (s_last && threadIdx.x == 0) {
+    __threadfence();
+    A.sel[0].done[3] = 0;
+    finalize_counters(A.step_ctr, A.total_ctr, A.pairs_add);
   }
 }
 
@@ -1906,15 +1912,6 @@ bool use_bulk(int tile) { return tile == bulk::kT; }
 
 // Whether the exact top-k's sample (blocks_per_worker x K blocks) fits on the
 // GPU at once, as its cooperative launch requires.
-bool sample_coop_fits(int blocks_per_worker, int K, int num_sms) {
-  int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_sample_coop, kThreads, 0) != cudaSuccess) {
-    cudaGetLastError();
-    return false;
-  }
-  return (int64_t)n * num_sms >= (int64_t)blocks_per_worker * K;
-}
-
 int accumulate_smem_bytes(int tile, int K) {
   return use_bulk(tile) ? bulk::smem_bytes(K) : tile * 12;
 }
@@ -1964,12 +1961,7 @@ cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
     const cudaError_t err = launch_pdl(k_sample_pending, dim3((n_s + kThreads - 1) / kThreads), dim3(kThreads), 0, s, A);
     if (err != cudaSuccess) return err;
   }
-  if (A.sample_coop && !A.approx) {
-    TopkArgs a = A;
-    void* args[] = {&a};
-    return cudaLaunchCooperativeKernel((const void*)k_sample_coop, dim3(A.sample_blocks, A.K),
-                                       dim3(kThreads), args, 0, s);
-  }
+  if (!A.approx) return launch_pdl(k_sample_cluster, dim3(scl::kCtas, A.K), dim3(scl::kThreadsC), 0, s, A);
   const cudaError_t err = launch_pdl(k_sample, dim3(A.sample_blocks, A.K), dim3(kThreads), 0, s, A);
   if (err != cudaSuccess || !A.approx) return err;
   return launch_pdl(k_sample_theta, dim3(A.theta_blocks, A.K), dim3(kThreads), kBucketCap * 4, s, A);

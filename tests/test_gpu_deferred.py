@@ -156,3 +156,22 @@ def test_bulk_pass_reports_non_finite_values():
     torch.cuda.synchronize()
     assert p.gpu.stats()["nonfinite"] == 2
     assert p.gpu.check() == 4  # GMC_ENONFINITE
+
+
+@pytest.mark.parametrize("K", [1, 2, 5])
+def test_claimed_tiles_and_odd_worker_counts(K):
+    """Several tiles per CTA beyond its fixed ones, so the bulk pass claims
+    the rest from its tile counter; the worker-parity warp groups each read
+    their own stages of the ring, in order, for every K (odd K gives the two
+    groups different item counts per tile, K = 1 leaves one group without
+    items)."""
+    d = 152 * 4096 * 9 + 1001  # about nine tiles per CTA
+    rng = np.random.default_rng(40 + K)
+    p = Pair(d, K, 0.9, 0.1, ratio=0.001, seed=9)
+    for t in range(3):
+        r = p.step(_grads(rng, K, d))
+        p.compare(r, state=False)
+    p.compare(r)
+    s = p.compare_stats()
+    assert s["fallbacks"] == 0
+    assert p.gpu.check() == 0

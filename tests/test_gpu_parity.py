@@ -158,7 +158,9 @@ def test_step_host_matches_step():
 @pytest.mark.parametrize("d,B,ratio", [(10_000, 64, 0.05), (5_003, 100, 0.1), (4096 * 3 + 5, 4096, 0.5),
                                         # enough tiles for the bulk-copy kernel: odd d (rows at
                                         # every alignment), blocks that straddle tiles, and B = tile
-                                        (700_001, 1000, 0.02), (4096 * 160 + 3, 4096, 0.05)])
+                                        (700_001, 1000, 0.02), (4096 * 160 + 3, 4096, 0.05),
+                                        # about five tiles per CTA: the later ones claimed
+                                        (4096 * 152 * 5 + 77, 4096, 0.02)])
 def test_rbgs_gmcplus(per_worker, d, B, ratio):
     import torch
     K = 4
