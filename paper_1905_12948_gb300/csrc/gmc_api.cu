@@ -564,14 +564,13 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         std::max<uint64_t>((uint64_t)h->regions * h->cap_region, h->limit), 0xfffffff0ull);
     const int64_t per = (h->cap + 8191) / 8192;
     h->grid_agg = h->regions > 1 ? h->regions : (int)std::max<int64_t>(1, 4 * (int64_t)h->num_sms / K);
-    // select passes: about 2048 expected candidates per block
-    const double expect = h->sample_chunks ? (double)d * h->sample_rank / (8.0 * kSampleChunks) : (double)h->ksel;
-    const int64_t want = std::max<int64_t>(1, (int64_t)(expect / 2048.0));
-    // on the bulk path a warp visits candidate parts one after another, each a
-    // dependent load of its count and then of its keys: spread them over at
-    // least four blocks per SM's worth of warps
+    // select: on the bulk path a warp walks the candidates of a run of at most
+    // 32 parts as one list; the grid is one wave of four blocks per SM (each
+    // holds kBucketCap keys of shared memory), for all the workers
+    const int64_t nparts = (int64_t)h->regions * kChunksPerTile;
     h->sel_blocks = h->regions > 1 ? (int)std::min<int64_t>(
-                                         h->regions, std::max<int64_t>(want, (4 * (int64_t)h->num_sms + K - 1) / K))
+                                         h->regions, std::max<int64_t>((nparts + 32 * kWarps - 1) / (32 * kWarps),
+                                                                       std::max<int64_t>(1, 4 * (int64_t)h->num_sms / K)))
                                    : (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
     if (compressor == GMC_TOPK) h->n_sample = (uint32_t)(h->sample_chunks ? 8 * kSampleChunks : d);
     h->sample_stride = std::max<uint32_t>(kSampleSlots, (h->n_sample + 3) & ~3u);

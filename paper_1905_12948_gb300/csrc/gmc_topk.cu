@@ -109,8 +109,13 @@ __device__ __forceinline__ int64_t sample_coord(const TopkArgs& A, uint64_t key,
     return (int64_t)(a + 8 * (uint64_t)below(draw(key, run), (hi - a) >> 3) + (i & 7));
   }
   if (!A.sample_chunks) return i;
+  // sample_chunks is kSampleChunks, a power of two: floor(ch * d / kSampleChunks)
+  // by a shift (a 64-bit division would cost more than the slot's loads)
+  static_assert((kSampleChunks & (kSampleChunks - 1)) == 0, "kSampleChunks must be a power of two");
+  constexpr int kChunkShift = __builtin_ctz(kSampleChunks);
+  static_assert((1 << kChunkShift) == kSampleChunks, "shift of kSampleChunks");
   const int64_t ch = i >> 3;
-  return ((ch * A.d / A.sample_chunks) & ~int64_t(7)) + (i & 7);
+  return (((ch * A.d) >> kChunkShift) & ~int64_t(7)) + (i & 7);
 }
 __device__ __forceinline__ uint64_t sample_key(const TopkArgs& A) {
   return A.approx ? stream_key(A.seed, A.t, 0) : 0ull;
@@ -142,6 +147,7 @@ __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
     float x[kMaxK];
 #pragma unroll
     for (int b = 0; b < kMaxK; ++b) x[b] = b < A.K ? __ldcg(A.e + (int64_t)b * A.ld + j) : 0.f;
+    const float wo = A.w[j];  // loaded with the residuals, used only where a worker sent
     float sum = 0.f;
 #pragma unroll
     for (int b = 0; b < kMaxK; ++b) {
@@ -150,10 +156,7 @@ __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
         m |= 1u << b;
       }
     }
-    if (m) {
-      const float wo = A.w[j];
-      dd = __fsub_rn(__fsub_rn(wo, __fmul_rn(A.a_prev, sum)), wo);
-    }
+    if (m) dd = __fsub_rn(__fsub_rn(wo, __fmul_rn(A.a_prev, sum)), wo);
   }
   if (A.approx) {
     if (!m) dd = A.dlt[j];
@@ -215,7 +218,8 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
       if (i < i_hi) {  // coordinate, senders and w_t - w_{t-1} from k_sample_pending
         const int64_t j = A.sample_pend[2 * A.sample_stride + i];
         const uint32_t m = A.sample_pend[i];
-        ev[q] = ((m >> k) & 1u) ? 0.f : ek[j];
+        const float e = ek[j];  // loaded whatever m holds: no load waits on another but j
+        ev[q] = ((m >> k) & 1u) ? 0.f : e;
         const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
         gv[q] = A.local_mom ? local_m(A, k, j, g) : (A.gscale ? __fmul_rn(A.gs, g) : g);
         dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
@@ -334,21 +338,25 @@ __global__ void __cluster_dims__(scl::kCtas, 1, 1) __launch_bounds__(scl::kThrea
   const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
   const int n_s = (int)A.n_sample;  // at most kSampleSlots
   const int i_lo = (int)crank * (kSlots * kThreadsC);
-  float ev[kSlots], gv[kSlots], dv[kSlots];
+  // every load of every slot is issued before any value is used (no load
+  // waits on another), then v is formed as if the previous step's
+  // aggregation were applied at j
+  float ev[kSlots], gv[kSlots], dv[kSlots], lv[kSlots];
+  uint32_t pm[kSlots], pd[kSlots];
 #pragma unroll
   for (int q = 0; q < kSlots; ++q) {
     const int i = i_lo + q * kThreadsC + threadIdx.x;
-    ev[q] = gv[q] = dv[q] = 0.f;
+    ev[q] = gv[q] = dv[q] = lv[q] = 0.f;
+    pm[q] = pd[q] = 0u;
     if (i < n_s) {
       const int64_t j = sample_coord(A, 0ull, i);
       ev[q] = ek[j];
-      const float g = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
-      gv[q] = A.local_mom ? local_m(A, k, j, g) : (A.gscale ? __fmul_rn(A.gs, g) : g);
+      gv[q] = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
       dv[q] = A.dlt[j];
-      if (A.pending) {  // as if the previous step's aggregation were applied at j
-        const uint32_t m = A.sample_pend[i];
-        if ((m >> k) & 1u) ev[q] = 0.f;
-        if (m) dv[q] = __uint_as_float(A.sample_pend[A.sample_stride + i]);
+      if (A.local_mom) lv[q] = A.lm[(int64_t)k * A.ld + j];
+      if (A.pending) {
+        pm[q] = A.sample_pend[i];
+        pd[q] = A.sample_pend[A.sample_stride + i];
       }
     }
   }
@@ -356,7 +364,11 @@ __global__ void __cluster_dims__(scl::kCtas, 1, 1) __launch_bounds__(scl::kThrea
 #pragma unroll
   for (int q = 0; q < kSlots; ++q) {
     const int i = i_lo + q * kThreadsC + threadIdx.x;
-    key[q] = i < n_s ? mag_key(accumulate(ev[q], gv[q], A.c, dv[q])) : 0xffffffffu;
+    const float g = A.local_mom ? __fadd_rn(__fmul_rn(A.beta, lv[q]), __fmul_rn(A.gs, gv[q]))
+                                : (A.gscale ? __fmul_rn(A.gs, gv[q]) : gv[q]);
+    const float e = ((pm[q] >> k) & 1u) ? 0.f : ev[q];
+    const float dl = pm[q] ? __uint_as_float(pd[q]) : dv[q];
+    key[q] = i < n_s ? mag_key(accumulate(e, g, A.c, dl)) : 0xffffffffu;
     warp_hist_add(hist, key[q] != 0xffffffffu ? (int)(key[q] >> 20) : -1);
   }
   // every CTA of the cluster runs and has zeroed its histograms before any remote add
@@ -1424,35 +1436,88 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
   const float* cv = A.cand_val + (int64_t)k * A.cap;
   const int nparts = candidate_parts(A);
-  for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
-    uint32_t lo, hi;
-    candidate_part(A, k, part, nparts, &lo, &hi);
-    for (uint32_t i0 = lo; i0 < hi; i0 += 4 * 32) {  // 128 candidates a round, one reservation
-      uint32_t key[4], m[4], n = 0;
+  // kQ * 32 candidates a round (slots slot[q]), their keys and indices loaded
+  // together, one bucket reservation per round
+  constexpr int kQ = 8;
+  auto collect = [&](const uint32_t (&slot)[kQ], const bool (&in)[kQ]) {
+    uint32_t key[kQ], idx[kQ], m[kQ], n = 0;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint32_t i = i0 + q * 32 + lane;
-        key[q] = i < hi ? mag_key(cv[i]) : 0u;
-      }
+    for (int q = 0; q < kQ; ++q) {
+      key[q] = in[q] ? mag_key(cv[slot[q]]) : 0u;
+      idx[q] = in[q] ? ci[slot[q]] : 0u;
+    }
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint32_t i = i0 + q * 32 + lane;
-        m[q] = __ballot_sync(0xffffffffu, i < hi && rel_bin(key[q], theta, A.sel_shift) == want);
-        n += __popc(m[q]);
-      }
-      if (n) {
-        uint32_t base = 0;
-        if (lane == 0) base = atomicAdd(&S.count_bucket, n);
-        base = __shfl_sync(0xffffffffu, base, 0);
+    for (int q = 0; q < kQ; ++q) {
+      m[q] = __ballot_sync(0xffffffffu, in[q] && rel_bin(key[q], theta, A.sel_shift) == want);
+      n += __popc(m[q]);
+    }
+    if (n) {
+      uint32_t base = 0;
+      if (lane == 0) base = atomicAdd(&S.count_bucket, n);
+      base = __shfl_sync(0xffffffffu, base, 0);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const uint32_t o = base + __popc(m[q] & lt);
-          if (((m[q] >> lane) & 1u) && o < (uint32_t)kBucketCap) {
-            bk[o] = key[q];
-            bk[kBucketCap + o] = ci[i0 + q * 32 + lane];
-          }
-          base += __popc(m[q]);
+      for (int q = 0; q < kQ; ++q) {
+        const uint32_t o = base + __popc(m[q] & lt);
+        if (((m[q] >> lane) & 1u) && o < (uint32_t)kBucketCap) {
+          bk[o] = key[q];
+          bk[kBucketCap + o] = idx[q];
         }
+        base += __popc(m[q]);
+      }
+    }
+  };
+  if (A.regions > 1) {
+    // bulk path: the warp takes a run of at most 32 consecutive parts, lane l
+    // reading the count of part p_lo + l, and walks their candidates as one
+    // list (each candidate's part by a binary search over the lanes' counts),
+    // so its loads do not wait for one part after another
+    const int nw = (int)gridDim.x * kWarps;
+    const int per = (nparts + nw - 1) / nw;  // at most 32 (sel_blocks)
+    const int p_lo = min(nparts, (int)(blockIdx.x * kWarps + (threadIdx.x >> 5)) * per);
+    const int p_hi = min(nparts, p_lo + per);
+    const uint32_t cnt = p_lo + lane < p_hi ? A.rcount[(int64_t)k * nparts + p_lo + lane] : 0u;
+    uint32_t incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const uint32_t total = __shfl_sync(0xffffffffu, incl, 31);
+    for (uint32_t i0 = 0; i0 < total; i0 += kQ * 32) {
+      uint32_t slot[kQ];
+      bool in[kQ];
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+        const uint32_t i = i0 + q * 32 + lane;
+        in[q] = i < total;
+        int lo = 0, hi = 32;  // the first lane whose inclusive count exceeds i (six halvings of 32)
+#pragma unroll
+        for (int it = 0; it < 6; ++it) {
+          const int mid = min((lo + hi) >> 1, 31);
+          const uint32_t v = __shfl_sync(0xffffffffu, incl, mid);
+          if (lo < hi) {
+            if (v <= i) lo = mid + 1; else hi = mid;
+          }
+        }
+        const int L = lo < 32 ? lo : 31;
+        const uint32_t before = __shfl_sync(0xffffffffu, incl - cnt, L);
+        slot[q] = in[q] ? (uint32_t)(p_lo + L) * A.cap_part + (i - before) : 0u;
+      }
+      collect(slot, in);
+    }
+  } else {
+    for (int part = blockIdx.x * kWarps + (threadIdx.x >> 5); part < nparts; part += gridDim.x * kWarps) {
+      uint32_t lo, hi;
+      candidate_part(A, k, part, nparts, &lo, &hi);
+      for (uint32_t i0 = lo; i0 < hi; i0 += kQ * 32) {
+        uint32_t slot[kQ];
+        bool in[kQ];
+#pragma unroll
+        for (int q = 0; q < kQ; ++q) {
+          slot[q] = i0 + q * 32 + lane;
+          in[q] = slot[q] < hi;
+        }
+        collect(slot, in);
       }
     }
   }
