@@ -1,20 +1,23 @@
 // Top-k path of one GMC step (Alg. 1 with the top-s compressor of Sec. 4).
 //
-//   sample      per worker, e_{t+1/2} at a stratified sample -> a threshold key
-//               theta below the k-th largest |v| with overwhelming probability
+//   sample      per worker, e_{t+1/2} at a stratified sample of 32,768
+//               coordinates -> a candidate threshold key theta below the k-th
+//               largest |v| with overwhelming probability (one thread-block
+//               cluster per worker)
 //   accumulate  ONE dense pass: v = (e + g) - c*(w_t - w_{t-1}) written over e;
-//               every v with key >= theta is appended to the worker's chunk of
-//               its tile, in index order
-//   select x3   the exact k-th largest key T among the candidates (radix digits
-//               of 11, 10 and 10 bits) and how many ties at T are kept
-//   ties        only when more candidates equal T than are kept: the largest
-//               index of a kept tie (ties go to the lower index)
+//               every v with key >= theta is appended to its worker's part of
+//               the candidate buffer (a tile's candidates in sub-chunks, in
+//               index order) and counted into a histogram relative to theta;
+//               the bulk version also applies the previous step's aggregation
+//   select      the bin of that histogram holding the k-th key, its candidates
+//               ranked in shared memory: the k-th largest key T and the ties at
+//               T that are kept (the lowest indices: the largest kept, t_idx)
 //   dense       for a worker whose filter missed (too few or too many
-//               candidates): exact select over dense v, chunks rewritten
-//   aggregate   per tile: keep the sent pairs in each chunk (in place: the
-//               chunks are C(e_{t+1/2,k})), e = +0 at sent coordinates, sum
-//               the workers' values in ascending worker order from +0,
-//               w -= (eta/K) * sum on the union, store w_{t+1} - w_t
+//               candidates): exact radix select over dense v, sub-chunks rewritten
+//   aggregate   a candidate is sent iff selected(key, j, T, t_idx): e = +0 where
+//               sent, the sent values summed in ascending worker order from +0,
+//               w -= (eta/K) * sum on the union, w_{t+1} - w_t kept -- in the
+//               next step's bulk pass, or at once (k_mark, k_owner_sum)
 //
 // Keys are the fp32 bit patterns with the sign cleared (monotone in |v|); the
 // selected set is the first k elements under (key descending, index ascending).
@@ -1975,8 +1978,7 @@ bool use_bulk(int tile) { return tile == bulk::kT; }
 
 }  // namespace
 
-// Whether the exact top-k's sample (blocks_per_worker x K blocks) fits on the
-// GPU at once, as its cooperative launch requires.
+// Dynamic shared memory of the accumulate pass for tiles of `tile` and K workers.
 int accumulate_smem_bytes(int tile, int K) {
   return use_bulk(tile) ? bulk::smem_bytes(K) : tile * 12;
 }
