@@ -6,6 +6,9 @@ A step is one pass of the whole hot path (accumulator, compression, residual,
 aggregate and update) for the K simulated workers of the workload over one
 batch of synthetic gradients already resident in HBM. ``value`` is
 K*d*steps*ranks / (max over ranks of the device time of the timed steps).
+``workloads`` holds the same timing for the other configurations the metric is
+quoted on (d >= 11 M, K >= 8: resnet18, and resnet50 with shared and per-worker
+RBGS blocks), each measured in the same invocation.
 ``e2e`` is the same metric through the host-memory entry point (host->device
 copy of the step's gradients and device->host read of the step's counters
 inside the timed region). ``roofline`` reports the dominant kernel's
@@ -43,6 +46,7 @@ import workloads  # noqa: E402
 METRIC = "GMC step throughput (worker-params/sec) and achieved HBM GB/s vs 8 TB/s, 1 GB300"
 UNIT = "worker-params/s"
 DEFAULT_WORKLOAD = "vgg16"
+DEFAULT_EXTRA = "resnet18,resnet50,resnet50_pw"
 FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129e6
 
@@ -309,15 +313,15 @@ def config_of(wl, args):
             "parallelism": f"replicas x{args.gpus}"}
 
 
-def run_gmc(args, wl, world, rank, local):
+def measure(args, wl, world, rank, local, breakdown=True):
+    """Time `args.steps` steps of one workload on this rank's GPU, with its
+    gradients already in HBM: the device time of the steps (max over ranks),
+    the dominant kernel's CUDA-event time, the clocks during the timed region
+    and, with `breakdown`, the per-kernel split from untimed steps after it.
+    Returns (the handle, w0, the result dict)."""
     import torch
     from paper_1905_12948_gb300 import GMC
-    from paper_1905_12948_gb300 import build as gbuild
-    if rank == 0:
-        gbuild.build()
-    barrier(world)
     dev = torch.device("cuda", local)
-    torch.cuda.set_device(dev)
     gpu = GMC(wl.d, wl.K, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
               block=wl.block, lam=wl.lam if wl.compressor == "rbgs" else None, seed=0,
               per_worker=wl.per_worker, variant=wl.variant, device=dev)
@@ -354,11 +358,11 @@ def run_gmc(args, wl, world, rank, local):
     gpu.profile(False)
     # the per-kernel breakdown and launch count, from untimed steps with every
     # launch bracketed (those events lengthen a step slightly)
-    n_bd = min(args.steps, 10)
+    n_bd = min(args.steps, 10) if breakdown else 2
     gpu.profile(True)
     for i in range(n_bd):
         gpu.step(batches[(args.warmup + args.steps + i) % n_batches])
-    breakdown = gpu.profile_read()
+    bd = gpu.profile_read()
     gpu.profile(False)
     status = gpu.check()
     totals = gpu.stats()
@@ -370,13 +374,41 @@ def run_gmc(args, wl, world, rank, local):
     avg_s = p["ms"] / p["launches"] / 1e3
     achieved = per_launch_bytes / avg_s / 1e9
     peak, peak_kind = measured_hbm_peak()
-    traffic = recorded_traffic(dom, wl.name)
-    step_ms = ms / args.steps
+    step_ms = ms_max / args.steps
     kernels = {k: {"ms_per_step": round(v["ms"] / n_bd, 4),
-                   "share": round(v["ms"] / max(sum(x["ms"] for x in breakdown.values()), 1e-12), 4)}
-               for k, v in breakdown.items()}
+                   "share": round(v["ms"] / max(sum(x["ms"] for x in bd.values()), 1e-12), 4)}
+               for k, v in bd.items()}
     del batches
     torch.cuda.synchronize()
+    launches_per_step = sum(v["launches"] for v in bd.values()) / n_bd
+    res = {
+        "value": value, "ms_per_step": step_ms,
+        "hbm_gbs_step": step_bytes(wl) / (step_ms / 1e3) / 1e9,
+        "frac_of_8tbs": step_bytes(wl) / (step_ms / 1e3) / 8e12,
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": recorded_traffic(dom, wl.name),
+                     "algorithmic_bytes_per_launch": per_launch_bytes,
+                     "avg_launch_ms": avg_s * 1e3},
+        "clocks": clk, "kernels": kernels, "status": status,
+        "gpu_launches": int(round(launches_per_step * args.steps)),
+        "select_fallbacks": totals["fallbacks"], "steps_run": totals["steps"],
+    }
+    return gpu, w0, res
+
+
+def run_gmc(args, wl, world, rank, local):
+    import torch
+    from paper_1905_12948_gb300 import build as gbuild
+    if rank == 0:
+        gbuild.build()
+    barrier(world)
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    gpu, w0, res = measure(args, wl, world, rank, local)
+    bf16 = wl.grad_dtype == "bf16"
+    gb = (2.0 if bf16 else 4.0) * wl.K * wl.d
 
     e2e = None
     if not args.no_e2e:
@@ -402,27 +434,41 @@ def run_gmc(args, wl, world, rank, local):
                "ms_per_step": e_ms / args.steps}
         del host
     gpu.close()
+    del gpu, w0
+    torch.cuda.empty_cache()
+
+    # the other configurations the metric is quoted on (d >= 11 M, K >= 8), each
+    # timed the same way in this invocation
+    others = {}
+    extra = args.extra if args.extra is not None else (DEFAULT_EXTRA if wl.name == DEFAULT_WORKLOAD else "")
+    for name in ([] if args.no_extra else [n for n in extra.split(",") if n and n != wl.name]):
+        owl = workloads.workload(name)
+        g2, _, r2 = measure(args, owl, world, rank, local, breakdown=False)
+        g2.close()
+        del g2
+        torch.cuda.empty_cache()
+        others[name] = {"config": config_of(owl, args)["workload"], **{
+            k: r2[k] for k in ("ms_per_step", "value", "hbm_gbs_step", "frac_of_8tbs", "roofline",
+                               "clocks", "status", "gpu_launches")}}
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_sample(wl, budget_s=args.cpu_budget)
         cpu.pop("seconds", None)
 
-    launches_per_step = sum(v["launches"] for v in breakdown.values()) / n_bd
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True,
+        "metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": config_of(wl, args),
-        "hbm_gbs_step": step_bytes(wl) / (step_ms / 1e3) / 1e9,
-        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
-                     "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": traffic, "algorithmic_bytes_per_launch": per_launch_bytes,
-                     "avg_launch_ms": avg_s * 1e3},
-        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
-        "gpu_launches": int(round(launches_per_step * args.steps)),
-        "kernels": kernels, "status": status,
-        "select_fallbacks": totals["fallbacks"], "steps_run": totals["steps"],
+        "hbm_gbs_step": res["hbm_gbs_step"], "frac_of_8tbs": res["frac_of_8tbs"],
+        "roofline": res["roofline"],
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": res["clocks"],
+        "gpu_launches": res["gpu_launches"] + sum(o["gpu_launches"] for o in others.values()),
+        "gpu_launches_headline": res["gpu_launches"],
+        "kernels": res["kernels"], "status": res["status"],
+        "select_fallbacks": res["select_fallbacks"], "steps_run": res["steps_run"],
+        "workloads": others,
     }
     return line if rank == 0 else None
 
@@ -435,6 +481,10 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["gmc", "reference"], default="gmc")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
                     help="one of " + ", ".join(w.name for w in workloads.WORKLOADS))
+    ap.add_argument("--extra", default=None,
+                    help="comma-separated workloads also timed in the same run (key `workloads`); "
+                         f"default {DEFAULT_EXTRA} with the default workload, none otherwise")
+    ap.add_argument("--no-extra", action="store_true", help="time the one workload only")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle CPU time")

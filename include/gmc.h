@@ -56,6 +56,7 @@ typedef struct gmc_ctx* gmc_t;
 #define GMC_ESTATE      5  /* call out of order (e.g. gmc_step before gmc_set_params) */
 #define GMC_EINTERNAL   6  /* an internal consistency check failed on the device */
 #define GMC_ETOOBIG     7  /* size above the fixed scratch of gmc_topk_noalloc */
+#define GMC_ETIMEOUT    8  /* a bounded wait in a step's kernel gave up: work was skipped */
 
 /* Compressors C(.). */
 #define GMC_TOPK 0 /* exact top-k by magnitude, ties to the lower index (Sec. 4 top-s) */
@@ -135,7 +136,10 @@ typedef struct gmc_ctx* gmc_t;
 int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta,
                int32_t compressor, double ratio, int64_t block);
 
-/* gmc_destroy -- synchronise the device and free everything the handle owns. */
+/* gmc_destroy -- synchronise the device and free everything the handle owns: the
+ * state Alg. 1 (Sec. 3.1) carries between steps (w_t, w_t - w_{t-1}, the K
+ * residuals e_{t,k}) and the workspace. NULL is ignored. Returns nothing; after
+ * it, h must not be used. */
 void gmc_destroy(gmc_t h);
 
 /* gmc_set_lambda -- GMC+ detach coefficient lambda in [0,1] (Alg. 2); 0 is GMC.
@@ -224,12 +228,18 @@ int gmc_step_bf16(gmc_t h, const uint16_t* grads_bf16_dev, void* stream);
 int gmc_step_host_bf16(gmc_t h, const uint16_t* grads_bf16_host, uint64_t* step_stats_host,
                        void* stream);
 
-/* gmc_get_params -- copy w_t (d floats) into w_dev_out (applying a pending
- * aggregation first, see gmc_step). */
+/* gmc_get_params -- copy the server's parameters w_t of Alg. 1 (Sec. 3.1; the
+ * w_{t+1} = w_t - (eta/K) sum_k C_k line of the last step applied), d floats, into
+ * w_dev_out (device, caller-owned, borrowed until the stream has passed the
+ * call), applying a pending aggregation first (see gmc_step). GMC_EINVAL for a
+ * NULL pointer, GMC_ESTATE before gmc_set_params. */
 int gmc_get_params(gmc_t h, float* w_dev_out, void* stream);
 
-/* gmc_get_residual -- copy e_{t,k} (d floats) into e_dev_out (applying a
- * pending aggregation first). */
+/* gmc_get_residual -- copy worker k's residual e_{t,k} = e_{t-1/2,k} - C(e_{t-1/2,k})
+ * of Alg. 1 (Sec. 3.1; +0 exactly where the worker sent), d floats, into
+ * e_dev_out (device, caller-owned, borrowed until the stream has passed the
+ * call), applying a pending aggregation first. GMC_EINVAL for k outside [0, K)
+ * or a NULL pointer, GMC_ESTATE before gmc_set_params. */
 int gmc_get_residual(gmc_t h, int32_t k, float* e_dev_out, void* stream);
 
 /* gmc_get_selected -- synchronising. The last step's C(e_{t-1/2,k}) of worker k
@@ -281,8 +291,16 @@ int gmc_save_state(gmc_t h, void* host_out, int64_t capacity);
  * gmc_get_selected returns GMC_ESTATE until that step. */
 int gmc_load_state(gmc_t h, const void* host_in, int64_t bytes);
 
-/* gmc_check -- synchronising. GMC_OK, or the first data-dependent error recorded
- * since gmc_set_params (GMC_ENONFINITE, GMC_EINTERNAL), or GMC_ECUDA. */
+/* gmc_check -- synchronising. Reports what the device recorded since gmc_set_params
+ * (or gmc_load_state), most severe first: GMC_ECUDA (a CUDA error, e.g. a failed
+ * kernel), GMC_EINTERNAL (an internal consistency check failed), GMC_ETIMEOUT (a
+ * bounded wait of a bulk pass gave up, about two seconds without progress, and the
+ * pass skipped the rest of that CTA's tiles: w and the residuals are not Alg. 1's
+ * and the handle must be reset with gmc_set_params or gmc_load_state), or
+ * GMC_ENONFINITE (a NaN or Inf accumulator value, Sec. 3.1's step otherwise
+ * completed). GMC_OK when none. The status is not cleared by reading it.
+ * The recorded state is Alg. 1's (Sec. 3.1): the step runs to completion or
+ * says which condition it met; the paper itself defines no error behaviour. */
 int gmc_check(gmc_t h);
 
 /* gmc_profile_enable -- when on, each kernel launch of gmc_step is bracketed by
@@ -306,6 +324,31 @@ int gmc_profile_read(gmc_t h, int32_t kernel, double* total_ms, int64_t* launche
 const char* gmc_kernel_name(int32_t kernel);
 
 /*
+ * Failure injection for tests. The paper has no counterpart: these exist so
+ * that the library's failure paths can be exercised without faulting a GPU.
+ *
+ * gmc_test_fail_alloc -- process-wide. With fail_at >= 0, the fail_at-th device
+ * allocation the library makes from now on (0 = the next one, by any handle)
+ * fails as cudaMalloc does when memory runs out, once; fail_at < 0 disarms it.
+ * Returns the number of device allocations all handles hold at the call, so a
+ * test can check that a failed gmc_create or gmc_set_variant leaks nothing.
+ */
+int64_t gmc_test_fail_alloc(int64_t fail_at);
+
+/*
+ * gmc_test_withhold_copy -- the next gmc_step of h (only that one) runs its bulk
+ * pass with the copy of one item, worker k's slice of tile `tile` (4096
+ * components from tile*4096), never issued, and with every wait of that pass
+ * bounded by wait_limit_ns (1 .. 2e9) instead of about two seconds. The waits on
+ * that item give up, the CTA skips its remaining tiles after the copies it did
+ * issue have landed, and gmc_check then reports GMC_ETIMEOUT. GMC_EINVAL when
+ * the handle's step has no bulk pass (exact or approximate top-k needs
+ * d >= 4096 * 2 * SMs and K <= 16; RBGS d >= 4096 * SMs), or for a tile, worker or
+ * limit out of range.
+ */
+int gmc_test_withhold_copy(gmc_t h, int64_t tile, int32_t k, uint64_t wait_limit_ns);
+
+/*
  * gmc_topk_noalloc -- the top-k compressor of one vector without allocating.
  * The paper has no counterpart: this is a library convenience for callers
  * that cannot call cudaMalloc, e.g. code whose device memory is all owned by
@@ -320,8 +363,12 @@ const char* gmc_kernel_name(int32_t kernel);
  * library's device memory, which every GPU that loads the library holds until
  * the process exits. All calls share that array, so calls that overlap on the
  * GPU (on different streams, or from different threads) race; serialise
- * them. The first call on each device looks up the array's device address;
- * make that first call before any stream capture. Stream-ordered, asynchronous.
+ * them. The first call on each device (and the first after the device's
+ * context was replaced, e.g. by cudaDeviceReset) looks up the array's device
+ * address and the SM count; make that first call before any stream capture.
+ * A NaN in x ranks above every finite value and Inf (its magnitude bit pattern
+ * is larger) and is not reported as an error. Stream-ordered, asynchronous;
+ * GMC_ECUDA if a launch fails (only that launch's error is reported).
  */
 int gmc_topk_noalloc(const float* x_dev, int64_t n, int64_t k, uint32_t* idx_dev, float* val_dev,
                      void* stream);

@@ -3,6 +3,7 @@
 // caller-given stream. Only host code lives here; the kernels are in
 // gmc_topk.cu and gmc_rbgs.cu.
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -92,6 +93,11 @@ struct gmc_ctx {
   uint32_t* tile_ctr = nullptr;  // tiles claimed by the persistent passes
   Counters* total_ctr = nullptr;
   unsigned* status = nullptr;
+  // test hook (gmc_test_withhold_copy): the next step's bulk pass withholds
+  // the copy of item (hold_tile, hold_k) and bounds its waits by hold_wait_ns
+  int64_t hold_tile = -1;
+  int hold_k = 0;
+  uint64_t hold_wait_ns = 0;
   float* gstage = nullptr;
   std::vector<void*> allocations;
   // profiling
@@ -121,22 +127,35 @@ class DeviceGuard {
   int prev_ = 0, dev_ = 0;
 };
 
+// Test hook (gmc_test_fail_alloc): the device allocation that finds the
+// countdown at 0 fails as cudaMalloc does when memory runs out; -1 = off.
+std::atomic<int64_t> g_fail_countdown{-1};
+std::atomic<int64_t> g_live_allocations{0};  // device allocations held by all handles
+
+bool injected_alloc_failure() {
+  int64_t c = g_fail_countdown.load();
+  while (c >= 0 && !g_fail_countdown.compare_exchange_weak(c, c - 1)) {
+  }
+  return c == 0;
+}
+
 template <typename T>
 cudaError_t dalloc(gmc_ctx* h, T** p, size_t count) {
   void* q = nullptr;
+  *p = nullptr;
   const size_t bytes = std::max<size_t>(count, 1) * sizeof(T);
+  if (injected_alloc_failure()) return cudaErrorMemoryAllocation;
   cudaError_t err = cudaMalloc(&q, bytes);
-  if (err != cudaSuccess) {
-    *p = nullptr;
-    return err;
-  }
+  if (err != cudaSuccess) return err;
   h->allocations.push_back(q);
+  g_live_allocations.fetch_add(1);
   *p = static_cast<T*>(q);
   return cudaMemset(q, 0, bytes);
 }
 
 void free_all(gmc_ctx* h) {
   for (void* p : h->allocations) cudaFree(p);
+  g_live_allocations.fetch_sub((int64_t)h->allocations.size());
   h->allocations.clear();
   if (h->ev_step) cudaEventDestroy(h->ev_step);
   if (h->ev_flush) cudaEventDestroy(h->ev_flush);
@@ -281,6 +300,8 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.chunk_prev = h->chunk[prev];
   A.step_ctr = h->step_ctr;
   A.tile_ctr = h->tile_ctr;
+  A.wait_ns = kWaitLimitNs;
+  A.hold_tile = -1;
   A.status = h->status;
   return A;
 }
@@ -318,6 +339,8 @@ RbgsArgs rbgs_args(gmc_ctx* h, const float* grads) {
   A.has_prev = h->t > 0;
   A.step_ctr = h->step_ctr;
   A.tile_ctr = h->tile_ctr;
+  A.wait_ns = kWaitLimitNs;
+  A.hold_tile = -1;
   A.status = h->status;
   return A;
 }
@@ -360,6 +383,12 @@ int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, 
     A.grads16 = grads16;
     A.bf16 = bf16 ? 1 : 0;
     A.g_direct = direct ? 1 : 0;
+    if (h->hold_tile >= 0) {  // test hook, one step
+      A.hold_tile = h->hold_tile;
+      A.hold_k = h->hold_k;
+      A.wait_ns = h->hold_wait_ns;
+      h->hold_tile = -1;
+    }
     A.pending = h->agg_pending ? 1 : 0;
     A.a_prev = h->a_pending;
     const bool defer = h->tile == kBulkTile && !eager && !h->detach_out && !A.server_mom && !A.mfm;
@@ -398,6 +427,12 @@ int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, 
     A.grads16 = grads16;
     A.bf16 = bf16 ? 1 : 0;
     A.g_direct = direct ? 1 : 0;
+    if (h->hold_tile >= 0) {  // test hook, one step
+      A.hold_tile = h->hold_tile;
+      A.hold_k = h->hold_k;
+      A.wait_ns = h->hold_wait_ns;
+      h->hold_tile = -1;
+    }
     // restored state: w_t - w_{t-1} may be non-zero in any block (zero outside
     // the last union, where dlt holds it): flag every block as the last union's
     if (h->restored && h->t > 0) GMC_TRY(cudaMemsetAsync(A.uflag_prev, 1, (size_t)h->nb, s));
@@ -458,6 +493,7 @@ const char* gmc_strerror(int status) {
     case GMC_ESTATE: return "call out of order";
     case GMC_EINTERNAL: return "internal consistency check failed";
     case GMC_ETOOBIG: return "size exceeds the fixed scratch of gmc_topk_noalloc (n <= 2^26)";
+    case GMC_ETIMEOUT: return "a bounded wait in a step's kernel gave up: the step skipped work and its state is invalid";
     default: return "unknown status";
   }
 }
@@ -1065,8 +1101,24 @@ int gmc_check(gmc_t h) {
   err = cudaMemcpy(&st, h->status, sizeof(unsigned), cudaMemcpyDeviceToHost);
   if (err != cudaSuccess) return GMC_ECUDA;
   if (st & kStatusInternal) return GMC_EINTERNAL;
+  if (st & kStatusTimeout) return GMC_ETIMEOUT;
   if (st & kStatusNonfinite) return GMC_ENONFINITE;
   return GMC_OK;
+}
+
+int gmc_test_withhold_copy(gmc_t h, int64_t tile, int32_t k, uint64_t wait_limit_ns) {
+  if (!h || k < 0 || k >= h->K || wait_limit_ns == 0 || wait_limit_ns > kWaitLimitNs) return GMC_EINVAL;
+  const bool bulk = h->compressor == GMC_RBGS ? h->rbgs_bulk : h->tile == kBulkTile;
+  if (!bulk || tile < 0 || tile >= h->n_tiles) return GMC_EINVAL;
+  h->hold_tile = tile;
+  h->hold_k = k;
+  h->hold_wait_ns = wait_limit_ns;
+  return GMC_OK;
+}
+
+int64_t gmc_test_fail_alloc(int64_t fail_at) {
+  g_fail_countdown.store(fail_at < 0 ? -1 : fail_at);
+  return g_live_allocations.load();
 }
 
 int gmc_profile_enable(gmc_t h, int32_t on) {

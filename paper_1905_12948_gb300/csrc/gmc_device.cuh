@@ -58,7 +58,7 @@ __device__ __forceinline__ void finalize_counters(Counters* step, Counters* tota
 // Device status bits (gmc_check).
 constexpr unsigned kStatusNonfinite = 1u;
 constexpr unsigned kStatusInternal = 2u;
-constexpr unsigned kStatusTimeout = 4u;     // a bounded wait gave up (see wait_bounded)
+constexpr unsigned kStatusTimeout = 4u;     // a bounded wait gave up (see wait_bounded): tiles were skipped
 constexpr int kChunksPerTile = 8;           // candidate sub-chunks per tile: one per warp
 constexpr uint32_t kNone = 0xffffffffu;     // no coordinate
 
@@ -246,13 +246,16 @@ __device__ __forceinline__ uint64_t global_ns() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
-// Wait for the phase with the given parity to complete, giving up after about
-// two seconds (returns false): a wait never hangs the GPU.
-__device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity) {
+// Bound of every mbarrier wait of the bulk passes (a test may shorten it for
+// one step), and of the wait for a CTA's own copies in flight before it exits.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+// Wait for the phase with the given parity to complete, giving up after
+// limit_ns (returns false): a wait never hangs the GPU.
+__device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   while (!mbar_try_wait(bar, parity)) {
-    if (global_ns() - t0 > 2000000000ull) return false;
+    if (global_ns() - t0 > limit_ns) return false;
   }
   return true;
 }

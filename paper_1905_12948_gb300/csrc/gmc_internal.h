@@ -99,6 +99,9 @@ struct TopkArgs {
   Counters* step_ctr;
   unsigned* status;
   uint32_t* tile_ctr;        // tiles claimed by k_accumulate_bulk (zeroed by the sample kernel)
+  uint64_t wait_ns;          // bound of the bulk pass's mbarrier waits (kWaitLimitNs)
+  int64_t hold_tile;         // test hook: the bulk pass issues no copy for item (hold_tile, hold_k),
+  int hold_k;                // so that the waits on it give up; hold_tile = -1: none
   int finalize;              // k_select_dense ends the step: adds step_ctr (+ pairs_add pairs) to the totals
   unsigned long long pairs_add;
 };
@@ -139,6 +142,9 @@ struct RbgsArgs {
   int bulk;                  // k_rbgs_bulk (bulk copies through shared memory), else k_rbgs_step
   int g_direct;              // grads is mapped host memory: read it with loads, not bulk copies
   uint32_t* tile_ctr;        // tiles claimed by k_rbgs_bulk (zeroed by k_rbgs_pick)
+  uint64_t wait_ns;          // bound of the bulk pass's mbarrier waits (kWaitLimitNs)
+  int64_t hold_tile;         // test hook, as in TopkArgs: no copy for item (hold_tile, hold_k)
+  int hold_k;
   Counters* step_ctr;
   unsigned* status;
 };

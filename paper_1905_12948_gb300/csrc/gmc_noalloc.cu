@@ -177,25 +177,87 @@ __global__ void __launch_bounds__(kNaThreads) k_na_write(const float* __restrict
   }
 }
 
+// Set-up of one device: the scratch array's device address and the SM count,
+// valid for the CUDA context they were taken in.
+struct DeviceSetup {
+  unsigned long long ctx_id = 0;  // 0: not set up
+  uint32_t* scratch = nullptr;
+  int sms = 1;
+};
 std::mutex g_setup_mutex;
-uint32_t* g_scratch_ptr[kNaMaxDevices] = {};
+DeviceSetup g_setup[kNaMaxDevices];
 
-// Device address of the scratch array on the current device, looked up once
-// per device (host code cannot use the array's name as a device address).
-cudaError_t scratch_address(uint32_t** out) {
+using CtxGetCurrentFn = int (*)(void** ctx);
+using CtxGetIdFn = int (*)(void* ctx, unsigned long long* id);
+
+// Id of the current thread's CUDA context on the current device (the
+// runtime's primary context, made current if it was not), through the driver
+// entry points the runtime exposes. 0 on failure.
+unsigned long long current_context_id(int dev) {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  if (!get_current || !get_id) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !f)
+      return 0;
+    get_current = reinterpret_cast<CtxGetCurrentFn>(f);
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !f)
+      return 0;
+    get_id = reinterpret_cast<CtxGetIdFn>(f);
+  }
+  void* ctx = nullptr;
+  if (get_current(&ctx) != 0) return 0;
+  if (!ctx) {  // the runtime has not made its context current on this thread yet
+    if (cudaSetDevice(dev) != cudaSuccess || get_current(&ctx) != 0 || !ctx) return 0;
+  }
+  unsigned long long id = 0;
+  return get_id(ctx, &id) == 0 ? id : 0;
+}
+
+// The scratch array's device address and the SM count of the current device.
+// Host code cannot use the array's name as a device address: the address is
+// looked up with cudaGetSymbolAddress once per device, with that device
+// current, and again only if the device's context was replaced since (e.g.
+// after cudaDeviceReset), so that a stale address is never passed on.
+cudaError_t device_setup(DeviceSetup* out) {
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
   if (dev < 0 || dev >= kNaMaxDevices) return cudaErrorInvalidDevice;
+  const unsigned long long ctx = current_context_id(dev);
+  if (ctx == 0) return cudaErrorInitializationError;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_ptr[dev]) {
+  DeviceSetup& st = g_setup[dev];
+  if (st.ctx_id != ctx) {
     void* p = nullptr;
     err = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (err != cudaSuccess) return err;
-    g_scratch_ptr[dev] = static_cast<uint32_t*>(p);
+    int sms = 0;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    st.scratch = static_cast<uint32_t*>(p);
+    st.sms = sms > 0 ? sms : 1;
+    st.ctx_id = ctx;
   }
-  *out = g_scratch_ptr[dev];
+  *out = st;
   return cudaSuccess;
+}
+
+// One plain launch; returns that launch's own error (it neither reads nor
+// clears an error left by earlier, unrelated work).
+template <typename... P, typename... Args>
+cudaError_t launch(void (*kernel)(P...), unsigned grid, unsigned block, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cfg.attrs = nullptr;
+  cfg.numAttrs = 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 }  // namespace
@@ -206,27 +268,25 @@ extern "C" int gmc_topk_noalloc(const float* x_dev, int64_t n, int64_t k, uint32
   using namespace gmc;
   if (!x_dev || !idx_dev || !val_dev || n < 1 || k < 1 || k > n) return GMC_EINVAL;
   if (n > kNoallocMaxN) return GMC_ETOOBIG;
-  uint32_t* scratch = nullptr;
-  cudaError_t err = scratch_address(&scratch);
-  if (err != cudaSuccess) return GMC_ECUDA;
+  DeviceSetup dv;
+  if (device_setup(&dv) != cudaSuccess) return GMC_ECUDA;
+  uint32_t* scratch = dv.scratch;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // the histogram and the pass state must start at zero; the tables are
   // fully rewritten by every call
-  err = cudaMemsetAsync(scratch, 0, (size_t)(kOffState + 16) * sizeof(uint32_t), s);
-  if (err != cudaSuccess) return GMC_ECUDA;
-  int sms = 1;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (cudaMemsetAsync(scratch, 0, (size_t)(kOffState + 16) * sizeof(uint32_t), s) != cudaSuccess)
+    return GMC_ECUDA;
   const int64_t want = (n + kNaThreads * 16 - 1) / (kNaThreads * 16);
-  const int grid = (int)(want < 2 * (int64_t)sms ? want : 2 * (int64_t)sms);
+  const unsigned grid = (unsigned)(want < 2 * (int64_t)dv.sms ? want : 2 * (int64_t)dv.sms);
   const int64_t n_tiles = (n + kNaTile - 1) / kNaTile;
   const uint32_t kk = (uint32_t)k;
-  k_na_pass<0><<<grid, kNaThreads, 0, s>>>(x_dev, n, kk, scratch);
-  k_na_pass<1><<<grid, kNaThreads, 0, s>>>(x_dev, n, kk, scratch);
-  k_na_pass<2><<<grid, kNaThreads, 0, s>>>(x_dev, n, kk, scratch);
-  k_na_count<<<(unsigned)n_tiles, kNaThreads, 0, s>>>(x_dev, n, scratch);
-  k_na_scan<<<1, 1024, 0, s>>>(n_tiles, kk, scratch);
-  k_na_write<<<(unsigned)n_tiles, kNaThreads, 0, s>>>(x_dev, n, kk, scratch, idx_dev, val_dev);
-  return cudaGetLastError() == cudaSuccess ? GMC_OK : GMC_ECUDA;
+  cudaError_t err = launch(k_na_pass<0>, grid, kNaThreads, s, x_dev, n, kk, scratch);
+  if (err == cudaSuccess) err = launch(k_na_pass<1>, grid, kNaThreads, s, x_dev, n, kk, scratch);
+  if (err == cudaSuccess) err = launch(k_na_pass<2>, grid, kNaThreads, s, x_dev, n, kk, scratch);
+  if (err == cudaSuccess) err = launch(k_na_count, (unsigned)n_tiles, kNaThreads, s, x_dev, n, scratch);
+  if (err == cudaSuccess) err = launch(k_na_scan, 1u, 1024u, s, n_tiles, kk, scratch);
+  if (err == cudaSuccess)
+    err = launch(k_na_write, (unsigned)n_tiles, kNaThreads, s, x_dev, n, kk,
+                 static_cast<const uint32_t*>(scratch), idx_dev, val_dev);
+  return err == cudaSuccess ? GMC_OK : GMC_ECUDA;
 }

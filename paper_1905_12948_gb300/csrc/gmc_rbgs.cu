@@ -315,6 +315,7 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
     const char* g_lo = kBf16 ? reinterpret_cast<const char*>(A.grads16) : reinterpret_cast<const char*>(A.grads);
     const char* g_hi = g_lo + (int64_t)A.K * A.d * es;
     uint32_t item = 0, claim = 0;
+    uint32_t held = ~0u;  // test hook: the item not copied
     bool ok = true;
     for (uint32_t n = 0; ok; ++n) {
       const int64_t tile = tile_claim<kFixed, kQ>(sm.tq, n, A.tile_ctr, claim, A.n_tiles);
@@ -323,9 +324,13 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
       const int64_t nvalid = A.d - j0 < kT ? A.d - j0 : kT;
       for (int k = 0; k < A.K; ++k, ++item) {
         const uint32_t s = item % kStages, r = item / kStages;
-        if (r > 0 && !wait_bounded(&sm.empty[s], (r - 1) & 1)) {
+        if (r > 0 && !wait_bounded(&sm.empty[s], (r - 1) & 1, A.wait_ns)) {
           ok = false;
           break;
+        }
+        if (tile == A.hold_tile && k == A.hold_k) {  // the stage's phase never completes
+          held = item;
+          continue;
         }
         const float* esrc = A.e + (int64_t)k * A.ld + j0;
         const uintptr_t ga = reinterpret_cast<uintptr_t>(g_lo + ((int64_t)k * A.d + j0) * es);
@@ -339,12 +344,16 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
         if (gbulk) bulk_load(sm.g[s], gsrc, gbytes, &sm.full[s]);
       }
     }
-    if (!ok) {
-      atomicOr(A.status, kStatusTimeout);
-      // let the copies already issued land before the CTA's shared memory goes away
-      const uint32_t first = item > (uint32_t)kStages ? item - kStages : 0u;
-      for (uint32_t i = first; i < item; ++i) wait_bounded(&sm.full[i % kStages], (i / kStages) & 1);
-    }
+    if (!ok) atomicOr(A.status, kStatusTimeout);
+    // Every copy issued lands before the CTA's shared memory goes away, even
+    // when the consumers gave up on their waits: the last kStages items (the
+    // earlier ones were read, as their stages' empty barriers showed) read
+    // valid global memory and complete without any other warp's help; no
+    // later phase is armed on their stages.
+    const uint32_t first = item > (uint32_t)kStages ? item - kStages : 0u;
+    for (uint32_t i = first; i < item; ++i)
+      if (i != held && !wait_bounded(&sm.full[i % kStages], (i / kStages) & 1, kWaitLimitNs))
+        atomicOr(A.status, kStatusTimeout | kStatusInternal);
     return;
   }
 
@@ -390,7 +399,7 @@ __global__ void __launch_bounds__(rbulk::kThreadsAll, 1) k_rbgs_bulk(RbgsArgs A)
     }
     for (int k = 0; k < A.K; ++k, ++item) {
       const uint32_t s = item % kStages, r = item / kStages;
-      if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
+      if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1, A.wait_ns))) {  // warp-uniform
         ok = false;
         break;
       }

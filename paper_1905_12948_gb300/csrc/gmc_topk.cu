@@ -1029,6 +1029,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     const char* g_lo = kBf16 ? reinterpret_cast<const char*>(A.grads16) : reinterpret_cast<const char*>(A.grads);
     const char* g_hi = g_lo + (int64_t)A.K * A.d * es;
     uint32_t issued[2] = {0u, 0u};  // items issued to each worker-parity group
+    uint32_t held = ~0u;            // test hook: (group << 31) | count of the item not copied
     uint32_t claim = 0;
     bool ok = true;
     for (uint32_t n = 0; ok; ++n) {
@@ -1039,9 +1040,14 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
       for (int k = 0; k < A.K; ++k) {
         const uint32_t grp = (uint32_t)k & 1u, c = issued[grp];
         const uint32_t s = grp * kGroupStages + c % kGroupStages, r = c / kGroupStages;
-        if (r > 0 && !wait_bounded(&sm.empty[s], (r - 1) & 1)) {
+        if (r > 0 && !wait_bounded(&sm.empty[s], (r - 1) & 1, A.wait_ns)) {
           ok = false;
           break;
+        }
+        issued[grp] = c + 1;
+        if (tile == A.hold_tile && k == A.hold_k) {  // the stage's phase never completes
+          held = (grp << 31) | c;
+          continue;
         }
         const float* esrc = A.e + (int64_t)k * A.ld + j0;
         const uintptr_t ga = reinterpret_cast<uintptr_t>(g_lo + ((int64_t)k * A.d + j0) * es);
@@ -1053,17 +1059,21 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         mbar_arrive_expect_tx(&sm.full[s], kT * 4 + (gbulk ? gbytes : 0));
         bulk_load(sm.e[s], esrc, kT * 4, &sm.full[s]);
         if (gbulk) bulk_load(sm.g[s], gsrc, gbytes, &sm.full[s]);
-        issued[grp] = c + 1;
       }
     }
-    if (!ok) {
-      atomicOr(A.status, kStatusTimeout);
-      // let the copies already issued land before the CTA's shared memory goes away
-      for (uint32_t grp = 0; grp < 2; ++grp) {
-        const uint32_t c1 = issued[grp], c0 = c1 > (uint32_t)kGroupStages ? c1 - kGroupStages : 0u;
-        for (uint32_t c = c0; c < c1; ++c)
-          wait_bounded(&sm.full[grp * kGroupStages + c % kGroupStages], (c / kGroupStages) & 1);
-      }
+    if (!ok) atomicOr(A.status, kStatusTimeout);
+    // Every copy issued lands before the CTA's shared memory goes away, even
+    // when the consumers gave up on their waits: the last kGroupStages items
+    // of each group (the earlier ones were read, as their stages' empty
+    // barriers showed) read valid global memory and complete without any
+    // other warp's help. No later phase is armed on their stages, so each
+    // parity wait is for exactly that copy.
+    for (uint32_t grp = 0; grp < 2; ++grp) {
+      const uint32_t c1 = issued[grp], c0 = c1 > (uint32_t)kGroupStages ? c1 - kGroupStages : 0u;
+      for (uint32_t c = c0; c < c1; ++c)
+        if (((grp << 31) | c) != held &&
+            !wait_bounded(&sm.full[grp * kGroupStages + c % kGroupStages], (c / kGroupStages) & 1, kWaitLimitNs))
+          atomicOr(A.status, kStatusTimeout | kStatusInternal);
     }
     return;
   }
@@ -1164,7 +1174,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         for (int u = 0; u < kSub / 128; ++u)
           mv[u] = __ldcs(reinterpret_cast<const float4*>(A.lm + (int64_t)k * A.ld + s0 + u * 128 + lane * 4));
       }
-      if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1))) {  // warp-uniform
+      if (!__all_sync(0xffffffffu, wait_bounded(&sm.full[s], r & 1, A.wait_ns))) {  // warp-uniform
         ok = false;
         break;
       }

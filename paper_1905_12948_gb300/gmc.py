@@ -14,7 +14,8 @@ from typing import Optional, Tuple
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libgmc.so")
 
-GMC_OK, GMC_EINVAL, GMC_ENOMEM, GMC_ECUDA, GMC_ENONFINITE, GMC_ESTATE, GMC_EINTERNAL, GMC_ETOOBIG = range(8)
+(GMC_OK, GMC_EINVAL, GMC_ENOMEM, GMC_ECUDA, GMC_ENONFINITE, GMC_ESTATE, GMC_EINTERNAL, GMC_ETOOBIG,
+ GMC_ETIMEOUT) = range(9)
 GMC_TOPK, GMC_RBGS, GMC_TOPK_APPROX = 0, 1, 2
 # Alg. 1, Alg. 3, Alg. 4, and the local-momentum baseline without / with masking
 VARIANTS = {"gmc": 0, "server_momentum": 1, "lr_in_residual": 2, "local_momentum": 3,
@@ -65,6 +66,8 @@ _SIGNATURES = {
     "gmc_kernel_name": (ctypes.c_char_p, [_i32]),
     "gmc_strerror": (ctypes.c_char_p, [ctypes.c_int]),
     "gmc_topk_noalloc": (ctypes.c_int, [_c_p, _i64, _i64, _c_p, _c_p, _c_p]),
+    "gmc_test_fail_alloc": (_i64, [_i64]),
+    "gmc_test_withhold_copy": (ctypes.c_int, [_c_p, _i64, _i32, _u64]),
 }
 
 _lib = None

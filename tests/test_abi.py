@@ -57,3 +57,15 @@ def test_invalid_arguments_rejected_without_gpu(lib):
         assert h.value is None
     assert lib.gmc_step(None, None, None) == 1
     assert lib.gmc_set_params(None, None, None) == 1
+
+
+def test_failure_hooks_without_gpu(lib):
+    """The allocation hook round-trips without a device (no handle holds
+    memory), the timeout has its own status and message, and the copy hook
+    refuses a NULL handle."""
+    assert lib.gmc_test_fail_alloc(3) == 0
+    assert lib.gmc_test_fail_alloc(-1) == 0
+    assert lib.gmc_strerror(8).startswith(b"a bounded wait")
+    assert lib.gmc_strerror(9) == b"unknown status"
+    assert lib.gmc_test_withhold_copy(None, 0, 0, 1000) == 1
+    assert lib.gmc_check(None) == 1

@@ -71,6 +71,10 @@ WORKLOADS = [
              eta=0.05, steps=50, n_segments=62, laplace_frac=0.1, laplace_scale=5.0),
     Workload("resnet50", d=25_557_032, K=32, compressor="rbgs", ratio=0.01, beta=0.9,
              eta=0.1, steps=20, block=4096, lam=0.5, n_segments=161, noniid=0.02),
+    # the resnet50 configuration with an independent block choice per worker and step
+    Workload("resnet50_pw", d=25_557_032, K=32, compressor="rbgs", ratio=0.01, beta=0.9,
+             eta=0.1, steps=20, block=4096, lam=0.5, per_worker=True, n_segments=161,
+             noniid=0.02),
     Workload("vgg16", d=138_357_544, K=8, compressor="topk", ratio=0.001, beta=0.9,
              eta=0.01, steps=10, n_segments=32, big_segment=102_760_448,
              scale_lo=1e-4, scale_hi=1e-1, noniid=0.02),
