@@ -10,6 +10,7 @@
   existing handle as it was.
 """
 import ctypes
+import gc
 
 import numpy as np
 import pytest
@@ -102,6 +103,7 @@ def test_create_allocation_failures_leak_nothing(d, K, compressor):
     import torch
     lib = _lib()
     torch.cuda.init()
+    gc.collect()  # handles of earlier tests still waiting for the collector
     live0 = lib.gmc_test_fail_alloc(-1)
     failures = 0
     for i in range(64):
@@ -128,6 +130,7 @@ def test_set_variant_allocation_failure_leaves_the_handle_usable():
     lib = _lib()
     d, K = 200_003, 3
     rng = np.random.default_rng(4)
+    gc.collect()
     p = Pair(d, K, 0.9, 0.1, compressor="topk", ratio=0.01)
     live = lib.gmc_test_fail_alloc(-1)
     for variant in (1, 3):  # Alg. 3's server momentum, the local momentum: one allocation each
