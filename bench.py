@@ -228,59 +228,107 @@ def barrier(world: int):
 # ---------------------------------------------------------------------------
 # CPU oracle on a bounded sample of the workload
 # ---------------------------------------------------------------------------
-def oracle_sample(wl, budget_s: float = 12.0, max_steps: int = 50, workers: int = 1,
-                  d_sample: int = 1 << 24, first_step: int = 0):
+def _oracle_kind(wl) -> str:
+    """The C++ oracle states Alg. 1 / Alg. 2 with top-s or RBGS; the appendix
+    variants and the approximate top-s are in the numpy oracle only."""
+    return "cpp" if wl.variant == "gmc" and wl.compressor in ("topk", "rbgs") else "numpy"
+
+
+def oracle_sample(wl, budget_s: float = 12.0, max_steps: int = 50, workers: int = 0,
+                  d_sample: int = 1 << 24, first_step: int = 0, threads: int = 0):
     """Time the oracle (as it stands) on a bounded sample of the workload:
-    `workers` of its workers over the leading `d_sample` parameters (same
-    per-parameter gradient scales, same compression ratio), running steps
-    until `budget_s` of CPU time is spent. Input generation is not timed."""
+    `workers` of its workers (0: all K) over the leading `d_sample` parameters
+    (same per-parameter gradient scales, same compression ratio), running
+    steps until `budget_s` of wall time is spent. The C++ oracle runs one
+    thread per worker, at most `threads` (0: the host's cores); the numpy
+    oracle one thread. Two gradient batches are drawn beforehand and
+    alternate; drawing them is not timed."""
     import oracle
-    K_s = min(workers, wl.K)
+    from oracle import cref
+    K_s = wl.K if workers <= 0 else min(workers, wl.K)
     d_s = min(wl.d, d_sample)
+    kind = _oracle_kind(wl)
     gen = workloads.NumpyGradients(wl, seed=0, d=d_s, K=K_s)
-    o = oracle.GMC(d_s, K_s, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
-                   block=wl.block, lam=wl.lam, seed=0, per_worker=wl.per_worker,
-                   variant=wl.variant)
+    batches = [gen(first_step + i) for i in range(2)]
+    args = dict(compressor=wl.compressor, ratio=wl.ratio, block=wl.block, lam=wl.lam, seed=0,
+                per_worker=wl.per_worker, variant=wl.variant)
+    if kind == "cpp":
+        o = cref.CGMC(d_s, K_s, wl.beta, wl.eta, threads=threads or (os.cpu_count() or 1), **args)
+        cores = o.threads
+    else:
+        o = oracle.GMC(d_s, K_s, wl.beta, wl.eta, **args)
+        cores = 1
     o.set_params(workloads.init_params(wl.d)[:d_s])
     spent, steps = 0.0, 0
     while steps < max_steps and (spent < budget_s or steps == 0):
-        g = gen(first_step + steps)
         t0 = time.perf_counter()
-        o.step(g)
+        o.step(batches[steps % 2])
         spent += time.perf_counter() - t0
         steps += 1
-        del g
-    return {"value": K_s * d_s * steps / spent, "unit": UNIT, "cores": 1, "kind": "oracle",
+    what = ((f"C++ oracle, {cores} threads, one worker each" if cores > 1 else "C++ oracle, one thread")
+            if kind == "cpp"
+            else "numpy oracle, one thread")
+    return {"value": K_s * d_s * steps / spent, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "host_cores": os.cpu_count(),
             "sample": f"{steps} oracle step(s) of {K_s} of the {wl.K} workers over the first "
-                      f"{d_s:,} of d={wl.d:,} parameters (numpy, one thread), {spent:.1f} s",
-            "seconds": spent, "d_sample": d_s}
+                      f"{d_s:,} of d={wl.d:,} parameters ({what}), {spent:.1f} s",
+            "seconds": spent, "d_sample": d_s, "steps": steps}
+
+
+def cpu_baseline(wl, budget_s: float):
+    """The oracle on the host's cores, with its one-thread figure beside it."""
+    many = oracle_sample(wl, budget_s=budget_s)
+    many.pop("seconds", None)
+    if many["cores"] > 1:
+        one = oracle_sample(wl, budget_s=budget_s / 2, threads=1)
+        many["one_thread"] = {"value": one["value"], "sample": one["sample"]}
+    return many
 
 
 # ---------------------------------------------------------------------------
 # arms
 # ---------------------------------------------------------------------------
 def run_reference(args, wl, world, rank):
+    """The reference arm: the oracle (the paper has no code to install), as it
+    stands, on the host's cores; each step one oracle step of all K workers
+    over the first `--ref-params` parameters of the workload."""
     if rank != 0:
         return None
-    d_s = args.ref_params
+    import oracle
+    from oracle import cref
+    d_s = min(wl.d, args.ref_params)
+    kind = _oracle_kind(wl)
+    gen = workloads.NumpyGradients(wl, seed=0, d=d_s, K=wl.K)
+    batches = [gen(i) for i in range(2)]
+    kw = dict(compressor=wl.compressor, ratio=wl.ratio, block=wl.block, lam=wl.lam, seed=0,
+              per_worker=wl.per_worker, variant=wl.variant)
+    if kind == "cpp":
+        o = cref.CGMC(d_s, wl.K, wl.beta, wl.eta, threads=os.cpu_count() or 1, **kw)
+        cores = o.threads
+    else:
+        o = oracle.GMC(d_s, wl.K, wl.beta, wl.eta, **kw)
+        cores = 1
+    o.set_params(workloads.init_params(wl.d)[:d_s])
     for i in range(args.warmup):
-        oracle_sample(wl, budget_s=0.0, max_steps=1, d_sample=d_s, first_step=i)
+        o.step(batches[i % 2])
     t0 = time.perf_counter()
-    samples = [oracle_sample(wl, budget_s=0.0, max_steps=1, d_sample=d_s, first_step=i)
-               for i in range(args.steps)]
-    elapsed = time.perf_counter() - t0
-    spent = sum(s["seconds"] for s in samples)
-    d_s = samples[0]["d_sample"]
-    value = d_s * args.steps / spent
+    for i in range(args.steps):
+        o.step(batches[(args.warmup + i) % 2])
+    spent = time.perf_counter() - t0
+    value = wl.K * d_s * args.steps / spent
+    what = ((f"C++ oracle, {cores} threads, one worker each" if cores > 1 else "C++ oracle, one thread")
+            if kind == "cpp"
+            else "numpy oracle, one thread")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * spent / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic", "config": config_of(wl, args),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"each step: one oracle step of 1 of the {wl.K} workers over "
-                                   f"the first {d_s:,} of d={wl.d:,} parameters (numpy, one "
-                                   f"thread); wall {elapsed:.1f} s including input generation"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "host_cores": os.cpu_count(),
+                         "sample": f"each step: one oracle step of all {wl.K} workers over the "
+                                   f"first {d_s:,} of d={wl.d:,} parameters ({what}); two "
+                                   f"gradient batches alternate"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     return line
@@ -453,8 +501,7 @@ def run_gmc(args, wl, world, rank, local):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        cpu = oracle_sample(wl, budget_s=args.cpu_budget)
-        cpu.pop("seconds", None)
+        cpu = cpu_baseline(wl, args.cpu_budget)
 
     line = {
         "metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -488,7 +535,7 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle CPU time")
-    ap.add_argument("--ref-params", type=int, default=1 << 23,
+    ap.add_argument("--ref-params", type=int, default=1 << 22,
                     help="reference arm: parameters of the oracle sample per step")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "gmc":

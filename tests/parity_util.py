@@ -4,6 +4,7 @@ bitwise and within the stated fp32 bar (1e-6 relative, 1e-7 absolute)."""
 import numpy as np
 
 import oracle
+from oracle import cref
 
 RTOL, ATOL = 1e-6, 1e-7
 
@@ -25,7 +26,7 @@ class Pair:
 
     def __init__(self, d, K, beta, eta, compressor="topk", ratio=0.01, block=4096, lam=None,
                  seed=0, per_worker=False, select_mode="sampled", w0=None, device="cuda",
-                 variant="gmc"):
+                 variant="gmc", ref="numpy"):
         import torch
         from paper_1905_12948_gb300 import GMC
         self.torch = torch
@@ -35,8 +36,11 @@ class Pair:
         self.gpu = GMC(d, K, beta, eta, compressor=compressor, ratio=ratio, block=block, lam=lam,
                        seed=seed, per_worker=per_worker, select_mode=select_mode, device=self.dev,
                        variant=variant)
-        self.ref = oracle.GMC(d, K, beta, eta, compressor=compressor, ratio=ratio, block=block,
-                              lam=lam_or, seed=seed, per_worker=per_worker, variant=variant)
+        # the numpy oracle, or the C++ one (Alg. 1 / Alg. 2 with top-s or RBGS;
+        # fast enough for whole trajectories at full size)
+        make = oracle.GMC if ref == "numpy" else cref.CGMC
+        self.ref = make(d, K, beta, eta, compressor=compressor, ratio=ratio, block=block,
+                        lam=lam_or, seed=seed, per_worker=per_worker, variant=variant)
         if w0 is None:
             w0 = (np.random.default_rng(seed + 17).standard_normal(d) * 0.01).astype(np.float32)
         self.gpu.set_params(torch.from_numpy(w0).to(self.dev))

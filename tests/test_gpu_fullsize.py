@@ -1,11 +1,19 @@
 """Parity at the full sizes of the benchmark workloads, in the configuration
 bench.py times: same handle parameters, same tile geometry and launch grids
-(they depend only on d, K and the compressor), the first steps of each
-trajectory. Inputs are drawn on the device and copied to the host for the
-oracle; every selected index and value is compared after each step, and w and
-every worker's residual after each step, or -- `deferred`, as the benchmark
-runs, each step applying the previous one's aggregation in its bulk pass --
-after the last one only."""
+(they depend only on d, K and the compressor). Inputs are drawn on the device
+and copied to the host for the oracle.
+
+The method's own workloads run their whole configured trajectories against
+the C++ oracle (threaded over workers): resnet18 for 50 steps, resnet50 for 20
+steps with shared and with per-worker RBGS blocks, vgg16 for 10 steps. Every
+selected index and value is compared after every step. w and every worker's
+residual are compared every `every` steps and after the last one; on the
+deferred path (as the benchmark runs, each step applying the previous one's
+aggregation in its bulk pass) reading them applies the pending aggregation
+first, so the step after a read runs without one. The appendix variants, the
+approximate top-s and the local-momentum baseline run their first steps
+against the numpy oracle.
+"""
 import numpy as np
 import pytest
 
@@ -15,18 +23,21 @@ from parity_util import Pair
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("name,steps,per_worker,deferred", [
-    ("resnet18", 3, False, False),  # d = 11,173,962 (d % 4 = 2: misaligned rows), K = 16, top-k 0.1%
-    ("resnet18", 3, False, True),
-    ("resnet50", 2, False, False),  # d = 25,557,032, K = 32, RBGS B = 4096, shared blocks, GMC+
-    ("resnet50", 2, True, False),   # same, per-worker blocks
-    ("vgg16", 3, False, True),      # d = 138,357,544, K = 8, top-k 0.1%
-    ("vgg16_approx", 3, False, True),  # the same under the approximate top-s of Sec. 5.1
-    ("vgg16_alg3", 2, False, False),   # the same under the appendix's Alg. 3 (eager, dense server step)
-    ("vgg16_alg4", 2, False, True),    # and Alg. 4
-    ("vgg16_local", 2, False, True),   # and the local-momentum baseline
+@pytest.mark.parametrize("name,steps,per_worker,deferred,every,ref", [
+    # d = 11,173,962 (d % 4 = 2: misaligned rows), K = 16, top-k 0.1%
+    ("resnet18", 50, False, True, 10, "cpp"),
+    ("resnet18", 4, False, False, 1, "cpp"),
+    # d = 25,557,032, K = 32, RBGS B = 4096, GMC+ lambda = 0.5, shared / per-worker blocks
+    ("resnet50", 20, False, False, 5, "cpp"),
+    ("resnet50", 20, True, False, 5, "cpp"),
+    # d = 138,357,544, K = 8, top-k 0.1%
+    ("vgg16", 10, False, True, 5, "cpp"),
+    ("vgg16_approx", 3, False, True, 3, "numpy"),  # the approximate top-s of Sec. 5.1
+    ("vgg16_alg3", 2, False, False, 1, "numpy"),   # the appendix's Alg. 3 (eager, dense server step)
+    ("vgg16_alg4", 2, False, True, 2, "numpy"),    # and Alg. 4
+    ("vgg16_local", 2, False, True, 2, "numpy"),   # and the local-momentum baseline
 ])
-def test_fullsize_parity(name, steps, per_worker, deferred):
+def test_fullsize_parity(name, steps, per_worker, deferred, every, ref):
     import torch
     wl = workloads.workload(name)
     dev = torch.device("cuda")
@@ -34,7 +45,7 @@ def test_fullsize_parity(name, steps, per_worker, deferred):
     rbgs = wl.compressor == "rbgs"
     p = Pair(wl.d, wl.K, wl.beta, wl.eta, compressor=wl.compressor, ratio=wl.ratio,
              block=wl.block, lam=wl.lam if rbgs else None, seed=0, per_worker=per_worker,
-             w0=workloads.init_params(wl.d), device=dev, variant=wl.variant)
+             w0=workloads.init_params(wl.d), device=dev, variant=wl.variant, ref=ref)
     for t in range(steps):
         g_dev = gen(t)
         assert bool(torch.isfinite(g_dev).all()), "synthetic gradients must be finite"
@@ -42,12 +53,13 @@ def test_fullsize_parity(name, steps, per_worker, deferred):
         r = p.step(g, grads_dev=g_dev)
         torch.cuda.synchronize()
         del g_dev
-        p.compare(r, state=not deferred or t == steps - 1)
+        state = (t + 1) % every == 0 or t == steps - 1
+        p.compare(r, state=state)
         del g, r
     s = p.compare_stats()
     if not rbgs:
         assert s["fallbacks"] == 0, "the sampled filter should not miss on these inputs"
     assert p.gpu.check() == 0
     p.gpu.close()
-    del gen
+    del gen, p
     torch.cuda.empty_cache()

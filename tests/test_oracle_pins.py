@@ -816,3 +816,82 @@ def test_p9b_toy_global_beats_local_momentum():
         tail = {v: _toy_distances(v, 20, s, start)[-1000:].mean()
                 for v in (oracle.ALG1, oracle.LOCAL, oracle.LOCAL_MFM)}
         assert tail[oracle.ALG1] < tail[oracle.LOCAL] and tail[oracle.ALG1] < tail[oracle.LOCAL_MFM], (s, tail)
+
+
+# ---------------------------------------------------------------------------
+# The appendix's comparison of Alg. 4 with GMC under a decaying learning rate
+# ---------------------------------------------------------------------------
+
+def _cosine_etas(eta0, T):
+    """Sec. 5.1's cosine annealing without restarts, per step:
+    eta_t = eta0 * 0.5 * (1 + cos(t pi / (T + 1))), each rounded to fp32."""
+    return [float(np.float32(eta0 * 0.5 * (1.0 + math.cos(t * math.pi / (T + 1))))) for t in range(T)]
+
+
+def _top_s_64(x, s):
+    """Top-s of a float64 vector: largest |x|, ties to the lower index, ascending."""
+    order = np.lexsort((np.arange(x.size), -np.abs(x)))
+    return np.sort(order[:s])
+
+
+def _toy_grads(w, d):
+    """The two workers' gradients of Sec. 3.2's quadratic at w (optimum 0)."""
+    i = np.arange(d)
+    wgt = (d - i).astype(np.float64)
+    return np.stack([2 * wgt * (w - (i + 1)), 2 * wgt * (w + (i + 1))]).astype(np.float32)
+
+
+@pytest.mark.parametrize("variant", [oracle.ALG1, oracle.ALG4])
+@pytest.mark.parametrize("problem", ["gaussian", "toy_quadratic"])
+def test_appendix_rewriting_under_decaying_eta(variant, problem):
+    """The appendix ("Other Ways for Combining Momentum and Error Feedback")
+    writes both forms with one scaled accumulator, under a learning rate eta_t:
+        a_{t,k} = r_{t,k} + eta_t g_{t,k} - beta (w_t - w_{t-1}),
+        w_{t+1} = w_t - (1/K) sum_k C(a_{t,k}),
+        r_{t+1,k} = rho_{t+1} (a_{t,k} - C(a_{t,k})),
+    where r is eta_t e_t for GMC (the residual rescaled, rho_{t+1} =
+    eta_{t+1}/eta_t) and Alg. 4's own residual (rho = 1): Alg. 4's residual
+    enters the next step with the larger coefficient, since eta_t does not
+    increase. Checked in float64 on the fp32 oracle's own state at every step
+    of Sec. 5.1's cosine schedule: the oracle sends top-s of a (compressors
+    are scale-invariant, C(eta x) = eta C(x)), its update is -(1/K) sum C(a),
+    and the residual it carries is rho (a - C(a)) with rho as stated; the
+    factor changes by up to a few per cent a step here, far above rounding."""
+    rng = np.random.default_rng(61)
+    if problem == "gaussian":
+        d, K, ratio, eta0, T = 2000, 4, 0.01, 0.1, 40
+    else:
+        d, K, ratio, eta0, T = 20, 2, 0.1, 0.005, 60
+    beta = 0.9
+    s = oracle.topk_count(d, ratio)
+    o = GMC(d, K, beta=beta, eta=eta0, compressor=TOPK, ratio=ratio, variant=variant)
+    o.set_params((rng.standard_normal(d) if problem == "gaussian"
+                  else np.linspace(-1.0, 2.0, d)).astype(np.float32))
+    etas = _cosine_etas(eta0, T)
+    b32 = float(np.float32(beta))
+    carry = None  # a_{t-1} - C(a_{t-1}), float64
+    w_prev = o.w.astype(np.float64)
+    for t, eta_t in enumerate(etas):
+        o.set_eta(eta_t)
+        w_t, e_t = o.w.astype(np.float64), o.e.astype(np.float64)
+        r_t = eta_t * e_t if variant == oracle.ALG1 else e_t  # the scaled residual
+        if carry is not None:
+            rho = eta_t / etas[t - 1] if variant == oracle.ALG1 else 1.0
+            if variant == oracle.ALG1:
+                assert rho < 1.0 - 1e-3 or t < 3
+            # the oracle formed a_{t-1} in fp32 (three roundings, c = fl(beta/eta)):
+            # a budget on the size of its terms, as in P5
+            np.testing.assert_array_less(np.abs(r_t - rho * carry), 8 * U * rho * carry_mag + 1e-30)
+        g = (_grads(rng, 1, K, d)[0] if problem == "gaussian" else _toy_grads(w_t, d))
+        a = r_t + eta_t * g.astype(np.float64) - b32 * (w_t - w_prev)
+        r = o.step(g)
+        C = np.zeros_like(a)
+        for k in range(K):
+            np.testing.assert_array_equal(r.supports[k], _top_s_64(a[k], s))
+            C[k, r.supports[k]] = a[k, r.supports[k]]
+        step = o.w.astype(np.float64) - w_t
+        budget = 8 * U * (np.abs(o.w) + np.abs(w_t) + np.abs(a).sum(0) / K * (K + 3))
+        np.testing.assert_array_less(np.abs(step + C.sum(0) / K), budget + 1e-30)
+        carry = a - C
+        carry_mag = np.abs(r_t) + eta_t * np.abs(g.astype(np.float64)) + b32 * np.abs(w_t - w_prev)
+        w_prev = w_t
