@@ -573,7 +573,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
       h->cap = (uint32_t)d;
     } else {
       h->sample_chunks = kSampleChunks;
-      const double ns = 8.0 * kSampleChunks;
+      const double ns = (double)kSampleSlots;
       const double mean = ns * (double)ks / (double)d;
       const double r = std::min(ns, std::ceil(mean + 5.0 * std::sqrt(mean) + 8.0));
       h->sample_rank = (uint32_t)r;
@@ -608,7 +608,7 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
                                          h->regions, std::max<int64_t>((nparts + 32 * kWarps - 1) / (32 * kWarps),
                                                                        std::max<int64_t>(1, 4 * (int64_t)h->num_sms / K)))
                                    : (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
-    if (compressor == GMC_TOPK) h->n_sample = (uint32_t)(h->sample_chunks ? 8 * kSampleChunks : d);
+    if (compressor == GMC_TOPK) h->n_sample = (uint32_t)(h->sample_chunks ? kSampleSlots : d);
     h->sample_stride = std::max<uint32_t>(kSampleSlots, (h->n_sample + 3) & ~3u);
     h->sample_blocks = (int)std::max<int64_t>(1, ((int64_t)h->n_sample + 2047) / 2048);
     h->theta_blocks = (int)std::max<int64_t>(1, std::min<int64_t>(2 * h->num_sms / K + 1,

@@ -13,9 +13,11 @@ constexpr uint32_t kNoCandidate = 0xffffffffu; // threshold above every key
 constexpr int kThreads = 256;                // block size of the streaming kernels
 constexpr int kWarps = kThreads / 32;
 constexpr int kSampleThreads = 1024;
-constexpr int kSampleChunks = 4096;          // sampled 8-element chunks per worker
+constexpr int kSampleRun = 8;                // consecutive coordinates per sampled run (power of two)
 constexpr int kSampleAll = 32768;            // d at or below which every element is sampled
-constexpr int kSampleSlots = 8 * kSampleChunks;  // sampled positions (= kSampleAll)
+constexpr int kSampleSlots = 32768;          // sampled positions per worker (= kSampleAll)
+constexpr int kSampleChunks = kSampleSlots / kSampleRun;  // sampled runs per worker
+static_assert((kSampleRun & (kSampleRun - 1)) == 0 && kSampleRun <= 32, "kSampleRun: a power of two, at most a warp");
 constexpr int kHistBins = 2048;              // first radix digit: key bits 30..20
 constexpr int kRelBins = 2048;               // bins of the candidates' relative histogram
 constexpr int kBucketCap = 12288;            // candidates of one bin ranked in shared memory

@@ -117,8 +117,9 @@ __device__ __forceinline__ int64_t sample_coord(const TopkArgs& A, uint64_t key,
   static_assert((kSampleChunks & (kSampleChunks - 1)) == 0, "kSampleChunks must be a power of two");
   constexpr int kChunkShift = __builtin_ctz(kSampleChunks);
   static_assert((1 << kChunkShift) == kSampleChunks, "shift of kSampleChunks");
-  const int64_t ch = i >> 3;
-  return (((ch * A.d) >> kChunkShift) & ~int64_t(7)) + (i & 7);
+  constexpr int kRunShift = __builtin_ctz(kSampleRun);
+  const int64_t ch = i >> kRunShift;
+  return (((ch * A.d) >> kChunkShift) & ~int64_t(kSampleRun - 1)) + (i & (kSampleRun - 1));
 }
 __device__ __forceinline__ uint64_t sample_key(const TopkArgs& A) {
   return A.approx ? stream_key(A.seed, A.t, 0) : 0ull;
