@@ -91,6 +91,9 @@ struct gmc_ctx {
   float* slab = nullptr;
   Counters* step_ctr = nullptr;
   uint32_t* tile_ctr = nullptr;  // tiles claimed by the persistent passes
+  uint32_t* blk_cost = nullptr;  // the bulk top-k pass's tile order (tile_order): costs, order
+  uint32_t* blk_order = nullptr;
+  uint32_t n_blk = 0, blk_mul = 1;
   Counters* total_ctr = nullptr;
   unsigned* status = nullptr;
   // test hook (gmc_test_withhold_copy): the next step's bulk pass withholds
@@ -300,6 +303,11 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
   A.chunk_prev = h->chunk[prev];
   A.step_ctr = h->step_ctr;
   A.tile_ctr = h->tile_ctr;
+  A.blk_cost = h->blk_cost;
+  A.blk_order = h->blk_order;
+  A.n_blk = h->n_blk;
+  A.blk_mul = h->blk_mul;
+  A.use_order = 0;
   A.wait_ns = kWaitLimitNs;
   A.hold_tile = -1;
   A.status = h->status;
@@ -307,6 +315,24 @@ TopkArgs topk_args_at(gmc_ctx* h, const float* grads, int64_t t) {
 }
 
 TopkArgs topk_args(gmc_ctx* h, const float* grads) { return topk_args_at(h, grads, h->t); }
+
+// The stride of the bulk top-k pass's block order (tile_order): the first
+// integer from nb times the golden ratio's fractional part that is coprime to
+// nb, so that (b * stride) mod nb visits every block once.
+uint32_t golden_stride(int64_t nb) {
+  if (nb < 3) return 1;
+  int64_t m = (int64_t)std::llround(0.6180339887498949 * (double)nb);
+  for (;; ++m) {
+    int64_t a = m, b = nb;
+    while (b) {
+      const int64_t r = a % b;
+      a = b;
+      b = r;
+    }
+    if (a == 1) return (uint32_t)(m % nb);
+  }
+}
+
 
 RbgsArgs rbgs_args(gmc_ctx* h, const float* grads) {
   RbgsArgs A;
@@ -391,6 +417,8 @@ int enqueue_step(gmc_ctx* h, const void* grads_any, cudaStream_t s, bool eager, 
     }
     A.pending = h->agg_pending ? 1 : 0;
     A.a_prev = h->a_pending;
+    // the tile order is built by k_sample_pending, which runs on these steps
+    A.use_order = (h->blk_order && (A.pending || approx) && !A.dense_mode) ? 1 : 0;
     const bool defer = h->tile == kBulkTile && !eager && !h->detach_out && !A.server_mom && !A.mfm;
     const double kk = (double)h->K * (double)h->ksel;
     pairs_add = approx ? 0ull : (unsigned long long)h->K * h->ksel;  // approximate: counted on the device
@@ -587,6 +615,8 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     // plus slack, in whole 128-byte lines); otherwise one region
     const uint32_t cap0 = h->cap;
     if (h->tile == kBulkTile) {
+      h->n_blk = (uint32_t)(h->n_tiles / h->grid_acc);
+      h->blk_mul = golden_stride(h->n_blk);
       h->regions = h->grid_acc;
       const uint64_t share = (2ull * cap0 + h->regions * kChunksPerTile - 1) / (h->regions * kChunksPerTile);
       h->cap_part = (uint32_t)((share + 128 + 31) & ~31ull);
@@ -634,6 +664,9 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
         (err = dalloc(h, &h->rcount, (size_t)K * h->regions * kChunksPerTile)) != cudaSuccess ||
         (err = dalloc(h, &h->mask, (size_t)h->ld)) != cudaSuccess ||
         (err = dalloc(h, &h->sample_pend, (size_t)3 * h->sample_stride)) != cudaSuccess)
+      return fail(err);
+    if (h->n_blk >= 8 && ((err = dalloc(h, &h->blk_cost, (size_t)h->n_blk)) != cudaSuccess ||
+                          (err = dalloc(h, &h->blk_order, (size_t)h->n_blk)) != cudaSuccess))
       return fail(err);
     if ((err = cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking)) != cudaSuccess ||
         (err = cudaEventCreateWithFlags(&h->ev_step, cudaEventDisableTiming)) != cudaSuccess ||
@@ -773,6 +806,7 @@ int reset_state(gmc_ctx* h, cudaStream_t s) {
       GMC_TRY(cudaMemsetAsync(h->chunk[p], 0, (size_t)h->K * h->n_tiles * kChunksPerTile * sizeof(uint2), s));
     GMC_TRY(cudaMemsetAsync(h->sel, 0, (size_t)h->K * sizeof(WorkerSel), s));
     GMC_TRY(cudaMemsetAsync(h->mask, 0, (size_t)h->ld * sizeof(uint32_t), s));
+    if (h->blk_cost) GMC_TRY(cudaMemsetAsync(h->blk_cost, 0, (size_t)h->n_blk * sizeof(uint32_t), s));
   } else {
     for (int p = 0; p < 2; ++p) GMC_TRY(cudaMemsetAsync(h->uflag[p], 0, (size_t)h->nb, s));
   }

@@ -278,18 +278,44 @@ __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wa
 // tq[m % kQ] only after it has synchronised with the producer's start of tile
 // m + 1 - kFixed. kQ must exceed the tiles between the oldest slot a thread
 // may still read and the newest the producer may write.
+// The number of fixed tiles may also be chosen at run time (uniform over the
+// grid): tile_at_n / tile_claim_n.
+template <int kQ>
+__device__ __forceinline__ int64_t tile_at_n(const uint32_t* tq, uint32_t n, uint32_t fixed) {
+  return n < fixed ? (int64_t)blockIdx.x + (int64_t)n * gridDim.x : (int64_t)tq[n % kQ];
+}
+// The order in which a pass visits its tiles, in blocks of G = gridDim.x
+// consecutive tiles: the i-th tile claimed is order[i / G] * G + i mod G over
+// the nb = n_tiles / G whole blocks (the partial block at the end stays last;
+// order: a permutation of [0, nb), or NULL for index order; i >= n_tiles: past
+// the last, unchanged). Within a block consecutive tiles still go to
+// different CTAs at about the same time, so a layer's tiles spread over the
+// CTAs' candidate parts as in index order.
+__device__ __forceinline__ int64_t tile_order(int64_t i, int64_t n_tiles, const uint32_t* order) {
+  if (i >= n_tiles || !order) return i;
+  const uint32_t G = gridDim.x, nb = (uint32_t)(n_tiles / G);
+  if ((uint64_t)i >= (uint64_t)nb * G) return i;
+  const uint32_t b = (uint32_t)i / G, o = (uint32_t)i - b * G;
+  const uint32_t ob = __ldg(order + b);
+  return (int64_t)(ob < nb ? ob : b) * G + o;
+}
 template <int kFixed, int kQ>
 __device__ __forceinline__ int64_t tile_at(const uint32_t* tq, uint32_t n) {
-  return n < (uint32_t)kFixed ? (int64_t)blockIdx.x + (int64_t)n * gridDim.x : (int64_t)tq[n % kQ];
+  return tile_at_n<kQ>(tq, n, (uint32_t)kFixed);
 }
 // The producer's part at the start of its tile n: returns the tile.
+template <int kQ>
+__device__ __forceinline__ int64_t tile_claim_n(uint32_t* tq, uint32_t n, uint32_t fixed, uint32_t* ctr,
+                                                uint32_t& claim, int64_t n_tiles) {
+  if (n > 0) tq[(n - 1 + fixed) % kQ] = fixed * gridDim.x + claim;
+  const int64_t tile = tile_at_n<kQ>(tq, n, fixed);
+  if (tile < n_tiles) claim = atomicAdd(ctr, 1u);
+  return tile;
+}
 template <int kFixed, int kQ>
 __device__ __forceinline__ int64_t tile_claim(uint32_t* tq, uint32_t n, uint32_t* ctr, uint32_t& claim,
                                               int64_t n_tiles) {
-  if (n > 0) tq[(n - 1 + kFixed) % kQ] = (uint32_t)kFixed * gridDim.x + claim;
-  const int64_t tile = tile_at<kFixed, kQ>(tq, n);
-  if (tile < n_tiles) claim = atomicAdd(ctr, 1u);
-  return tile;
+  return tile_claim_n<kQ>(tq, n, (uint32_t)kFixed, ctr, claim, n_tiles);
 }
 
 // Order this thread's generic-proxy shared-memory accesses before later

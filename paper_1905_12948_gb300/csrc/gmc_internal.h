@@ -99,6 +99,15 @@ struct TopkArgs {
   Counters* step_ctr;
   unsigned* status;
   uint32_t* tile_ctr;        // tiles claimed by k_accumulate_bulk (zeroed by the sample kernel)
+  // k_accumulate_bulk's tile order (tile_order): blk_cost accumulates the
+  // candidates each block of gridDim.x tiles produced; k_sample_pending turns
+  // it into blk_order -- the golden-stride sequence of blocks (b * blk_mul)
+  // mod n_blk with the coldest few moved to the end -- and clears it.
+  uint32_t* blk_cost;        // n_tiles / grid blocks (bulk top-k only, else NULL)
+  uint32_t* blk_order;       // the same count
+  uint32_t n_blk;            // whole blocks of the bulk pass's grid of tiles: n_tiles / grid
+  uint32_t blk_mul;          // the golden stride, coprime to n_blk
+  int use_order;             // this step's pass follows blk_order (it was built this step)
   uint64_t wait_ns;          // bound of the bulk pass's mbarrier waits (kWaitLimitNs)
   int64_t hold_tile;         // test hook: the bulk pass issues no copy for item (hold_tile, hold_k),
   int hold_k;                // so that the waits on it give up; hold_tile = -1: none

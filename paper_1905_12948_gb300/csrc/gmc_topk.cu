@@ -133,6 +133,8 @@ __device__ __forceinline__ uint64_t sample_key(const TopkArgs& A) {
 // +0 (Alg. 1). The approximate top-s runs it every step: it also stores each
 // slot's coordinate, and the step's w_t - w_{t-1} there (from dlt when no
 // aggregation is pending), for k_sample to read in order.
+constexpr int kTailBlocks = 4;  // blocks of tiles the bulk pass ends with: the coldest (tile_order)
+
 __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
   griddep_wait();
   __shared__ uint32_t Tp[kMaxK], tip[kMaxK];
@@ -141,6 +143,61 @@ __global__ void __launch_bounds__(kThreads) k_sample_pending(TopkArgs A) {
     tip[kk] = A.sel[kk].t_idx;
   }
   __syncthreads();
+  if (A.use_order && blockIdx.x == gridDim.x - 1) {  // the launch's extra block
+    // The block order of this step's bulk pass (tile_order): the blocks in
+    // the golden-stride sequence (b * blk_mul) mod nb, which spreads every run
+    // of neighbouring blocks evenly over the pass, except the kTailBlocks
+    // blocks that produced the fewest candidates since the last order was
+    // made, which go last (the coldest at the very end): the pass then ends
+    // on light tiles. Deterministic: minima by (count, block), one scan.
+    __shared__ unsigned long long ws64[32];
+    __shared__ unsigned long long s_pick[kTailBlocks];
+    const uint32_t nb = A.n_blk, per = (nb + blockDim.x - 1) / blockDim.x;
+    const uint32_t lo = min(nb, threadIdx.x * per), hi = min(nb, lo + per);
+    for (int r = 0; r < kTailBlocks; ++r) {
+      unsigned long long m = ~0ull;
+      for (uint32_t b = lo; b < hi; ++b) {
+        const unsigned long long key = ((unsigned long long)A.blk_cost[b] << 32) | b;
+        bool taken = false;
+        for (int q = 0; q < r; ++q) taken |= s_pick[q] == key;
+        if (!taken && key < m) m = key;
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long y = __shfl_xor_sync(0xffffffffu, m, o);
+        m = y < m ? y : m;
+      }
+      if ((threadIdx.x & 31) == 0) ws64[threadIdx.x >> 5] = m;
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        unsigned long long mm = ~0ull;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) mm = ws64[w] < mm ? ws64[w] : mm;
+        s_pick[r] = mm;
+      }
+      __syncthreads();
+    }
+    uint32_t pick[kTailBlocks];
+#pragma unroll
+    for (int r = 0; r < kTailBlocks; ++r) pick[r] = (uint32_t)s_pick[r];
+    auto picked = [&](uint32_t b) {
+      bool t = false;
+#pragma unroll
+      for (int r = 0; r < kTailBlocks; ++r) t |= pick[r] == b;
+      return t;
+    };
+    // positions q of the sequence in this thread's chunk, less the picked blocks before
+    unsigned long long skip = 0, n_skip;
+    for (uint32_t q = lo; q < hi; ++q) skip += picked((uint32_t)(((unsigned long long)q * A.blk_mul) % nb));
+    uint32_t pos = lo - (uint32_t)(block_inclusive_scan<unsigned long long>(skip, ws64, &n_skip) - skip);
+    for (uint32_t q = lo; q < hi; ++q) {
+      const uint32_t b = (uint32_t)(((unsigned long long)q * A.blk_mul) % nb);
+      if (!picked(b)) A.blk_order[pos++] = b;
+    }
+    if (threadIdx.x < kTailBlocks) A.blk_order[nb - 1 - threadIdx.x] = pick[threadIdx.x];
+    __syncthreads();  // every cost read: this step's pass counts afresh
+    for (uint32_t b = lo; b < hi; ++b) A.blk_cost[b] = 0u;
+    return;
+  }
   const int n_s = (int)A.n_sample;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n_s) return;
@@ -836,14 +893,22 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 // step's sent pairs. Those are reached through two dependent loads -- the
 // sub-chunk table, then the pairs -- and the pending case reads w at the
 // pairs' coordinates: a chain of three memory latencies. The warp runs that
-// chain as a pipeline over its tiles: while it works on tile n it loads w for
-// tile n+1, the pairs of tile n+2 and the sub-chunk entries of tile n+3, so
-// no latency lies on its path. A sub-tile with more than 32 pairs takes the
-// direct path (stage_pending_warp / stage_delta_warp).
+// chain as a pipeline, so that no latency lies on its path. With few workers
+// (K <= 5, short tiles) the pipeline spans tiles: while the warp works on
+// tile n it loads w for tile n+1, the pairs of tile n+2 and the sub-chunk
+// entries of tile n+3. With more workers a tile lasts long enough for the
+// whole chain of tile n+1: its entries at the start of tile n, its pairs
+// after the warp's first item, w after its second. A sub-tile with more than
+// 32 pairs takes the direct path (stage_pending_warp / stage_delta_warp).
 //
 // A CTA's first tiles are fixed and every later one is claimed from a counter
-// (tile_at, tile_claim), so that CTAs whose streams run faster take more
-// tiles and all of them finish together.
+// (tile_at_n, tile_claim_n), so that CTAs whose streams run faster take more
+// tiles and all of them finish together. A claim is made a few tiles before
+// the CTA starts it (the pipeline must know its tiles ahead), so when the
+// counter runs out each CTA still holds those tiles; the SMs' streaming rates
+// differ by up to a fifth, and the CTAs' finishing times spread by that share
+// of the tiles they hold. The shallow pipeline lets a CTA claim two tiles
+// ahead instead of four, which halves that spread.
 // ---------------------------------------------------------------------------
 namespace bulk {
 constexpr int kT = kBulkTile;
@@ -878,16 +943,19 @@ struct Smem {
   // followed by the candidate staging lines: per consumer warp and worker, 32
   // indices then 32 values (staging_bytes)
 };
-// Tiles: a CTA's first five fixed, the rest claimed four tiles ahead of the
-// producer's start of the tile before it. Only the lead warp of a sub-tile
-// (it has worker 0's items) reads the queue; the earliest read of a slot is
-// its load of tile n + 3's sub-chunk entries during tile n, after it waited
-// on an item of tile n - 1, whose issue followed the producer's publishing of
-// slots up to n + 3. The producer runs at most kStages items (tiles, for
-// K <= 2) ahead of the slowest consumer.
-constexpr int kFixed = 5;
+// Tiles: a CTA's first F fixed, the rest claimed F - 1 tiles ahead of the
+// producer's start of the tile before it (tile_claim_n publishes the claim of
+// tile n - 1 into slot n - 1 + F when it starts tile n). Only the lead warp of
+// a sub-tile (it has worker 0's items) reads the queue; the earliest read of a
+// slot is that of tile n + D (D: the pipeline's depth, 3 or 1) during tile n,
+// after it waited on an item of tile n - 1, whose issue followed the
+// producer's publishing of slots up to n - 2 + F: so F = D + 2. The producer
+// runs at most kStages items (tiles, for K <= 2) ahead of the slowest consumer.
+constexpr int kFixedDeep = 5;     // K <= kDeepMaxK: depth 3
+constexpr int kFixedShallow = 3;  // more workers: depth 1
+constexpr int kDeepMaxK = 5;      // from K = 6 the lead warp has three items a tile or more
 constexpr int kQ = 16;
-static_assert(kQ > kStages + kFixed, "the producer may overwrite a claimed tile not yet read");
+static_assert(kQ > kStages + kFixedDeep, "the producer may overwrite a claimed tile not yet read");
 // Dynamic shared memory of the bulk pass for K workers.
 __host__ __device__ constexpr int smem_bytes(int K) {
   return (int)((sizeof(Smem) + 127) / 128 * 128) + kSubTiles * K * 64 * 4;
@@ -1008,6 +1076,10 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool deep = A.K <= kDeepMaxK;  // the lead warp's pipeline spans three tiles
+  const uint32_t F = deep ? kFixedDeep : kFixedShallow;
+  const uint32_t* order = A.use_order ? A.blk_order : nullptr;  // the tiles' order (tile_order)
+  const uint32_t G = gridDim.x, nbw = (uint32_t)(A.n_tiles / G);  // whole blocks of G tiles
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.full[s], 1);
@@ -1034,7 +1106,8 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     uint32_t claim = 0;
     bool ok = true;
     for (uint32_t n = 0; ok; ++n) {
-      const int64_t tile = tile_claim<kFixed, kQ>(sm.tq, n, A.tile_ctr, claim, A.n_tiles);
+      const int64_t tile =
+          tile_order(tile_claim_n<kQ>(sm.tq, n, F, A.tile_ctr, claim, A.n_tiles), A.n_tiles, order);
       if (tile >= A.n_tiles) break;
       const int64_t j0 = tile * kT;
       const int64_t nvalid = A.d - j0 < kT ? A.d - j0 : kT;
@@ -1097,24 +1170,27 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   bool ok = true;  // false after a bounded wait gave up: the items are skipped, the tile loop
                    // still runs (its named barriers need both warps of the sub-tile)
   // The sub-tile's w_t - w_{t-1} is formed by one of its two warps, the lead
-  // (the warp of the even workers), which pipelines the loads of the CTA's
-  // next tiles: while it works on tile n it loads w for tile n + 1, the pairs
-  // of tile n + 2 and the sub-chunk entries of tile n + 3. Fill: tiles 0-2.
+  // (the warp of the even workers), from the pairs pc and w at them wc of its
+  // tile, which it loaded while working on the tiles before (see above):
+  // deep, pn and cx are the pairs of tile n + 1 and the entries of tile n + 2;
+  // shallow, cx, pn and wn are the entries, pairs and w of tile n + 1.
   const bool lead = gp == 0;
-  Pairs p0{kNone, 0.f, 0, 0u}, p1{kNone, 0.f, 0, 0u};
-  float w0 = 0.f;
-  uint2 c2 = make_uint2(0u, 0u);
-  if (lead) {
-    p0 = pipe_pairs(A, pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, 0), sw, lane), own, lane);
-    p1 = pipe_pairs(A, pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, 1), sw, lane), own, lane);
-    w0 = pipe_w(A, p0, sm.Tp, sm.tip);
-    c2 = pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, 2), sw, lane);
+  // the CTA's n-th tile (tile_order)
+  auto tile_n = [&](uint32_t n) { return tile_order(tile_at_n<kQ>(sm.tq, n, F), A.n_tiles, order); };
+  Pairs pc{kNone, 0.f, 0, 0u}, pn{kNone, 0.f, 0, 0u};
+  float wc = 0.f;
+  uint2 cx = make_uint2(0u, 0u);
+  if (lead) {  // fill: the first tiles' chains
+    pc = pipe_pairs(A, pipe_chunk(A, tile_n(0), sw, lane), own, lane);
+    if (deep) pn = pipe_pairs(A, pipe_chunk(A, tile_n(1), sw, lane), own, lane);
+    wc = pipe_w(A, pc, sm.Tp, sm.tip);
+    if (deep) cx = pipe_chunk(A, tile_n(2), sw, lane);
   }
   const uint32_t pair_bar = 1 + sw;  // named barrier of the sub-tile's two warps
   // The sub-tile's two warps take their next tile from one read of its
   // queue slot (sm.next), so that both leave the loop together: the named
   // barriers need both. A warp whose wait gave up ends the CTA's tiles.
-  int64_t tile = tile_at<kFixed, kQ>(sm.tq, 0);
+  int64_t tile = tile_n(0);
   for (uint32_t n = 0; tile < A.n_tiles; ++n) {  // n: tiles done
     const uint32_t s0 = (uint32_t)(tile * kT) + sw * kSub;
     // this sub-tile's w_t - w_{t-1}, and the pending senders (their residual
@@ -1125,8 +1201,8 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
       bool many = false;
       if (A.dense_prev) {  // restored state: no pairs, w_t - w_{t-1} read densely
         stage_delta_dense(A, s0, kSub, dlw, lane);
-      } else if (p0.total <= 32u) {
-        up = apply_pairs(A, s0, p0, sm.Tp, sm.tip, w0, dlw, mkw, lane, lt, uni, chg);
+      } else if (pc.total <= 32u) {
+        up = apply_pairs(A, s0, pc, sm.Tp, sm.tip, wc, dlw, mkw, lane, lt, uni, chg);
       } else if (A.pending) {
         stage_pending_warp(A, tile, sw, s0, kSub, dlw, mkw, lane, uni, chg);
         many = true;
@@ -1146,17 +1222,22 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
     for (int u = 0; u < kSub / 128; ++u) dl4[u] = *reinterpret_cast<const float4*>(dlw + u * 128 + lane * 4);
     if (lead && lane == 0)  // the slot of tile n + 1 was published before tile n - 3's items
       sm.next[sw] = (!ok || n + 1 >= (uint64_t)A.n_tiles) ? (uint32_t)A.n_tiles
-                                                          : (uint32_t)tile_at<kFixed, kQ>(sm.tq, n + 1);
+                                                          : (uint32_t)tile_n(n + 1);
     // the lead warp rewrites the sub-tile's buffers for the next tile only after this
     asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
-    float w1 = 0.f;
-    Pairs p2{kNone, 0.f, 0, 0u};
-    uint2 c3 = make_uint2(0u, 0u);
+    float wn = 0.f;
+    Pairs pnn{kNone, 0.f, 0, 0u};
+    uint2 cxn = make_uint2(0u, 0u);
     if (lead) {  // the next tiles' loads, in flight while this tile is processed
-      w1 = pipe_w(A, p1, sm.Tp, sm.tip);
-      p2 = pipe_pairs(A, c2, own, lane);
-      c3 = pipe_chunk(A, tile_at<kFixed, kQ>(sm.tq, n + 3), sw, lane);
+      if (deep) {
+        wn = pipe_w(A, pn, sm.Tp, sm.tip);
+        pnn = pipe_pairs(A, cx, own, lane);
+        cxn = pipe_chunk(A, tile_n(n + 3), sw, lane);
+      } else {
+        cx = pipe_chunk(A, tile_n(n + 1), sw, lane);
+      }
     }
+    uint32_t item = 0;  // this warp's items of the tile so far
     const int64_t rem = A.d - (int64_t)s0;
     const int lim = rem < kSub ? (int)rem : kSub;
     // candidate flags of this lane's 16 values (bit 4u + i: value u*128 + lane*4 + i)
@@ -1166,6 +1247,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
 #pragma unroll
       for (int i = 0; i < 4; ++i) valid |= (u * 128 + lane * 4 + i < lim ? 1u : 0u) << (4 * u + i);
     uint2 bc_lane = make_uint2(0u, 0u);
+    uint32_t tcnt = 0;  // this warp's candidates of the tile (the block's cost, tile_order)
     for (int k = gp; ok && k < A.K; k += 2) {
       const uint32_t s = gp * kGroupStages + taken % kGroupStages, r = taken / kGroupStages;
       ++taken;
@@ -1250,6 +1332,7 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
       }
       bits &= th == kNoCandidate ? 0u : valid;
       const uint32_t cnt = __reduce_add_sync(0xffffffffu, __popc(bits));
+      tcnt += cnt;
       const uint32_t run_k = __shfl_sync(0xffffffffu, run, k);  // worker k's candidates so far
       if (cnt) {
         if (lane == 0 && run_k + cnt > A.cap_part) A.sel[k].dense = 1;  // part full: dense path
@@ -1307,14 +1390,26 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
         if (lane == k) run += cnt;
       }
       if (lane == k) bc_lane = make_uint2(part0 + run_k, cnt);
+      if (lead && !deep) {  // the next tile's chain, one link per item
+        if (item == 0) pn = pipe_pairs(A, cx, own, lane);
+        else if (item == 1) wn = pipe_w(A, pn, sm.Tp, sm.tip);
+      }
+      ++item;
+    }
+    if (lead && !deep && item < 2) {  // a wait gave up before the chain was complete
+      if (item == 0) pn = pipe_pairs(A, cx, own, lane);
+      wn = pipe_w(A, pn, sm.Tp, sm.tip);
     }
     // the tile's sub-chunk entries of this warp's workers: lane k holds worker k's
     if (ok && lane < A.K && (lane & 1) == gp) A.chunk[chunk_at(A, lane, tile, sw)] = bc_lane;
+    if (A.blk_cost && lane == 0 && tcnt && tile < (int64_t)nbw * G) atomicAdd(&A.blk_cost[tile / G], tcnt);
     if (lead) {
-      p0 = p1;
-      w0 = w1;
-      p1 = p2;
-      c2 = c3;
+      pc = pn;
+      wc = wn;
+      if (deep) {
+        pn = pnn;
+        cx = cxn;
+      }
     }
     // the per-element masks of a many-sender sub-tile stay in use until both warps are done
     if (many) asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
@@ -1565,6 +1660,256 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
     const uint32_t i = i0 + threadIdx.x;
     const bool tie = i < n && keys[i] == T;
     const uint32_t j = tie ? __ldcg(&bk[kBucketCap + i]) : 0u;
+    __syncthreads();
+    if (tie) keys[atomicAdd(&s_n, 1u)] = j;
+  }
+  __syncthreads();
+  const uint32_t ties = s_n;
+  uint32_t t_idx = 0xffffffffu;
+  if (ties > n_tie) {  // keep the n_tie lowest indices: t_idx = (ties - n_tie + 1)-th largest
+    uint32_t unused;
+    t_idx = smem_select(keys, ties, ties - n_tie + 1, h, ws, &s_bin, &s_rank, &unused);
+  }
+  if (threadIdx.x == 0) {
+    S.T = T;
+    S.n_tie = n_tie;
+    S.ties = ties;
+    S.t_idx = t_idx;
+    // ||C_k||_0: every key sent is >= T; only when T is the zero key are the
+    // n_tie ties kept zeros
+    atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(A.ksel - (T == 0u ? n_tie : 0u)));
+  }
+}
+
+// Radix select in shared memory over values below 2^nbits (nbits <= 31): the
+// r-th largest of n, in passes of at most 11 bits from the top (none for
+// nbits = 0: every value is 0). *rank_out receives r's rank among the values
+// equal to the result.
+__device__ __forceinline__ uint32_t smem_select_bits(const uint32_t* x, uint32_t n, uint32_t r, int nbits,
+                                                     uint32_t* h, uint32_t* ws, uint32_t* s_bin,
+                                                     uint32_t* s_rank, uint32_t* rank_out) {
+  uint32_t prefix = 0;
+  for (int hi = nbits; hi > 0;) {
+    const int width = hi < 11 ? hi : 11, lo = hi - width;
+    // block_find_from_top takes a multiple of the block's threads: the bins
+    // above 2^width stay empty
+    const int nbins = (1 << width) > (int)blockDim.x ? (1 << width) : (int)blockDim.x;
+    for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
+    if (threadIdx.x == 0) {
+      *s_bin = 0;
+      *s_rank = 0;
+    }
+    __syncthreads();
+    for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
+      const uint32_t i = i0 + threadIdx.x;
+      int bin = -1;
+      if (i < n) {
+        const uint32_t v = x[i];
+        if (hi == nbits || (v >> hi) == prefix) bin = (int)((v >> lo) & ((1u << width) - 1u));
+      }
+      warp_hist_add(h, bin);
+    }
+    __syncthreads();
+    block_find_from_top(h, nbins, r, ws, s_bin, s_rank);
+    prefix = (prefix << width) | *s_bin;
+    r = *s_rank;
+    __syncthreads();
+    hi = lo;
+  }
+  *rank_out = r;
+  return prefix;
+}
+
+// ---------------------------------------------------------------------------
+// Exact select on the bulk path with more than eight workers, one cluster of
+// eight CTAs per worker. The bulk pass has counted its
+// candidates into the relative histogram already. Every CTA first issues the
+// loads of its warps' part counts and candidates, and only then reads the
+// histogram and finds the bin holding the k-th key and its rank there, so
+// that the latencies overlap. The candidates in that bin are gathered in the
+// CTA's own shared memory first (warp reservations on a local counter), and
+// each CTA then reserves its block of the cluster's bucket in the first CTA's
+// shared memory with a single remote atomic and copies it there (a CTA whose
+// local bucket overflows writes the rest straight to the first CTA). After a
+// cluster barrier the first CTA ranks the bucket: the bin fixes the key's
+// high bits, so T is the bin's base plus the rank's offset, found in at most
+// two radix passes over the sel_shift bits the bin leaves open (three over
+// the whole key in the top bin, which also holds everything above it); then
+// the ties and the largest kept tie index, as k_select_finish does.
+// ---------------------------------------------------------------------------
+namespace ssel {
+constexpr int kCtas = 8;                        // CTAs per cluster, one cluster per worker
+constexpr int kThreadsC = 1024;
+constexpr int kWarpsC = kThreadsC / 32;
+constexpr int kQ = 8;                           // candidates per lane and round
+constexpr int kLocal = 1024;                    // a CTA's own bucket (two CTAs fit on an SM)
+constexpr int kSmem = (2 * kBucketCap + 2 * kLocal) * 4;  // the cluster's bucket (first CTA), the local one
+}  // namespace ssel
+
+__global__ void __launch_bounds__(ssel::kThreadsC) k_select_cluster(TopkArgs A) {
+  using namespace ssel;
+  griddep_wait();
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  extern __shared__ __align__(16) uint32_t sbuf[];
+  uint32_t* bkt = sbuf;                     // first CTA: kBucketCap keys, then kBucketCap indices
+  uint32_t* loc = sbuf + 2 * kBucketCap;    // this CTA: kLocal keys, then kLocal indices
+  __shared__ uint32_t h[kRelBins];
+  __shared__ uint32_t ws[32];
+  __shared__ uint32_t s_bin, s_rank, s_n, s_cnt, s_loc, s_base, s_skip, s_theta;
+  const int k = blockIdx.y;
+  const unsigned crank = cl.block_rank();
+  const int nctas = (int)cl.num_blocks();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t lt = lanemask_lt();
+  WorkerSel& S = A.sel[k];
+  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
+  const float* cv = A.cand_val + (int64_t)k * A.cap;
+  // this warp's run of at most 32 consecutive candidate parts, walked as one
+  // list: lane l holds the count of part p_lo + l
+  const int nparts = A.regions * kChunksPerTile;
+  const int nw = nctas * kWarpsC;
+  const int per = (nparts + nw - 1) / nw;
+  const int p_lo = min(nparts, ((int)crank * kWarpsC + warp) * per);
+  const int p_hi = min(nparts, p_lo + per);
+  const uint32_t cnt = p_lo + lane < p_hi ? A.rcount[(int64_t)k * nparts + p_lo + lane] : 0u;
+  uint32_t incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  const uint32_t total = __shfl_sync(0xffffffffu, incl, 31);
+  // the candidates of the round starting at list position i0
+  auto load_round = [&](uint32_t i0, uint32_t (&key)[kQ], uint32_t (&idx)[kQ], bool (&in)[kQ]) {
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      const uint32_t i = i0 + q * 32 + lane;
+      in[q] = i < total;
+      int lo = 0, hi = 32;  // the first lane whose inclusive count exceeds i
+#pragma unroll
+      for (int it = 0; it < 6; ++it) {
+        const int mid = min((lo + hi) >> 1, 31);
+        const uint32_t v = __shfl_sync(0xffffffffu, incl, mid);
+        if (lo < hi) {
+          if (v <= i) lo = mid + 1; else hi = mid;
+        }
+      }
+      const int L = lo < 32 ? lo : 31;
+      const uint32_t before = __shfl_sync(0xffffffffu, incl - cnt, L);
+      const uint32_t slot = (uint32_t)(p_lo + L) * A.cap_part + (i - before);
+      key[q] = in[q] ? mag_key(cv[slot]) : 0u;
+      idx[q] = in[q] ? ci[slot] : 0u;
+    }
+  };
+  uint32_t key[kQ], idx[kQ];
+  bool in[kQ];
+  load_round(0u, key, idx, in);
+  // the worker's state and histogram, read by every CTA before any CTA of the
+  // cluster writes the state (first barrier): all of them decide alike
+  if (threadIdx.x == 0) {
+    s_skip = needs_dense(S, A.ksel, A.cap) ? 1u : 0u;
+    s_theta = S.theta;
+    s_bin = 0;
+    s_rank = 0;
+    s_cnt = 0;
+    s_loc = 0;
+  }
+  for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) h[b] = __ldcg(&A.chist[(int64_t)k * kRelBins + b]);
+  __syncthreads();
+  block_find_from_top(h, kRelBins, A.ksel, ws, &s_bin, &s_rank);
+  const int want = (int)s_bin;
+  const uint32_t want_rank = s_rank;
+  const uint32_t theta = s_theta;
+  const bool skip = s_skip != 0u;
+  cl.sync();  // every CTA runs, has read the state, and the first CTA's count is zero
+  if (skip || want_rank == 0) {  // fewer candidates than k counted: the dense path decides
+    if (!skip && crank == 0 && threadIdx.x == 0) S.dense = 1;
+    return;
+  }
+  uint32_t* rcount = cl.map_shared_rank(&s_cnt, 0);
+  uint32_t* rb = cl.map_shared_rank(bkt, 0);
+  for (uint32_t i0 = 0; i0 < total; i0 += kQ * 32) {
+    uint32_t nkey[kQ], nidx[kQ];
+    bool nin[kQ];
+    if (i0 + kQ * 32 < total) load_round(i0 + kQ * 32, nkey, nidx, nin);  // warp-uniform
+    uint32_t m[kQ], n = 0;
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      m[q] = __ballot_sync(0xffffffffu, in[q] && rel_bin(key[q], theta, A.sel_shift) == want);
+      n += __popc(m[q]);
+    }
+    if (n) {
+      uint32_t base = 0;
+      if (lane == 0) base = atomicAdd(&s_loc, n);
+      base = __shfl_sync(0xffffffffu, base, 0);
+      uint32_t rbase = 0;  // the part beyond the local bucket goes straight to the first CTA
+      const uint32_t over = base + n > (uint32_t)kLocal ? base + n - max(base, (uint32_t)kLocal) : 0u;
+      if (over && lane == 0) rbase = atomicAdd(rcount, over);
+      rbase = __shfl_sync(0xffffffffu, rbase, 0);
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+        const uint32_t o = base + __popc(m[q] & lt);
+        if ((m[q] >> lane) & 1u) {
+          if (o < (uint32_t)kLocal) {
+            loc[o] = key[q];
+            loc[kLocal + o] = idx[q];
+          } else {
+            const uint32_t r = rbase + (o - max(base, (uint32_t)kLocal));
+            if (r < (uint32_t)kBucketCap) {
+              rb[r] = key[q];
+              rb[kBucketCap + r] = idx[q];
+            }
+          }
+        }
+        base += __popc(m[q]);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      key[q] = nkey[q];
+      idx[q] = nidx[q];
+      in[q] = i0 + kQ * 32 < total && nin[q];
+    }
+  }
+  __syncthreads();
+  const uint32_t nl = min(s_loc, (uint32_t)kLocal);
+  if (threadIdx.x == 0) s_base = nl ? atomicAdd(rcount, nl) : 0u;
+  __syncthreads();
+  for (uint32_t i = threadIdx.x; i < nl; i += blockDim.x) {
+    const uint32_t r = s_base + i;
+    if (r < (uint32_t)kBucketCap) {
+      rb[r] = loc[i];
+      rb[kBucketCap + r] = loc[kLocal + i];
+    }
+  }
+  cl.sync();  // the bucket is complete; no CTA touches another's shared memory after this
+  if (crank != 0) return;
+  const uint32_t n = s_cnt;
+  if (n > (uint32_t)kBucketCap) {  // the k-th key's bin is too crowded: the dense path decides
+    if (threadIdx.x == 0) S.dense = 1;
+    return;
+  }
+  uint32_t* keys = bkt;
+  uint32_t n_tie, T;
+  if (want < kRelBins - 1) {  // the bin's keys are base + [0, 2^sel_shift)
+    const uint32_t base = theta + ((uint32_t)want << A.sel_shift);
+    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) keys[i] -= base;
+    __syncthreads();
+    T = base + smem_select_bits(keys, n, want_rank, A.sel_shift, h, ws, &s_bin, &s_rank, &n_tie);
+    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) keys[i] += base;
+    __syncthreads();
+  } else {
+    T = smem_select(keys, n, want_rank, h, ws, &s_bin, &s_rank, &n_tie);
+  }
+  // ties: the indices of the keys equal to T, gathered over the keys in
+  // place; a round writes below the end of what the block has read so far
+  if (threadIdx.x == 0) s_n = 0;
+  __syncthreads();
+  for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
+    const uint32_t i = i0 + threadIdx.x;
+    const bool tie = i < n && keys[i] == T;
+    const uint32_t j = tie ? bkt[kBucketCap + i] : 0u;
     __syncthreads();
     if (tie) keys[atomicAdd(&s_n, 1u)] = j;
   }
@@ -2018,6 +2363,7 @@ cudaError_t configure_topk_kernels() {
   set((const void*)k_accumulate_bulk<true, true>, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_select_finish, kBucketCap * 4);
   set((const void*)k_sample_theta, kBucketCap * 4);
+  set((const void*)k_select_cluster, ssel::kSmem);
   return err;
 }
 
@@ -2036,7 +2382,8 @@ int accumulate_blocks_per_sm(int tile) {
 cudaError_t launch_sample(const TopkArgs& A, cudaStream_t s) {
   if ((A.pending || A.approx) && !A.dense_mode) {
     const int n_s = (int)A.n_sample;
-    const cudaError_t err = launch_pdl(k_sample_pending, dim3((n_s + kThreads - 1) / kThreads), dim3(kThreads), 0, s, A);
+    const unsigned grid = (unsigned)((n_s + kThreads - 1) / kThreads) + (A.use_order ? 1u : 0u);
+    const cudaError_t err = launch_pdl(k_sample_pending, dim3(grid), dim3(kThreads), 0, s, A);
     if (err != cudaSuccess) return err;
   }
   if (!A.approx) return launch_pdl(k_sample_cluster, dim3(scl::kCtas, A.K), dim3(scl::kThreadsC), 0, s, A);
@@ -2071,6 +2418,27 @@ cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
 }
 
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s) {
+  // the bulk pass's candidate parts with more than eight workers: one cluster
+  // per worker, each warp a run of at most 32 parts (with fewer workers eight
+  // CTAs a worker are too few: k_select_finish spreads them over the SMs)
+  const int C = ssel::kCtas;
+  if (A.regions > 1 && A.K > 8 && A.regions * kChunksPerTile <= 32 * C * ssel::kWarpsC) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(C, A.K);
+    cfg.blockDim = dim3(ssel::kThreadsC);
+    cfg.dynamicSmemBytes = ssel::kSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = C;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, k_select_cluster, A);
+  }
   const dim3 grid(blocks_per_worker, A.K);
   if (A.regions == 1) {  // the bulk pass histogrammed its candidates already
     const cudaError_t err = launch_pdl(k_select_hist, grid, dim3(kThreads), 0, s, A);

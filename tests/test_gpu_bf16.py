@@ -25,6 +25,7 @@ def _bf16_grads(rng, K, d, dev, offset=0):
 
 CASES = [
     dict(compressor="topk", d=1_300_001, K=4, ratio=0.002),
+    dict(compressor="topk", d=1_300_001, K=6, ratio=0.002),
     dict(compressor="topk", d=1_300_001, K=3, ratio=0.002, offset=1),
     dict(compressor="topk", d=50_003, K=3, ratio=0.01),
     dict(compressor="topk_approx", d=1_300_001, K=3, ratio=1 / 1024),

@@ -23,6 +23,7 @@ def _fresh(p, **kw):
 
 CASES = [
     dict(compressor="topk", d=1_300_001, K=4, ratio=0.002),               # bulk pass, deferred
+    dict(compressor="topk", d=1_300_001, K=6, ratio=0.002),               # and its one-tile pipeline
     dict(compressor="topk", d=50_003, K=3, ratio=0.01),                   # load/store pass
     dict(compressor="topk_approx", d=1_300_001, K=3, ratio=1 / 1024),
     dict(compressor="rbgs", d=4096 * 160 + 3, K=5, ratio=0.05, block=4096, lam=0.5),
@@ -30,6 +31,7 @@ CASES = [
     dict(compressor="topk", d=1_300_001, K=3, ratio=0.002, variant="server_momentum"),
     dict(compressor="topk", d=1_300_001, K=3, ratio=0.002, variant="lr_in_residual"),
     dict(compressor="topk", d=1_300_001, K=3, ratio=0.002, variant="local_momentum"),
+    dict(compressor="topk", d=1_300_001, K=7, ratio=0.002, variant="local_momentum"),
     dict(compressor="topk_approx", d=50_003, K=2, ratio=0.01, variant="local_momentum_mfm"),
 ]
 

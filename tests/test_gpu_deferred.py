@@ -120,10 +120,11 @@ def test_host_steps_pinned_and_pageable(pinned):
 
 def test_dense_sub_tiles_and_ties_on_the_bulk_pass():
     """Many sent pairs per 512-coordinate sub-tile (more than one per lane:
-    the per-element sender masks), K = 1 and an odd K, ties across tiles,
+    the per-element sender masks), K = 1, an odd K and K = 12 (the select
+    runs as one cluster per worker above eight workers), ties across tiles,
     deferred and host (applied at once) steps alternating."""
     import torch
-    for K, ratio in ((1, 0.05), (7, 0.02)):
+    for K, ratio in ((1, 0.05), (7, 0.02), (12, 0.01)):
         rng = np.random.default_rng(40 + K)
         p = Pair(D_BULK, K, 0.9, 0.1, ratio=ratio, seed=9)
         stats = torch.zeros(8, dtype=torch.int64).pin_memory()
@@ -158,16 +159,17 @@ def test_bulk_pass_reports_non_finite_values():
     assert p.gpu.check() == 4  # GMC_ENONFINITE
 
 
-@pytest.mark.parametrize("K", [1, 2, 5])
+@pytest.mark.parametrize("K", [1, 2, 5, 6, 7, 16])
 def test_claimed_tiles_and_odd_worker_counts(K):
     """Several tiles per CTA beyond its fixed ones, so the bulk pass claims
     the rest from its tile counter; the worker-parity warp groups each read
     their own stages of the ring, in order, for every K (odd K gives the two
     groups different item counts per tile, K = 1 leaves one group without
-    items)."""
+    items). K <= 5 runs the three-tile pipeline of w_t - w_{t-1}, K >= 6 the
+    one-tile pipeline with two tiles claimed ahead."""
     d = 152 * 4096 * 9 + 1001  # about nine tiles per CTA
     rng = np.random.default_rng(40 + K)
-    p = Pair(d, K, 0.9, 0.1, ratio=0.001, seed=9)
+    p = Pair(d, K, 0.9, 0.1, ratio=0.001, seed=9, ref="cpp")
     for t in range(3):
         r = p.step(_grads(rng, K, d))
         p.compare(r, state=False)
