@@ -631,12 +631,14 @@ int gmc_create(gmc_t* out, int64_t d, int32_t K, float beta, float eta, int32_t 
     const int64_t per = (h->cap + 8191) / 8192;
     h->grid_agg = h->regions > 1 ? h->regions : (int)std::max<int64_t>(1, 4 * (int64_t)h->num_sms / K);
     // select: on the bulk path a warp walks the candidates of a run of at most
-    // 32 parts as one list; the grid is one wave of four blocks per SM (each
-    // holds kBucketCap keys of shared memory), for all the workers
+    // 32 parts as one list; the grid is one wave of as many blocks as fit on
+    // an SM (each holds kBucketCap keys of shared memory: three on GB300), for
+    // all the workers -- a second, partial wave cost about 10 us
     const int64_t nparts = (int64_t)h->regions * kChunksPerTile;
+    const int64_t sel_wave = (int64_t)select_blocks_per_sm() * h->num_sms;
     h->sel_blocks = h->regions > 1 ? (int)std::min<int64_t>(
                                          h->regions, std::max<int64_t>((nparts + 32 * kWarps - 1) / (32 * kWarps),
-                                                                       std::max<int64_t>(1, 4 * (int64_t)h->num_sms / K)))
+                                                                       std::max<int64_t>(1, sel_wave / K)))
                                    : (int)std::max<int64_t>(1, std::min<int64_t>(per, std::max<int64_t>(1, streams_wide / K)));
     if (compressor == GMC_TOPK) h->n_sample = (uint32_t)(h->sample_chunks ? kSampleSlots : d);
     h->sample_stride = std::max<uint32_t>(kSampleSlots, (h->n_sample + 3) & ~3u);

@@ -218,6 +218,7 @@ cudaError_t launch_finalize(Counters* step, Counters* total, unsigned long long 
 // Occupancy-derived persistent grid sizes.
 int accumulate_blocks_per_sm(int tile);
 int rbgs_blocks_per_sm();
+int select_blocks_per_sm();  // resident k_select_finish blocks per SM (its grid is one wave)
 int accumulate_smem_bytes(int tile, int K);
 cudaError_t configure_topk_kernels();
 cudaError_t configure_rbgs_kernels();

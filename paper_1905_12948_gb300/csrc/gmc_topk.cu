@@ -430,7 +430,9 @@ __global__ void __cluster_dims__(scl::kCtas, 1, 1) __launch_bounds__(scl::kThrea
     const float e = ((pm[q] >> k) & 1u) ? 0.f : ev[q];
     const float dl = pm[q] ? __uint_as_float(pd[q]) : dv[q];
     key[q] = i < n_s ? mag_key(accumulate(e, g, A.c, dl)) : 0xffffffffu;
-    warp_hist_add(hist, key[q] != 0xffffffffu ? (int)(key[q] >> 20) : -1);
+    // plain shared-memory atomics: a warp's keys spread over a few dozen bins,
+    // and the warp-aggregated form (match_any) measured slower here
+    if (key[q] != 0xffffffffu) atomicAdd(&hist[key[q] >> 20], 1u);
   }
   // every CTA of the cluster runs and has zeroed its histograms before any remote add
   cl.sync();
@@ -452,7 +454,7 @@ __global__ void __cluster_dims__(scl::kCtas, 1, 1) __launch_bounds__(scl::kThrea
   __syncthreads();
 #pragma unroll
   for (int q = 0; q < kSlots; ++q)
-    warp_hist_add(hist, (key[q] != 0xffffffffu && (key[q] >> 20) == b1) ? (int)((key[q] >> 10) & 1023u) : -1);
+    if (key[q] != 0xffffffffu && (key[q] >> 20) == b1) atomicAdd(&hist[(key[q] >> 10) & 1023u], 1u);
   __syncthreads();
   uint32_t* r2 = cl.map_shared_rank(red2, 0);
   for (int b = threadIdx.x; b < 1024; b += blockDim.x)
@@ -1681,256 +1683,6 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   }
 }
 
-// Radix select in shared memory over values below 2^nbits (nbits <= 31): the
-// r-th largest of n, in passes of at most 11 bits from the top (none for
-// nbits = 0: every value is 0). *rank_out receives r's rank among the values
-// equal to the result.
-__device__ __forceinline__ uint32_t smem_select_bits(const uint32_t* x, uint32_t n, uint32_t r, int nbits,
-                                                     uint32_t* h, uint32_t* ws, uint32_t* s_bin,
-                                                     uint32_t* s_rank, uint32_t* rank_out) {
-  uint32_t prefix = 0;
-  for (int hi = nbits; hi > 0;) {
-    const int width = hi < 11 ? hi : 11, lo = hi - width;
-    // block_find_from_top takes a multiple of the block's threads: the bins
-    // above 2^width stay empty
-    const int nbins = (1 << width) > (int)blockDim.x ? (1 << width) : (int)blockDim.x;
-    for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
-    if (threadIdx.x == 0) {
-      *s_bin = 0;
-      *s_rank = 0;
-    }
-    __syncthreads();
-    for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
-      const uint32_t i = i0 + threadIdx.x;
-      int bin = -1;
-      if (i < n) {
-        const uint32_t v = x[i];
-        if (hi == nbits || (v >> hi) == prefix) bin = (int)((v >> lo) & ((1u << width) - 1u));
-      }
-      warp_hist_add(h, bin);
-    }
-    __syncthreads();
-    block_find_from_top(h, nbins, r, ws, s_bin, s_rank);
-    prefix = (prefix << width) | *s_bin;
-    r = *s_rank;
-    __syncthreads();
-    hi = lo;
-  }
-  *rank_out = r;
-  return prefix;
-}
-
-// ---------------------------------------------------------------------------
-// Exact select on the bulk path with more than eight workers, one cluster of
-// eight CTAs per worker. The bulk pass has counted its
-// candidates into the relative histogram already. Every CTA first issues the
-// loads of its warps' part counts and candidates, and only then reads the
-// histogram and finds the bin holding the k-th key and its rank there, so
-// that the latencies overlap. The candidates in that bin are gathered in the
-// CTA's own shared memory first (warp reservations on a local counter), and
-// each CTA then reserves its block of the cluster's bucket in the first CTA's
-// shared memory with a single remote atomic and copies it there (a CTA whose
-// local bucket overflows writes the rest straight to the first CTA). After a
-// cluster barrier the first CTA ranks the bucket: the bin fixes the key's
-// high bits, so T is the bin's base plus the rank's offset, found in at most
-// two radix passes over the sel_shift bits the bin leaves open (three over
-// the whole key in the top bin, which also holds everything above it); then
-// the ties and the largest kept tie index, as k_select_finish does.
-// ---------------------------------------------------------------------------
-namespace ssel {
-constexpr int kCtas = 8;                        // CTAs per cluster, one cluster per worker
-constexpr int kThreadsC = 1024;
-constexpr int kWarpsC = kThreadsC / 32;
-constexpr int kQ = 8;                           // candidates per lane and round
-constexpr int kLocal = 1024;                    // a CTA's own bucket (two CTAs fit on an SM)
-constexpr int kSmem = (2 * kBucketCap + 2 * kLocal) * 4;  // the cluster's bucket (first CTA), the local one
-}  // namespace ssel
-
-__global__ void __launch_bounds__(ssel::kThreadsC) k_select_cluster(TopkArgs A) {
-  using namespace ssel;
-  griddep_wait();
-  namespace cg = cooperative_groups;
-  cg::cluster_group cl = cg::this_cluster();
-  extern __shared__ __align__(16) uint32_t sbuf[];
-  uint32_t* bkt = sbuf;                     // first CTA: kBucketCap keys, then kBucketCap indices
-  uint32_t* loc = sbuf + 2 * kBucketCap;    // this CTA: kLocal keys, then kLocal indices
-  __shared__ uint32_t h[kRelBins];
-  __shared__ uint32_t ws[32];
-  __shared__ uint32_t s_bin, s_rank, s_n, s_cnt, s_loc, s_base, s_skip, s_theta;
-  const int k = blockIdx.y;
-  const unsigned crank = cl.block_rank();
-  const int nctas = (int)cl.num_blocks();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t lt = lanemask_lt();
-  WorkerSel& S = A.sel[k];
-  const uint32_t* ci = A.cand_idx + (int64_t)k * A.cap;
-  const float* cv = A.cand_val + (int64_t)k * A.cap;
-  // this warp's run of at most 32 consecutive candidate parts, walked as one
-  // list: lane l holds the count of part p_lo + l
-  const int nparts = A.regions * kChunksPerTile;
-  const int nw = nctas * kWarpsC;
-  const int per = (nparts + nw - 1) / nw;
-  const int p_lo = min(nparts, ((int)crank * kWarpsC + warp) * per);
-  const int p_hi = min(nparts, p_lo + per);
-  const uint32_t cnt = p_lo + lane < p_hi ? A.rcount[(int64_t)k * nparts + p_lo + lane] : 0u;
-  uint32_t incl = cnt;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += y;
-  }
-  const uint32_t total = __shfl_sync(0xffffffffu, incl, 31);
-  // the candidates of the round starting at list position i0
-  auto load_round = [&](uint32_t i0, uint32_t (&key)[kQ], uint32_t (&idx)[kQ], bool (&in)[kQ]) {
-#pragma unroll
-    for (int q = 0; q < kQ; ++q) {
-      const uint32_t i = i0 + q * 32 + lane;
-      in[q] = i < total;
-      int lo = 0, hi = 32;  // the first lane whose inclusive count exceeds i
-#pragma unroll
-      for (int it = 0; it < 6; ++it) {
-        const int mid = min((lo + hi) >> 1, 31);
-        const uint32_t v = __shfl_sync(0xffffffffu, incl, mid);
-        if (lo < hi) {
-          if (v <= i) lo = mid + 1; else hi = mid;
-        }
-      }
-      const int L = lo < 32 ? lo : 31;
-      const uint32_t before = __shfl_sync(0xffffffffu, incl - cnt, L);
-      const uint32_t slot = (uint32_t)(p_lo + L) * A.cap_part + (i - before);
-      key[q] = in[q] ? mag_key(cv[slot]) : 0u;
-      idx[q] = in[q] ? ci[slot] : 0u;
-    }
-  };
-  uint32_t key[kQ], idx[kQ];
-  bool in[kQ];
-  load_round(0u, key, idx, in);
-  // the worker's state and histogram, read by every CTA before any CTA of the
-  // cluster writes the state (first barrier): all of them decide alike
-  if (threadIdx.x == 0) {
-    s_skip = needs_dense(S, A.ksel, A.cap) ? 1u : 0u;
-    s_theta = S.theta;
-    s_bin = 0;
-    s_rank = 0;
-    s_cnt = 0;
-    s_loc = 0;
-  }
-  for (int b = threadIdx.x; b < kRelBins; b += blockDim.x) h[b] = __ldcg(&A.chist[(int64_t)k * kRelBins + b]);
-  __syncthreads();
-  block_find_from_top(h, kRelBins, A.ksel, ws, &s_bin, &s_rank);
-  const int want = (int)s_bin;
-  const uint32_t want_rank = s_rank;
-  const uint32_t theta = s_theta;
-  const bool skip = s_skip != 0u;
-  cl.sync();  // every CTA runs, has read the state, and the first CTA's count is zero
-  if (skip || want_rank == 0) {  // fewer candidates than k counted: the dense path decides
-    if (!skip && crank == 0 && threadIdx.x == 0) S.dense = 1;
-    return;
-  }
-  uint32_t* rcount = cl.map_shared_rank(&s_cnt, 0);
-  uint32_t* rb = cl.map_shared_rank(bkt, 0);
-  for (uint32_t i0 = 0; i0 < total; i0 += kQ * 32) {
-    uint32_t nkey[kQ], nidx[kQ];
-    bool nin[kQ];
-    if (i0 + kQ * 32 < total) load_round(i0 + kQ * 32, nkey, nidx, nin);  // warp-uniform
-    uint32_t m[kQ], n = 0;
-#pragma unroll
-    for (int q = 0; q < kQ; ++q) {
-      m[q] = __ballot_sync(0xffffffffu, in[q] && rel_bin(key[q], theta, A.sel_shift) == want);
-      n += __popc(m[q]);
-    }
-    if (n) {
-      uint32_t base = 0;
-      if (lane == 0) base = atomicAdd(&s_loc, n);
-      base = __shfl_sync(0xffffffffu, base, 0);
-      uint32_t rbase = 0;  // the part beyond the local bucket goes straight to the first CTA
-      const uint32_t over = base + n > (uint32_t)kLocal ? base + n - max(base, (uint32_t)kLocal) : 0u;
-      if (over && lane == 0) rbase = atomicAdd(rcount, over);
-      rbase = __shfl_sync(0xffffffffu, rbase, 0);
-#pragma unroll
-      for (int q = 0; q < kQ; ++q) {
-        const uint32_t o = base + __popc(m[q] & lt);
-        if ((m[q] >> lane) & 1u) {
-          if (o < (uint32_t)kLocal) {
-            loc[o] = key[q];
-            loc[kLocal + o] = idx[q];
-          } else {
-            const uint32_t r = rbase + (o - max(base, (uint32_t)kLocal));
-            if (r < (uint32_t)kBucketCap) {
-              rb[r] = key[q];
-              rb[kBucketCap + r] = idx[q];
-            }
-          }
-        }
-        base += __popc(m[q]);
-      }
-    }
-#pragma unroll
-    for (int q = 0; q < kQ; ++q) {
-      key[q] = nkey[q];
-      idx[q] = nidx[q];
-      in[q] = i0 + kQ * 32 < total && nin[q];
-    }
-  }
-  __syncthreads();
-  const uint32_t nl = min(s_loc, (uint32_t)kLocal);
-  if (threadIdx.x == 0) s_base = nl ? atomicAdd(rcount, nl) : 0u;
-  __syncthreads();
-  for (uint32_t i = threadIdx.x; i < nl; i += blockDim.x) {
-    const uint32_t r = s_base + i;
-    if (r < (uint32_t)kBucketCap) {
-      rb[r] = loc[i];
-      rb[kBucketCap + r] = loc[kLocal + i];
-    }
-  }
-  cl.sync();  // the bucket is complete; no CTA touches another's shared memory after this
-  if (crank != 0) return;
-  const uint32_t n = s_cnt;
-  if (n > (uint32_t)kBucketCap) {  // the k-th key's bin is too crowded: the dense path decides
-    if (threadIdx.x == 0) S.dense = 1;
-    return;
-  }
-  uint32_t* keys = bkt;
-  uint32_t n_tie, T;
-  if (want < kRelBins - 1) {  // the bin's keys are base + [0, 2^sel_shift)
-    const uint32_t base = theta + ((uint32_t)want << A.sel_shift);
-    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) keys[i] -= base;
-    __syncthreads();
-    T = base + smem_select_bits(keys, n, want_rank, A.sel_shift, h, ws, &s_bin, &s_rank, &n_tie);
-    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) keys[i] += base;
-    __syncthreads();
-  } else {
-    T = smem_select(keys, n, want_rank, h, ws, &s_bin, &s_rank, &n_tie);
-  }
-  // ties: the indices of the keys equal to T, gathered over the keys in
-  // place; a round writes below the end of what the block has read so far
-  if (threadIdx.x == 0) s_n = 0;
-  __syncthreads();
-  for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
-    const uint32_t i = i0 + threadIdx.x;
-    const bool tie = i < n && keys[i] == T;
-    const uint32_t j = tie ? bkt[kBucketCap + i] : 0u;
-    __syncthreads();
-    if (tie) keys[atomicAdd(&s_n, 1u)] = j;
-  }
-  __syncthreads();
-  const uint32_t ties = s_n;
-  uint32_t t_idx = 0xffffffffu;
-  if (ties > n_tie) {  // keep the n_tie lowest indices: t_idx = (ties - n_tie + 1)-th largest
-    uint32_t unused;
-    t_idx = smem_select(keys, ties, ties - n_tie + 1, h, ws, &s_bin, &s_rank, &unused);
-  }
-  if (threadIdx.x == 0) {
-    S.T = T;
-    S.n_tie = n_tie;
-    S.ties = ties;
-    S.t_idx = t_idx;
-    // ||C_k||_0: every key sent is >= T; only when T is the zero key are the
-    // n_tie ties kept zeros
-    atomicAdd(&A.step_ctr->v[kNnz], (unsigned long long)(A.ksel - (T == 0u ? n_tie : 0u)));
-  }
-}
-
 // ---------------------------------------------------------------------------
 // Approximate top-s (Sec. 5.1): the candidates are C(v) itself -- every key
 // >= theta, all ties kept. One block per worker records T = theta and the
@@ -2363,8 +2115,14 @@ cudaError_t configure_topk_kernels() {
   set((const void*)k_accumulate_bulk<true, true>, bulk::smem_bytes(kBulkMaxK));
   set((const void*)k_select_finish, kBucketCap * 4);
   set((const void*)k_sample_theta, kBucketCap * 4);
-  set((const void*)k_select_cluster, ssel::kSmem);
   return err;
+}
+
+int select_blocks_per_sm() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_select_finish, kThreads, kBucketCap * 4) != cudaSuccess)
+    cudaGetLastError();
+  return n > 0 ? n : 1;
 }
 
 int accumulate_blocks_per_sm(int tile) {
@@ -2418,27 +2176,6 @@ cudaError_t launch_accumulate(const TopkArgs& A, int grid, cudaStream_t s) {
 }
 
 cudaError_t launch_select(const TopkArgs& A, int blocks_per_worker, cudaStream_t s) {
-  // the bulk pass's candidate parts with more than eight workers: one cluster
-  // per worker, each warp a run of at most 32 parts (with fewer workers eight
-  // CTAs a worker are too few: k_select_finish spreads them over the SMs)
-  const int C = ssel::kCtas;
-  if (A.regions > 1 && A.K > 8 && A.regions * kChunksPerTile <= 32 * C * ssel::kWarpsC) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(C, A.K);
-    cfg.blockDim = dim3(ssel::kThreadsC);
-    cfg.dynamicSmemBytes = ssel::kSmem;
-    cfg.stream = s;
-    cudaLaunchAttribute at[2];
-    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    at[0].val.programmaticStreamSerializationAllowed = 1;
-    at[1].id = cudaLaunchAttributeClusterDimension;
-    at[1].val.clusterDim.x = C;
-    at[1].val.clusterDim.y = 1;
-    at[1].val.clusterDim.z = 1;
-    cfg.attrs = at;
-    cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, k_select_cluster, A);
-  }
   const dim3 grid(blocks_per_worker, A.K);
   if (A.regions == 1) {  // the bulk pass histogrammed its candidates already
     const cudaError_t err = launch_pdl(k_select_hist, grid, dim3(kThreads), 0, s, A);

@@ -120,9 +120,8 @@ def test_host_steps_pinned_and_pageable(pinned):
 
 def test_dense_sub_tiles_and_ties_on_the_bulk_pass():
     """Many sent pairs per 512-coordinate sub-tile (more than one per lane:
-    the per-element sender masks), K = 1, an odd K and K = 12 (the select
-    runs as one cluster per worker above eight workers), ties across tiles,
-    deferred and host (applied at once) steps alternating."""
+    the per-element sender masks), K = 1, an odd K and K = 12, ties across
+    tiles, deferred and host (applied at once) steps alternating."""
     import torch
     for K, ratio in ((1, 0.05), (7, 0.02), (12, 0.01)):
         rng = np.random.default_rng(40 + K)
