@@ -326,7 +326,7 @@ __device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, u
         const uint32_t v = x[i];
         if (pass == 0 || (v >> (shift + 10)) == prefix) bin = (int)((v >> shift) & (uint32_t)(nbins - 1));
       }
-      warp_hist_add(h, bin);
+      if (bin >= 0) atomicAdd(&h[bin], 1u);  // plain atomics measured faster than match_any here
     }
     __syncthreads();
     block_find_from_top(h, nbins, r, ws, s_bin, s_rank);
