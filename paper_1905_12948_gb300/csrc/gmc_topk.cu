@@ -896,7 +896,8 @@ __global__ void __launch_bounds__(kThreads) k_accumulate(TopkArgs A) {
 // sub-chunk table, then the pairs -- and the pending case reads w at the
 // pairs' coordinates: a chain of three memory latencies. The warp runs that
 // chain as a pipeline, so that no latency lies on its path. With few workers
-// (K <= 5, short tiles) the pipeline spans tiles: while the warp works on
+// (K <= 5, short tiles), and in the bf16 and local-momentum forms, the
+// pipeline spans tiles: while the warp works on
 // tile n it loads w for tile n+1, the pairs of tile n+2 and the sub-chunk
 // entries of tile n+3. With more workers a tile lasts long enough for the
 // whole chain of tile n+1: its entries at the start of tile n, its pairs
@@ -1078,7 +1079,10 @@ __global__ void __launch_bounds__(bulk::kThreadsAll, 1) k_accumulate_bulk(TopkAr
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool deep = A.K <= kDeepMaxK;  // the lead warp's pipeline spans three tiles
+  // the lead warp's pipeline spans three tiles: for few workers, and for the
+  // bf16 and local-momentum forms, where the one-tile pipeline measured slower
+  // (vgg16_bf16 1.98 -> 1.93 ms, vgg16_local 3.51 -> 3.45 ms with it spanning three)
+  const bool deep = (kLocal || kBf16) ? true : A.K <= kDeepMaxK;
   const uint32_t F = deep ? kFixedDeep : kFixedShallow;
   const uint32_t* order = A.use_order ? A.blk_order : nullptr;  // the tiles' order (tile_order)
   const uint32_t G = gridDim.x, nbw = (uint32_t)(A.n_tiles / G);  // whole blocks of G tiles
