@@ -13,7 +13,8 @@ constexpr uint32_t kNoCandidate = 0xffffffffu; // threshold above every key
 constexpr int kThreads = 256;                // block size of the streaming kernels
 constexpr int kWarps = kThreads / 32;
 constexpr int kSampleThreads = 1024;
-constexpr int kSampleRun = 8;                // consecutive coordinates per sampled run (power of two)
+constexpr int kSampleRun = 16;               // consecutive coordinates per sampled run (power of two):
+                                             // 64 bytes of a row, one DRAM burst
 constexpr int kSampleAll = 32768;            // d at or below which every element is sampled
 constexpr int kSampleSlots = 32768;          // sampled positions per worker (= kSampleAll)
 constexpr int kSampleChunks = kSampleSlots / kSampleRun;  // sampled runs per worker
@@ -201,6 +202,32 @@ __device__ __forceinline__ void block_find_from_top(const uint32_t* hist, int nb
   uint32_t above = incl - mine;  // keys in buckets above mine
   if (above < r && r <= incl) {
     for (int i = 1; i <= per; ++i) {
+      const uint32_t h = hist[hi - i];
+      if (r <= above + h) {
+        *out_bin = uint32_t(hi - i);
+        *out_rank = r - above;
+        break;
+      }
+      above += h;
+    }
+  }
+  __syncthreads();
+}
+
+// The same for any power-of-two nbins, also fewer bins than threads (a thread
+// owns at most max(1, nbins / blockDim.x) of them; the others none).
+__device__ __forceinline__ void block_find_from_top_any(const uint32_t* hist, int nbins, uint32_t r,
+                                                        uint32_t* ws, uint32_t* out_bin,
+                                                        uint32_t* out_rank) {
+  const int per = nbins >= (int)blockDim.x ? nbins / (int)blockDim.x : 1;
+  const int hi = nbins - (int)threadIdx.x * per;  // this thread's bins: [hi - per, hi), none when hi <= 0
+  uint32_t mine = 0;
+  for (int i = 1; i <= per && hi - i >= 0; ++i) mine += hist[hi - i];
+  uint32_t total;
+  const uint32_t incl = block_inclusive_scan<uint32_t>(mine, ws, &total);
+  uint32_t above = incl - mine;
+  if (above < r && r <= incl) {
+    for (int i = 1; i <= per && hi - i >= 0; ++i) {
       const uint32_t h = hist[hi - i];
       if (r <= above + h) {
         *out_bin = uint32_t(hi - i);

@@ -97,9 +97,10 @@ __device__ __forceinline__ uint32_t warp_excl_scan(uint32_t x, uint32_t* total) 
   return incl - x;
 }
 
-// Sampled coordinate of slot i. Exact top-k: 8 consecutive coordinates from
-// (c * d / chunks) rounded down to a multiple of 8, c = 0 .. chunks-1 (every
-// coordinate when chunks = 0). Approximate top-s (Sec. 5.1): run i/8 of the
+// Sampled coordinate of slot i. Exact top-k: kSampleRun (16) consecutive
+// coordinates from (c * d / chunks) rounded down to a multiple of kSampleRun,
+// c = 0 .. chunks-1 (every coordinate when chunks = 0); this sample only sets
+// the candidate threshold, never the result. Approximate top-s (Sec. 5.1): run i/8 of the
 // n = n_sample/8 runs of 8 consecutive coordinates, one per stratum
 // [r d / n, (r+1) d / n), starting on a multiple of 8 inside it at the slot
 // the r-th draw of the step's shared stream `key` picks (d < 8: slot i).
@@ -305,6 +306,43 @@ __global__ void __launch_bounds__(kThreads) k_sample(TopkArgs A) {
   // k_sample_theta fixes theta exactly from the keys and this histogram
 }
 
+// Radix select in shared memory over values below 2^bits (bits <= 31), taken
+// relative to `base` (x[i] - base): digits of at most 11 bits from the top.
+// Returns base + the r-th largest; rank_out = its rank among the values equal
+// to it. With bits = 31 and base = 0 this is a select over whole keys.
+__device__ __forceinline__ uint32_t smem_select_bits(const uint32_t* x, uint32_t n, uint32_t r, int bits,
+                                                     uint32_t base, uint32_t* h, uint32_t* ws,
+                                                     uint32_t* s_bin, uint32_t* s_rank, uint32_t* rank_out) {
+  uint32_t prefix = 0;  // the digits fixed so far
+  int done = 0;         // bits fixed so far (from the top)
+  while (done < bits) {
+    const int width = min(11, bits - done), shift = bits - done - width, nbins = 1 << width;
+    for (int b = threadIdx.x; b < nbins; b += blockDim.x) h[b] = 0;
+    if (threadIdx.x == 0) {
+      *s_bin = 0;
+      *s_rank = 0;
+    }
+    __syncthreads();
+    for (uint32_t i0 = 0; i0 < n; i0 += blockDim.x) {
+      const uint32_t i = i0 + threadIdx.x;
+      if (i < n) {
+        const uint32_t v = x[i] - base;
+        // the digits above this one must match the prefix (a shift by 32 is
+        // avoided: no digit is fixed before the first pass)
+        if (done == 0 || (v >> (shift + width)) == prefix) atomicAdd(&h[(v >> shift) & (uint32_t)(nbins - 1)], 1u);
+      }
+    }
+    __syncthreads();
+    block_find_from_top_any(h, nbins, r, ws, s_bin, s_rank);
+    prefix = (prefix << width) | *s_bin;
+    r = *s_rank;
+    done += width;
+    __syncthreads();
+  }
+  *rank_out = r;
+  return base + prefix;
+}
+
 // Radix select in shared memory: the r-th largest of n values (digits 11/10/10).
 __device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, uint32_t r,
                                                 uint32_t* h, uint32_t* ws, uint32_t* s_bin,
@@ -350,11 +388,53 @@ __device__ __forceinline__ uint32_t smem_select(const uint32_t* x, uint32_t n, u
 // sampled key within 2^10 keys. Distributed shared memory and hardware
 // barriers only: no global scratch, no spin-wait.
 // ---------------------------------------------------------------------------
+// Eight consecutive values from p: two 16-byte loads when p is 16-byte
+// aligned, else eight 4-byte (or 2-byte) loads.
+__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+  if ((reinterpret_cast<uintptr_t>(p) & 15u) == 0) {
+    const float4 a = *reinterpret_cast<const float4*>(p), b = *reinterpret_cast<const float4*>(p + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  } else {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) v[q] = p[q];
+  }
+}
+__device__ __forceinline__ void load8u(const uint32_t* p, uint32_t (&v)[8]) {
+  if ((reinterpret_cast<uintptr_t>(p) & 15u) == 0) {
+    const uint4 a = *reinterpret_cast<const uint4*>(p), b = *reinterpret_cast<const uint4*>(p + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  } else {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) v[q] = p[q];
+  }
+}
+__device__ __forceinline__ void load8_bf16(const uint16_t* p, float (&v)[8]) {
+  if ((reinterpret_cast<uintptr_t>(p) & 15u) == 0) {
+    const uint4 a = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      v[2 * q] = bf16_f32((uint16_t)(w[q] & 0xffffu));
+      v[2 * q + 1] = bf16_f32((uint16_t)(w[q] >> 16));
+    }
+  } else {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) v[q] = bf16_f32(p[q]);
+  }
+}
+
 namespace scl {
-constexpr int kCtas = 8;                                    // CTAs per cluster, one cluster per worker
-constexpr int kThreadsC = 512;
+// Four CTAs of 1024 threads per worker: clusters of eight CTAs left the
+// sixteenth worker's cluster waiting for a second wave at K = 16 (only
+// fifteen were co-resident on GB300), which doubled the sample's time
+constexpr int kCtas = 4;                                    // CTAs per cluster, one cluster per worker
+constexpr int kThreadsC = 1024;
 constexpr int kSlots = kSampleSlots / (kCtas * kThreadsC);  // sampled slots per thread
 static_assert(kSlots * kCtas * kThreadsC == kSampleSlots, "the cluster covers the whole sample");
+static_assert(kSlots == 8 && kSampleRun % kSlots == 0,
+              "a thread's slots are 8 consecutive coordinates of one sampled run (load8)");
 static_assert(kHistBins % kThreadsC == 0 && 1024 % kThreadsC == 0, "histograms split evenly over a block");
 }  // namespace scl
 
@@ -398,38 +478,54 @@ __global__ void __cluster_dims__(scl::kCtas, 1, 1) __launch_bounds__(scl::kThrea
   const float* gk = A.grads + (int64_t)k * A.d;
   const uint16_t* gk16 = A.grads16 + (int64_t)k * A.d;
   const int n_s = (int)A.n_sample;  // at most kSampleSlots
-  const int i_lo = (int)crank * (kSlots * kThreadsC);
-  // every load of every slot is issued before any value is used (no load
-  // waits on another), then v is formed as if the previous step's
-  // aggregation were applied at j
+  // this thread's slots: kSlots consecutive coordinates j0 .. j0 + 7 of one
+  // run (every coordinate when the sample is the whole vector), read with 16-byte
+  // loads where the rows allow; every load is issued before any value is
+  // used, then v is formed as if the previous step's aggregation were applied
+  const int i0 = ((int)crank * kThreadsC + (int)threadIdx.x) * kSlots;
+  const int nv = max(0, min(kSlots, n_s - i0));  // valid slots
   float ev[kSlots], gv[kSlots], dv[kSlots], lv[kSlots];
   uint32_t pm[kSlots], pd[kSlots];
 #pragma unroll
   for (int q = 0; q < kSlots; ++q) {
-    const int i = i_lo + q * kThreadsC + threadIdx.x;
     ev[q] = gv[q] = dv[q] = lv[q] = 0.f;
     pm[q] = pd[q] = 0u;
-    if (i < n_s) {
-      const int64_t j = sample_coord(A, 0ull, i);
-      ev[q] = ek[j];
-      gv[q] = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
-      dv[q] = A.dlt[j];
-      if (A.local_mom) lv[q] = A.lm[(int64_t)k * A.ld + j];
-      if (A.pending) {
-        pm[q] = A.sample_pend[i];
-        pd[q] = A.sample_pend[A.sample_stride + i];
+  }
+  if (nv == kSlots) {
+    const int64_t j0 = sample_coord(A, 0ull, i0);  // a multiple of kSlots (runs start on kSampleRun)
+    load8(ek + j0, ev);  // rows of e, lm and dlt start on 16 bytes (ld: whole tiles)
+    load8(A.dlt + j0, dv);
+    if (A.local_mom) load8(A.lm + (int64_t)k * A.ld + j0, lv);
+    if (A.bf16) load8_bf16(gk16 + j0, gv);
+    else load8(gk + j0, gv);  // a row of g starts on 4 bytes: 16-byte loads only where aligned
+    if (A.pending) {
+      load8u(A.sample_pend + i0, pm);
+      load8u(A.sample_pend + A.sample_stride + i0, pd);
+    }
+  } else {
+#pragma unroll
+    for (int q = 0; q < kSlots; ++q) {
+      if (q < nv) {
+        const int64_t j = sample_coord(A, 0ull, i0 + q);
+        ev[q] = ek[j];
+        gv[q] = A.bf16 ? bf16_f32(gk16[j]) : gk[j];
+        dv[q] = A.dlt[j];
+        if (A.local_mom) lv[q] = A.lm[(int64_t)k * A.ld + j];
+        if (A.pending) {
+          pm[q] = A.sample_pend[i0 + q];
+          pd[q] = A.sample_pend[A.sample_stride + i0 + q];
+        }
       }
     }
   }
   uint32_t key[kSlots];
 #pragma unroll
   for (int q = 0; q < kSlots; ++q) {
-    const int i = i_lo + q * kThreadsC + threadIdx.x;
     const float g = A.local_mom ? __fadd_rn(__fmul_rn(A.beta, lv[q]), __fmul_rn(A.gs, gv[q]))
                                 : (A.gscale ? __fmul_rn(A.gs, gv[q]) : gv[q]);
     const float e = ((pm[q] >> k) & 1u) ? 0.f : ev[q];
     const float dl = pm[q] ? __uint_as_float(pd[q]) : dv[q];
-    key[q] = i < n_s ? mag_key(accumulate(e, g, A.c, dl)) : 0xffffffffu;
+    key[q] = q < nv ? mag_key(accumulate(e, g, A.c, dl)) : 0xffffffffu;
     // plain shared-memory atomics: a warp's keys spread over a few dozen bins,
     // and the warp-aggregated form (match_any) measured slower here
     if (key[q] != 0xffffffffu) atomicAdd(&hist[key[q] >> 20], 1u);
@@ -1557,13 +1653,15 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   auto collect = [&](const uint32_t (&slot)[kQ], const bool (&in)[kQ]) {
     uint32_t key[kQ], idx[kQ], m[kQ], n = 0;
 #pragma unroll
-    for (int q = 0; q < kQ; ++q) {
-      key[q] = in[q] ? mag_key(cv[slot[q]]) : 0u;
-      idx[q] = in[q] ? ci[slot[q]] : 0u;
-    }
+    for (int q = 0; q < kQ; ++q) key[q] = in[q] ? mag_key(cv[slot[q]]) : 0u;
+    // the index only of a candidate in the k-th key's bin (about 2,048 of a
+    // worker's candidates), loaded while the bucket is reserved: about half
+    // the bytes of loading every candidate's index
 #pragma unroll
     for (int q = 0; q < kQ; ++q) {
-      m[q] = __ballot_sync(0xffffffffu, in[q] && rel_bin(key[q], theta, A.sel_shift) == want);
+      const bool mine = in[q] && rel_bin(key[q], theta, A.sel_shift) == want;
+      idx[q] = mine ? ci[slot[q]] : 0u;
+      m[q] = __ballot_sync(0xffffffffu, mine);
       n += __popc(m[q]);
     }
     if (n) {
@@ -1657,7 +1755,13 @@ __global__ void __launch_bounds__(kThreads) k_select_finish(TopkArgs A) {
   for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) keys[i] = __ldcg(&bk[i]);
   __syncthreads();
   uint32_t n_tie;
-  const uint32_t T = smem_select(keys, n, want_rank, h, ws, &s_bin, &s_rank, &n_tie);
+  // every key of the bucket lies in the bin `want`: below the top bin its
+  // keys are theta + want * 2^s + [0, 2^s), and only those low s bits are ranked
+  const bool bounded = want < kRelBins - 1;
+  const uint32_t T = bounded ? smem_select_bits(keys, n, want_rank, A.sel_shift,
+                                                theta + ((uint32_t)want << A.sel_shift), h, ws, &s_bin,
+                                                &s_rank, &n_tie)
+                             : smem_select(keys, n, want_rank, h, ws, &s_bin, &s_rank, &n_tie);
   // ties: gather the indices of the keys equal to T over the keys, in place;
   // a round writes below the end of what the block has read so far
   if (threadIdx.x == 0) s_n = 0;

@@ -266,6 +266,11 @@ class GMC:
         _check(self.lib.gmc_profile_kernels(self.h, mask), "gmc_profile_kernels")
         _check(self.lib.gmc_profile_enable(self.h, int(on)), "gmc_profile_enable")
 
+    def profile_mask(self, kernels=None) -> None:
+        """Choose the launches bracketed while profiling is on (all, or the named ones)."""
+        mask = 0xFFFFFFFF if kernels is None else sum(1 << KERNELS.index(k) for k in kernels)
+        _check(self.lib.gmc_profile_kernels(self.h, mask), "gmc_profile_kernels")
+
     def profile_read(self) -> dict:
         out = {}
         for i, name in enumerate(KERNELS):
