@@ -158,15 +158,18 @@ def test_bulk_pass_reports_non_finite_values():
     assert p.gpu.check() == 4  # GMC_ENONFINITE
 
 
-@pytest.mark.parametrize("K", [1, 2, 5, 6, 7, 16])
-def test_claimed_tiles_and_odd_worker_counts(K):
+@pytest.mark.parametrize("K,tail", [(1, 1001), (2, 1001), (5, 1001), (6, 1001), (7, 1001), (16, 1001),
+                                    (6, 3001)])
+def test_claimed_tiles_and_odd_worker_counts(K, tail):
     """Several tiles per CTA beyond its fixed ones, so the bulk pass claims
     the rest from its tile counter; the worker-parity warp groups each read
     their own stages of the ring, in order, for every K (odd K gives the two
     groups different item counts per tile, K = 1 leaves one group without
     items). K <= 5 runs the three-tile pipeline of w_t - w_{t-1}, K >= 6 the
-    one-tile pipeline with two tiles claimed ahead."""
-    d = 152 * 4096 * 9 + 1001  # about nine tiles per CTA
+    one-tile pipeline with two tiles claimed ahead. The ragged last tile's
+    last four sub-tiles lie past d (tail 1001) or hold its last 953
+    coordinates (tail 3001)."""
+    d = 152 * 4096 * 9 + tail  # about nine tiles per CTA
     rng = np.random.default_rng(40 + K)
     p = Pair(d, K, 0.9, 0.1, ratio=0.001, seed=9, ref="cpp")
     for t in range(3):
