@@ -12,8 +12,8 @@ RBGS blocks), each measured in the same invocation.
 ``e2e`` is the same metric through the host-memory entry point (host->device
 copy of the step's gradients and device->host read of the step's counters
 inside the timed region). ``roofline`` reports the dominant kernel's
-algorithmic bytes per launch over its CUDA-event duration against the measured
-HBM copy peak. ``cpu_baseline`` times the oracle on the host cores on a bounded
+algorithmic bytes per launch over its CUDA-event duration (events around it on
+every EVENTS_EVERY-th timed step) against the measured HBM copy peak. ``cpu_baseline`` times the oracle on the host cores on a bounded
 sample of the same workload.
 
 Multi-GPU: the step does not shard (K workers are simulated on one GPU), so
